@@ -1,0 +1,182 @@
+"""CPU oracle for the additive-codebook dequantize-and-multiply (test infrastructure only).
+
+Only the tests, the smoke check and the CPU-baseline leg of the benchmark may import this
+package. It wraps oracle.cpp (ctypes, numpy arrays in and out) and shares nothing with the
+CUDA library. See oracle.cpp for the paper passages each function follows.
+"""
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+DT_F16, DT_BF16 = 0, 1
+_DT = {"f16": DT_F16, "bf16": DT_BF16}
+
+_lib = None
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        # ORACLE_LIB points at another build of oracle.cpp (the mutation tests use it).
+        path = os.environ.get("ORACLE_LIB") or _build.build()
+        L = ctypes.CDLL(path)
+        vp, i32, u16p = ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p
+        L.oracle_avg_bits.restype = ctypes.c_double
+        L.oracle_avg_bits.argtypes = [ctypes.c_long, ctypes.c_long, i32, i32, i32]
+        L.oracle_prefix_code_bits.restype = ctypes.c_double
+        L.oracle_prefix_code_bits.argtypes = [i32, i32, i32]
+        L.oracle_decode.restype = i32
+        L.oracle_decode.argtypes = [i32] * 6 + [vp, u16p, i32, u16p, i32, u16p]
+        L.oracle_product_exact.restype = i32
+        L.oracle_product_exact.argtypes = [i32] * 6 + [vp, u16p, i32, u16p, i32, u16p, i32, i32, vp]
+        L.oracle_product_dense.restype = i32
+        L.oracle_product_dense.argtypes = [i32, i32, u16p, i32, u16p, i32, i32, vp]
+        L.oracle_pack.restype = i32
+        L.oracle_pack.argtypes = [i32] * 5 + [vp, vp]
+        L.oracle_f32_to_f16.restype = ctypes.c_uint16
+        L.oracle_f32_to_f16.argtypes = [ctypes.c_float]
+        L.oracle_f32_to_bf16.restype = ctypes.c_uint16
+        L.oracle_f32_to_bf16.argtypes = [ctypes.c_float]
+        L.oracle_f16_to_f64.restype = ctypes.c_double
+        L.oracle_f16_to_f64.argtypes = [ctypes.c_uint16]
+        L.oracle_bf16_to_f64.restype = ctypes.c_double
+        L.oracle_bf16_to_f64.argtypes = [ctypes.c_uint16]
+        L.oracle_f32_to_bits_array.restype = None
+        L.oracle_f32_to_bits_array.argtypes = [vp, vp, ctypes.c_long, i32]
+        L.oracle_bits_to_f64_array.restype = None
+        L.oracle_bits_to_f64_array.argtypes = [vp, vp, ctypes.c_long, i32]
+        L.oracle_num_threads.restype = i32
+        L.oracle_num_threads.argtypes = []
+        _lib = L
+    return _lib
+
+
+def _p(a):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _codes_ok(codes, B):
+    want = np.uint8 if B <= 8 else np.uint16
+    if codes.dtype != want or not codes.flags.c_contiguous:
+        raise TypeError("codes must be C-contiguous %s for B=%d" % (np.dtype(want).name, B))
+
+
+def avg_bits(d_out, d_in, g, M, B):
+    """App. C, Eq. avg_bits (codes term times M)."""
+    return lib().oracle_avg_bits(d_out, d_in, g, M, B)
+
+
+def prefix_code_bits(g, m, B):
+    return lib().oracle_prefix_code_bits(g, m, B)
+
+
+def decode(layer, m):
+    """Bit patterns [out][in] (uint16) of the book dtype: s[o]*sum_{k<m} C_k[b], fp32, one RNE."""
+    out, inp, G, M, B = layer["out"], layer["in"], layer["G"], layer["M"], layer["B"]
+    codes = layer["codes"]
+    _codes_ok(codes, B)
+    w = np.empty((out, inp), dtype=np.uint16)
+    rc = lib().oracle_decode(out, inp, G, M, B, m, _p(codes), _p(layer["books"]),
+                             _DT[layer["book_dtype"]], _p(layer["scales"]),
+                             _DT[layer["scale_dtype"]], _p(w))
+    if rc:
+        raise ValueError("oracle_decode rejected the shape")
+    return w
+
+
+def product_exact(layer, x, x_dtype, m, rows=None):
+    """fp64 y[t,o] = sum_i x[t,i] * (s[o]*sum_{k<m} C_k[b_{o,g,k}][e]) for t < batch.
+
+    rows: optional (r0, r1) to evaluate only output rows r0..r1-1 (a bounded sample).
+    """
+    out, inp, G, M, B = layer["out"], layer["in"], layer["G"], layer["M"], layer["B"]
+    codes, scales = layer["codes"], layer["scales"]
+    _codes_ok(codes, B)
+    if rows is not None:
+        r0, r1 = rows
+        codes = np.ascontiguousarray(codes[r0:r1])
+        scales = np.ascontiguousarray(scales[r0:r1])
+        out = r1 - r0
+    x = np.ascontiguousarray(x, dtype=np.uint16).reshape(-1, inp)
+    batch = x.shape[0]
+    y = np.empty((batch, out), dtype=np.float64)
+    rc = lib().oracle_product_exact(out, inp, G, M, B, m, _p(codes), _p(layer["books"]),
+                                    _DT[layer["book_dtype"]], _p(scales),
+                                    _DT[layer["scale_dtype"]], _p(x), _DT[x_dtype], batch, _p(y))
+    if rc:
+        raise ValueError("oracle_product_exact rejected the shape")
+    return y
+
+
+def product_dense(w_bits, w_dtype, x, x_dtype):
+    w_bits = np.ascontiguousarray(w_bits, dtype=np.uint16)
+    out, inp = w_bits.shape
+    x = np.ascontiguousarray(x, dtype=np.uint16).reshape(-1, inp)
+    y = np.empty((x.shape[0], out), dtype=np.float64)
+    rc = lib().oracle_product_dense(out, inp, _p(w_bits), _DT[w_dtype], _p(x), _DT[x_dtype],
+                                    x.shape[0], _p(y))
+    if rc:
+        raise ValueError("oracle_product_dense rejected the shape")
+    return y
+
+
+def pack(layer):
+    """Packed code planes (see oracle.cpp for the index map) as a flat uint8 array."""
+    out, inp, G, M, B = layer["out"], layer["in"], layer["G"], layer["M"], layer["B"]
+    codes = layer["codes"]
+    _codes_ok(codes, B)
+    rows_pad = (out + 31) // 32 * 32
+    ng_pad = (inp // G + 31) // 32 * 32
+    esz = 1 if B <= 8 else 2
+    buf = np.zeros(M * rows_pad * ng_pad * esz, dtype=np.uint8)
+    rc = lib().oracle_pack(out, inp, G, M, B, _p(codes), _p(buf))
+    if rc:
+        raise ValueError("oracle_pack rejected the shape")
+    return buf
+
+
+def f32_to_f16(v):
+    return lib().oracle_f32_to_f16(float(v))
+
+
+def f32_to_bf16(v):
+    return lib().oracle_f32_to_bf16(float(v))
+
+
+def f16_to_f64(h):
+    return lib().oracle_f16_to_f64(int(h))
+
+
+def bf16_to_f64(b):
+    return lib().oracle_bf16_to_f64(int(b))
+
+
+def round_bits(a, dtype):
+    """float32 array -> fp16/bf16 bit patterns with the oracle's own round-to-nearest-even."""
+    a = np.ascontiguousarray(a, dtype=np.float32)
+    out = np.empty(a.shape, dtype=np.uint16)
+    lib().oracle_f32_to_bits_array(_p(a), _p(out), a.size, _DT[dtype])
+    return out
+
+
+def bits_value(v, dtype):
+    """fp16/bf16 bit patterns -> float64 values with the oracle's own widening."""
+    v = np.ascontiguousarray(v, dtype=np.uint16)
+    out = np.empty(v.shape, dtype=np.float64)
+    lib().oracle_bits_to_f64_array(_p(v), _p(out), v.size, _DT[dtype])
+    return out
+
+
+def num_threads():
+    return lib().oracle_num_threads()
+
+
+def widen(bits, dtype):
+    """Exact widening of fp16/bf16 bit patterns to float64 (numpy, vectorised)."""
+    bits = np.asarray(bits, dtype=np.uint16)
+    if dtype == "f16":
+        return bits.view(np.float16).astype(np.float64)
+    return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)

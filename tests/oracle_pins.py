@@ -1,0 +1,343 @@
+"""Pins of the CPU oracle to facts that do not come from the oracle itself.
+
+Each pin_* function raises AssertionError when the oracle (the `oracle` package, possibly
+loaded from another build via ORACLE_LIB) disagrees with:
+  * a value the paper prints (App. C worked example of Eq. avg_bits),
+  * an independent library routine (numpy float16 / torch bfloat16 rounding),
+  * brute force in the paper's own notation (one-hot code vectors times C_m, Sec. 3.2 / Sec. 5),
+  * exact rational arithmetic (fractions.Fraction) on dyadic inputs,
+  * closed forms of special cases, or invariants (prefix linearity, prefix packing).
+The same functions run under pytest (test_oracle_pins.py) and against deliberately broken
+builds of the oracle (test_oracle_mutants.py), which must each fail at least one pin.
+"""
+import os
+from fractions import Fraction
+
+import numpy as np
+import torch
+
+import oracle
+import workloads
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def _rng(seed):
+    return np.random.Generator(np.random.PCG64(seed))
+
+
+# ---------------------------------------------------------------- storage model (App. C)
+
+def pin_avg_bits_paper_example():
+    """App. C: the 70B gate projection with g=8, M=2, B=8 costs approximately 2.002 bits."""
+    with open(os.path.join(GOLDEN, "avg_bits_70b_gate_proj.txt")) as f:
+        rows = [l.split() for l in f if l.strip() and not l.startswith("#")]
+    for d_out, d_in, g, M, B, printed, decimals in rows:
+        v = oracle.avg_bits(int(d_out), int(d_in), int(g), int(M), int(B))
+        assert round(v, int(decimals)) == float(printed), (v, printed)
+
+
+def pin_avg_bits_limit():
+    """For huge layers the codebook and scale terms vanish: avg bits -> M*B/g (closed form)."""
+    for (g, M, B) in [(8, 2, 8), (8, 4, 8), (8, 2, 16), (16, 3, 8)]:
+        v = oracle.avg_bits(1 << 22, 1 << 22, g, M, B)
+        assert abs(v - M * B / g) < 1e-3, (g, M, B, v)
+        assert oracle.prefix_code_bits(g, M, B) == M * B / g
+
+
+# ---------------------------------------------------------------- number formats
+
+def _special_f32():
+    vals = [0.0, -0.0, 1.0, -1.0, 65504.0, 65519.99, 65520.0, 1e6, -1e6, 6.1035156e-05,
+            5.9604645e-08, 2.9802322e-08, 2.9802326e-08, 8.940697e-08, 1e-40, -1e-45,
+            float("inf"), float("-inf"), 3.0e38, 3.4028235e38]
+    # exact binary16 ties: midpoints between neighbouring fp16 values
+    h = np.arange(0, 0x7c00, 97, dtype=np.uint16).view(np.float16).astype(np.float64)
+    mids = (h[:-1] + np.nextafter(h[:-1].astype(np.float16), np.float16(np.inf)).astype(np.float64)) / 2
+    return np.concatenate([np.array(vals, dtype=np.float64), mids, -mids]).astype(np.float32)
+
+
+def pin_f16_rounding_matches_numpy():
+    """float32 -> binary16 RNE against numpy's independent implementation."""
+    rng = _rng(11)
+    bits = rng.integers(0, 2**32, size=200000, dtype=np.uint64).astype(np.uint32)
+    x = bits.view(np.float32)
+    x = x[np.isfinite(x)]
+    x = np.concatenate([x, _special_f32(), (rng.standard_normal(50000) * 1e-5).astype(np.float32)])
+    got = oracle.round_bits(x, "f16")
+    want = x.astype(np.float16).view(np.uint16)
+    assert np.array_equal(got, want), np.flatnonzero(got != want)[:10]
+
+
+def pin_bf16_rounding_matches_torch():
+    """float32 -> bfloat16 RNE against torch's independent implementation."""
+    rng = _rng(12)
+    bits = rng.integers(0, 2**32, size=200000, dtype=np.uint64).astype(np.uint32)
+    x = bits.view(np.float32)
+    x = x[np.isfinite(x)]
+    ties = (rng.integers(0, 2**16, size=5000, dtype=np.uint32) << 16 | 0x8000).view(np.float32)
+    x = np.concatenate([x, _special_f32(), ties[np.isfinite(ties)]])
+    got = oracle.round_bits(x, "bf16")
+    want = torch.from_numpy(x.copy()).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(got, want), np.flatnonzero(got != want)[:10]
+
+
+def pin_widening_matches_numpy():
+    """Every binary16 bit pattern widens to numpy's value (NaNs compared as NaN)."""
+    allh = np.arange(0, 1 << 16, dtype=np.uint32).astype(np.uint16)
+    got = oracle.bits_value(allh, "f16")
+    want = allh.view(np.float16).astype(np.float64)
+    same = (got == want) | (np.isnan(got) & np.isnan(want))
+    assert same.all()
+    b = np.arange(0, 1 << 16, 7, dtype=np.uint32).astype(np.uint16)
+    got = oracle.bits_value(b, "bf16")
+    want = torch.from_numpy(b.view(np.int16).copy()).view(torch.bfloat16).double().numpy()
+    same = (got == want) | (np.isnan(got) & np.isnan(want))
+    assert same.all()
+
+
+# ---------------------------------------------------------------- reconstruction (Sec. 3.2, Sec. 5)
+
+def _onehot_reconstruction(layer, m):
+    """Brute force in the paper's notation: C_k is a g x 2^B matrix, b_{i,j,k} a one-hot
+    vector in {0,1}^{2^B}; group j of row i is sum_{k<m} C_k b_{i,j,k}; the row is the
+    concatenation of its groups; the scale multiplies the row (reading R1). fp64, exact."""
+    out, inp, G, M, B = layer["out"], layer["in"], layer["G"], layer["M"], layer["B"]
+    nb = 1 << B
+    books = workloads_values(layer["books"], layer["book_dtype"]).reshape(M, nb, G)
+    C = [books[k].T.copy() for k in range(M)]          # g x 2^B, column j = codeword j
+    s = workloads_values(layer["scales"], layer["scale_dtype"])
+    W = np.zeros((out, inp))
+    for i in range(out):
+        parts = []
+        for j in range(inp // G):
+            acc = np.zeros(G)
+            for k in range(m):
+                onehot = np.zeros(nb)
+                onehot[int(layer["codes"][i, j, k])] = 1.0
+                acc = acc + C[k] @ onehot
+            parts.append(acc)
+        W[i] = s[i] * np.concatenate(parts)
+    return W
+
+
+def workloads_values(bits, dtype):
+    """Exact float64 values of bit patterns, via numpy / torch (not via the oracle)."""
+    bits = np.asarray(bits, dtype=np.uint16)
+    if dtype == "f16":
+        return bits.view(np.float16).astype(np.float64)
+    return torch.from_numpy(bits.view(np.int16).copy()).view(torch.bfloat16).double().numpy()
+
+
+def _tiny_layers():
+    shapes = [(1, 8, 1, 8), (3, 16, 2, 8), (8, 24, 4, 8), (5, 8, 3, 16), (33, 40, 2, 8)]
+    for idx, (out, inp, M, B) in enumerate(shapes):
+        for bd in ("f16", "bf16"):
+            yield workloads.make_layer(out, inp, G=8, M=M, B=B, book_dtype=bd, book_std=0.3,
+                                       scale_dtype=bd, seed=100 + idx)
+
+
+def pin_product_matches_onehot_bruteforce():
+    """oracle_product_exact == x @ W^T with W from one-hot matrix products (fp64)."""
+    for layer in _tiny_layers():
+        x = workloads.make_x(3, layer["in"], "f16", seed=7)
+        xv = x.view(np.float16).astype(np.float64)
+        for m in range(1, layer["M"] + 1):
+            W = _onehot_reconstruction(layer, m)
+            want = xv @ W.T
+            got = oracle.product_exact(layer, x, "f16", m)
+            assert np.allclose(got, want, rtol=1e-12, atol=1e-12), (m, np.abs(got - want).max())
+
+
+def pin_decode_matches_onehot_within_rounding():
+    """oracle_decode == RNE(W) up to the fp32 summation error: at most one unit in the last
+    place of the book format away from the exactly rounded one-hot reconstruction."""
+    for layer in _tiny_layers():
+        dt = layer["book_dtype"]
+        for m in range(1, layer["M"] + 1):
+            W = _onehot_reconstruction(layer, m)
+            got = workloads_values(oracle.decode(layer, m), dt)
+            if dt == "f16":
+                ref = W.astype(np.float32).astype(np.float16).astype(np.float64)
+                ulp = np.spacing(np.abs(ref).astype(np.float16)).astype(np.float64)
+            else:
+                ref = workloads_values(workloads.to_bits(W.astype(np.float32), "bf16"), "bf16")
+                ulp = np.abs(ref) * 2.0 ** -7 + 2.0 ** -133
+            assert np.all(np.abs(got - ref) <= ulp * 1.0001), (m, dt)
+
+
+def pin_decode_exact_dyadic():
+    """Dyadic inputs (multiples of 2^-10 in (-1,1), power-of-two scales): every fp32 step is
+    exact, so decode must equal numpy's RNE of the exact one-hot reconstruction, bit for bit."""
+    rng = _rng(5)
+    for (out, inp, M) in [(7, 32, 4), (32, 64, 3)]:
+        for dt in ("f16", "bf16"):
+            layer = workloads.make_layer(out, inp, G=8, M=M, B=8, book_dtype=dt, scale_dtype=dt,
+                                         seed=out)
+            vals = rng.integers(-1023, 1024, size=layer["books"].shape) / 1024.0
+            layer["books"] = workloads.to_bits(vals.astype(np.float32), dt)
+            layer["scales"] = workloads.to_bits(
+                2.0 ** rng.integers(-3, 4, size=out).astype(np.float32), dt)
+            for m in range(1, M + 1):
+                W = _onehot_reconstruction(layer, m)
+                want = workloads.to_bits(W.astype(np.float32), dt)
+                assert np.array_equal(oracle.decode(layer, m), want), (out, dt, m)
+
+
+def pin_product_exact_rational():
+    """Dyadic books, small-integer activations, unit scales: the fp64 product is exact, so it
+    must equal the rational sum computed with Python Fractions."""
+    rng = _rng(6)
+    layer = workloads.make_layer(5, 24, G=8, M=3, B=8, book_dtype="f16", scale_dtype="f16", seed=9)
+    vals = rng.integers(-1023, 1024, size=layer["books"].shape)
+    layer["books"] = workloads.to_bits((vals / 1024.0).astype(np.float32), "f16")
+    layer["scales"] = workloads.to_bits(np.ones(5, np.float32), "f16")
+    xi = rng.integers(-8, 9, size=(2, 24))
+    x = workloads.to_bits(xi.astype(np.float32), "f16")
+    for m in (1, 2, 3):
+        got = oracle.product_exact(layer, x, "f16", m)
+        for t in range(2):
+            for o in range(5):
+                tot = Fraction(0)
+                for g in range(3):
+                    for e in range(8):
+                        w = sum(Fraction(int(vals[k, layer["codes"][o, g, k], e]), 1024)
+                                for k in range(m))
+                        tot += Fraction(int(xi[t, g * 8 + e])) * w
+                assert Fraction(got[t, o]) == tot, (m, t, o)
+
+
+def pin_constant_codeword_closed_form():
+    """All codes 0 and C_k[0] = constant vector c_k: y[t,o] = s[o]*(sum_k c_k)*sum_i x[t,i]."""
+    rng = _rng(8)
+    layer = workloads.make_layer(6, 32, G=8, M=4, B=8, seed=3)
+    layer["codes"][:] = 0
+    books = layer["books"].reshape(4, 256, 8).copy()
+    c = workloads.to_bits(rng.standard_normal(4).astype(np.float32) * 0.1, "f16")
+    books[:, 0, :] = c[:, None]
+    layer["books"] = books
+    x = workloads.make_x(2, 32, "f16", seed=4)
+    xs = x.view(np.float16).astype(np.float64).sum(axis=1)
+    s = layer["scales"].view(np.float16).astype(np.float64)
+    cv = c.view(np.float16).astype(np.float64)
+    for m in range(1, 5):
+        want = np.outer(xs, s * cv[:m].sum())
+        got = oracle.product_exact(layer, x, "f16", m)
+        assert np.allclose(got, want, rtol=1e-12, atol=1e-13), m
+
+
+def pin_onehot_codebook_selection():
+    """One book whose codeword j is the unit vector e_(j mod 8): W is a scaled selection
+    matrix, y[t,o] = s[o] * sum_g x[t, 8g + (b[o,g] mod 8)]."""
+    layer = workloads.make_layer(9, 40, G=8, M=1, B=8, seed=12)
+    books = np.zeros((1, 256, 8), np.float32)
+    books[0, np.arange(256), np.arange(256) % 8] = 1.0
+    layer["books"] = workloads.to_bits(books, "f16")
+    x = workloads.make_x(3, 40, "f16", seed=5)
+    xv = x.view(np.float16).astype(np.float64)
+    s = layer["scales"].view(np.float16).astype(np.float64)
+    got = oracle.product_exact(layer, x, "f16", 1)
+    for t in range(3):
+        for o in range(9):
+            want = s[o] * sum(xv[t, 8 * g + int(layer["codes"][o, g, 0]) % 8] for g in range(5))
+            assert abs(got[t, o] - want) <= 1e-12 * (1 + abs(want))
+
+
+def pin_prefix_linearity():
+    """Successive refinement (the nested increments of Sec. 4 / App. E): y_m - y_{m-1} equals
+    the product with book m-1 alone (scaled by s), for every m."""
+    for layer in _tiny_layers():
+        x = workloads.make_x(2, layer["in"], "f16", seed=3)
+        ys = [oracle.product_exact(layer, x, "f16", m) for m in range(1, layer["M"] + 1)]
+        for m in range(2, layer["M"] + 1):
+            single = dict(layer)
+            single["M"] = 1
+            nb = 1 << layer["B"]
+            single["books"] = np.ascontiguousarray(
+                layer["books"].reshape(layer["M"], nb, layer["G"])[m - 1])
+            single["codes"] = np.ascontiguousarray(layer["codes"][:, :, m - 1:m])
+            inc = oracle.product_exact(single, x, "f16", 1)
+            scale = 1 + np.abs(ys[m - 1]).max()
+            assert np.allclose(ys[m - 1] - ys[m - 2], inc, rtol=0, atol=1e-12 * scale), m
+
+
+def pin_full_prefix_uses_every_book():
+    """m = M reconstructs with all books: changing any single book changes y at m = M, and
+    changing book M-1 leaves every m < M untouched."""
+    layer = workloads.make_layer(4, 16, G=8, M=3, B=8, book_std=0.2, seed=21)
+    x = workloads.make_x(1, 16, "f16", seed=2)
+    base = [oracle.product_exact(layer, x, "f16", m) for m in (1, 2, 3)]
+    for k in range(3):
+        alt = dict(layer)
+        books = layer["books"].reshape(3, 256, 8).copy()
+        books[k] = workloads.to_bits(np.full((256, 8), 0.5, np.float32), "f16")
+        alt["books"] = books
+        ys = [oracle.product_exact(alt, x, "f16", m) for m in (1, 2, 3)]
+        assert not np.allclose(ys[2], base[2])
+        for m in range(1, 4):
+            if m <= k:
+                assert np.array_equal(ys[m - 1], base[m - 1]), (k, m)
+
+
+def pin_dense_product_of_decode():
+    """product_dense(decode) stays within the book-format rounding of product_exact."""
+    layer = workloads.make_layer(16, 64, G=8, M=2, B=8, book_std=0.1, seed=31)
+    x = workloads.make_x(2, 64, "f16", seed=8)
+    for m in (1, 2):
+        a = oracle.product_exact(layer, x, "f16", m)
+        b = oracle.product_dense(oracle.decode(layer, m), "f16", x, "f16")
+        bound = np.abs(x.view(np.float16).astype(np.float64)).sum(axis=1, keepdims=True) * 0.1 * 4 * 2.0 ** -10
+        assert np.all(np.abs(a - b) <= bound + 1e-12), m
+
+
+# ---------------------------------------------------------------- packed planes
+
+def pin_pack_positions():
+    """Codes that spell their own coordinates: position p of row o in slice s must hold the
+    code of group s*32 + (p+o) mod 32 of plane k; padding holds 0."""
+    out, ng, M = 37, 70, 3
+    inp = ng * 8
+    codes = np.zeros((out, ng, M), np.uint16)
+    for o in range(out):
+        for g in range(ng):
+            for k in range(M):
+                codes[o, g, k] = 1 + g + 100 * k     # unique per (g, k), never 0
+    layer = dict(out=out, **{"in": inp}, G=8, M=M, B=16, codes=codes)
+    planes = oracle.pack(layer).view(np.uint16)
+    rows_pad, ng_pad = 64, 96
+    planes = planes.reshape(M, ng_pad // 32, rows_pad, 32)
+    for k in range(M):
+        for s in range(ng_pad // 32):
+            for o in range(rows_pad):
+                for p in range(32):
+                    g = s * 32 + (p + o) % 32
+                    want = (1 + g + 100 * k) if (o < out and g < ng) else 0
+                    assert planes[k, s, o, p] == want
+
+
+def pin_pack_prefix_property():
+    """The first m planes of a packed M-book layer equal the packed m-book truncation."""
+    layer = workloads.make_layer(40, 272, G=8, M=4, B=8, seed=2)
+    full = oracle.pack(layer)
+    for m in (1, 2, 3):
+        trunc = dict(layer)
+        trunc["M"] = m
+        trunc["codes"] = np.ascontiguousarray(layer["codes"][:, :, :m])
+        p = oracle.pack(trunc)
+        assert np.array_equal(full[: p.size], p), m
+
+
+ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]
+
+
+if __name__ == "__main__":
+    # Used by the mutation tests: run every pin, print the failing ones, exit 1 if any fail.
+    import sys
+    failed = []
+    for fn in ALL_PINS:
+        try:
+            fn()
+        except Exception as exc:  # noqa: BLE001 - any failure counts as a caught mutant
+            failed.append("%s: %s" % (fn.__name__, type(exc).__name__))
+    print("\n".join(failed) if failed else "all pins passed")
+    sys.exit(1 if failed else 0)
