@@ -1,0 +1,335 @@
+#!/usr/bin/env python
+"""Benchmark of the additive-codebook dequantize-and-multiply hot path on GB300.
+
+Workload (default): a Llama-style 4096 x 4096 attention projection stored with M = 4
+codebooks of 2^8 fp16 codewords (g = 8, uint8 codes), evaluated at batch 1 for every prefix
+m = 1..4 (1..4 bits per weight). One step = the four GEMVs m = 1, 2, 3, 4 on one weight copy.
+Weight copies rotate so the timed reads come from HBM, not L2 (copies x packed bytes >= 3x L2).
+
+Prints one JSON line. `value` is the achieved algorithmic HBM bandwidth of the whole step,
+sum over m of bytes(m) / step time, with bytes(m) = codes m*out*(in/8) + books m*2^8*8*2 +
+scales 2*out + x 2*in + y 2*out. Per-m times come from CUDA events around each launch inside
+the timed CUDA graph.
+
+--impl reference times the CPU oracle (the plain C++ statement of the same product) on the
+host cores, on a bounded row sample of the same workload, with the same metric.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "batch-1 GEMV µs & achieved HBM GB/s per prefix m (bits/wt); prefill GEMM TFLOP/s"
+WORKLOAD = "attn_4096"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="own", choices=["own", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def layer_bytes(out, inp, m, B=8, G=8, batch=1, xsize=2, ysize=2):
+    """Algorithmic bytes of one prefix-m call: codes, first m books, scales, x, y."""
+    return (m * out * (inp // G) * (B // 8) + m * (1 << B) * G * 2 + 2 * out
+            + batch * inp * xsize + batch * out * ysize)
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.dev = device_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.dev), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        self.proc.wait()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 8:
+                rows.append(parts)
+        os.unlink(self.path)
+        sm = [float(r[0]) for r in rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[4 + i] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+def cpu_oracle_rate(layer, x_bits, ms, budget_s, rows=None):
+    """Time the oracle on (a row sample of) one step: returns (GB/s, seconds/step, steps)."""
+    import oracle
+    out = layer["out"] if rows is None else rows[1] - rows[0]
+    bytes_step = sum(layer_bytes(out, layer["in"], m) for m in ms)
+    n, t0 = 0, time.perf_counter()
+    while True:
+        for m in ms:
+            oracle.product_exact(layer, x_bits, "f16", m, rows=rows)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s:
+            break
+    return bytes_step * n / el / 1e9, el / n, n
+
+
+def reference_arm(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    import oracle
+    import workloads
+    (_, layer), = list(workloads.config_layers(WORKLOAD))
+    x_bits = workloads.config_x(WORKLOAD, 1, layer["in"])
+    ms = (1, 2, 3, 4)
+    # size the row sample so W + K steps take about a minute
+    t_full = cpu_oracle_rate(layer, x_bits, ms, 0.0)[1]
+    frac = min(1.0, 60.0 / max(1, args.steps + args.warmup) / max(t_full, 1e-6))
+    nrows = max(32, int(layer["out"] * frac) // 32 * 32)
+    rows = (0, nrows)
+    for _ in range(args.warmup):
+        for m in ms:
+            oracle.product_exact(layer, x_bits, "f16", m, rows=rows)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        for m in ms:
+            oracle.product_exact(layer, x_bits, "f16", m, rows=rows)
+    el = time.perf_counter() - t0
+    bytes_step = sum(layer_bytes(nrows, layer["in"], m) for m in ms)
+    value = bytes_step * args.steps / el / 1e9
+    sample = "rows 0..%d of the 4096x4096 layer, batch 1, m=1..4 per step" % nrows
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": el / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "GB/s", "cores": oracle.num_threads(),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def own_arm(args):
+    import numpy as np
+    import torch
+
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    import paper_2606_12876_gb300 as aq
+    from paper_2606_12876_gb300 import build as libbuild
+    from paper_2606_12876_gb300.linear import AQLinear, x_to_device
+    import workloads
+
+    libbuild.build()
+    ms = (1, 2, 3, 4)
+    (_, layer), = list(workloads.config_layers(WORKLOAD))
+    out, inp = layer["out"], layer["in"]
+    lin = AQLinear.from_layer(layer, device=dev)
+    L = lin.layout
+    x_bits = workloads.config_x(WORKLOAD, 1, inp)
+    x = x_to_device(x_bits, "f16", dev)
+    ys = {m: torch.empty(1, out, dtype=torch.float16, device=dev) for m in ms}
+    ws = aq.workspace(aq.gemv_workspace_bytes(L, 1), dev)
+
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    pbytes = aq.packed_bytes(L, 4)
+    ncopies = max(2, -(-3 * l2 // pbytes))
+    copies = [lin.planes.clone() for _ in range(ncopies)]
+    bytes_m = {m: layer_bytes(out, inp, m) for m in ms}
+    bytes_step = sum(bytes_m.values())
+
+    stream = torch.cuda.Stream(device=dev)
+
+    def step(i, events=None):
+        planes = copies[i % ncopies]
+        for m in ms:
+            if events is not None:
+                events[i][m][0].record()
+            aq.aq_gemv(L, m, planes, lin.books, lin.scales, x, aq.AQ_F16, 1, ys[m], aq.AQ_F16, ws)
+            if events is not None:
+                events[i][m][1].record()
+
+    with torch.cuda.stream(stream):
+        for i in range(3):                      # eager warm-up: sets kernel attributes
+            step(i)
+    torch.cuda.synchronize(dev)
+
+    try:
+        mk = lambda: torch.cuda.Event(enable_timing=True, external=True)  # noqa: E731
+        events = [{m: (mk(), mk()) for m in ms} for _ in range(args.steps)]
+    except TypeError:
+        events = None
+    g_warm, g_timed = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_warm, stream=stream):
+        for i in range(args.warmup):
+            step(i)
+    with torch.cuda.graph(g_timed, stream=stream):
+        for i in range(args.steps):
+            step(i, events)
+    torch.cuda.synchronize(dev)
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    g_warm.replay()
+    torch.cuda.synchronize(dev)
+    clocks = ClockSampler(local)
+    clocks.start()
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize(dev)
+    with torch.cuda.stream(stream):
+        t_start.record()
+        g_timed.replay()
+        t_end.record()
+    torch.cuda.synchronize(dev)
+    barrier()
+    clk = clocks.stop()
+    ms_total = t_start.elapsed_time(t_end)
+    if world > 1:
+        t = torch.tensor([ms_total], device=dev, dtype=torch.float64)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms_total = float(t.item())
+    ms_step = ms_total / args.steps
+    value = world * bytes_step * args.steps / (ms_total / 1e3) / 1e9
+
+    peaks = {}
+    ppath = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(ppath):
+        peaks = json.load(open(ppath))
+    hbm_peak = peaks.get("hbm_gbs", 6800.0)
+    peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
+
+    per_m = []
+    if events is not None:
+        for m in ms:
+            us = statistics.mean(events[i][m][0].elapsed_time(events[i][m][1])
+                                 for i in range(args.steps)) * 1e3
+            gbs = bytes_m[m] / (us * 1e-6) / 1e9
+            per_m.append({"m": m, "bits_per_weight": m, "us": round(us, 3),
+                          "GB_s": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4),
+                          "bytes": bytes_m[m]})
+    dom = max(per_m, key=lambda r: r["us"]) if per_m else None
+
+    # end to end through the public API: pinned host x -> device, 4 GEMVs, y -> pinned host
+    e2e = None
+    if not args.no_e2e:
+        x_host = torch.from_numpy(x_bits.view(np.int16)).view(torch.float16).pin_memory()
+        y_host = torch.empty(len(ms), out, dtype=torch.float16).pin_memory()
+        x_dev = torch.empty_like(x_host, device=dev)
+        e_s, e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n_e2e = max(20, args.steps // 2)
+        with torch.cuda.stream(stream):
+            for i in range(args.warmup + n_e2e):
+                if i == args.warmup:
+                    torch.cuda.synchronize(dev)
+                    e_s.record()
+                x_dev.copy_(x_host, non_blocking=True)
+                planes = copies[i % ncopies]
+                for j, m in enumerate(ms):
+                    aq.aq_gemv(L, m, planes, lin.books, lin.scales, x_dev, aq.AQ_F16, 1, ys[m],
+                               aq.AQ_F16, ws)
+                    y_host[j].copy_(ys[m][0], non_blocking=True)
+            e_e.record()
+        torch.cuda.synchronize(dev)
+        e2e_ms = e_s.elapsed_time(e_e) / n_e2e
+        e2e = {"value": world * bytes_step / (e2e_ms / 1e3) / 1e9, "unit": "GB/s",
+               "ms_per_step": e2e_ms, "h2d_bytes_per_step": x_host.numel() * 2,
+               "d2h_bytes_per_step": y_host.numel() * 2,
+               "api": "paper_2606_12876_gb300.aq_gemv (ctypes -> libaq.so), eager"}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        rate, per, n = cpu_oracle_rate(layer, x_bits, ms, 10.0)
+        cpu = {"value": rate, "unit": "GB/s", "cores": oracle.num_threads(), "kind": "oracle",
+               "sample": "%d full steps (4096x4096, batch 1, m=1..4), %.2f s/step" % (n, per)}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f32", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "out": out, "in": inp, "G": 8, "M": 4, "B": 8,
+                       "books": "2^8 x 8 f16 N(0,0.02^2)", "codes": "u8 uniform",
+                       "scales": "f16 U(0.5,1.5)", "x": "f16 N(0,1), batch 1",
+                       "step": "aq_gemv for m=1,2,3,4", "parallelism": "replicas",
+                       "l2": "rotating %d weight copies (%d x %.1f MB >= 3x L2 %.0f MB)" % (
+                           ncopies, ncopies, pbytes / 1e6, l2 / 1e6)},
+            "per_m": per_m,
+            "roofline": None if dom is None else {
+                "bound": "hbm", "kernel": "gemv_lut_kernel m=%d" % dom["m"],
+                "achieved": dom["GB_s"], "peak": hbm_peak, "unit": "GB/s",
+                "frac": round(dom["GB_s"] / hbm_peak, 4), "traffic": None,
+                "peak_source": peak_src},
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": len(ms) * args.steps,
+            "clocks": clk,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        reference_arm(args)
+    else:
+        own_arm(args)
+
+
+if __name__ == "__main__":
+    main()

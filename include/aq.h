@@ -1,0 +1,141 @@
+/*
+ * aq.h - C ABI of the multi-bitwidth additive-codebook dequantize-and-multiply library
+ * (GB300 / sm_103a). Drop-by-Drop, arxiv 2606.12876.
+ *
+ * A linear layer W (d_out x d_in) is stored once as M additive codebooks C_0..C_{M-1}
+ * (each 2^B codewords of g = 8 values), per-output-row scales s, and one B-bit code per
+ * (row, group of g inputs, codebook). At call time a prefix length m (1 <= m <= M) selects
+ * how many codebooks are summed (Sec. 5: "partial reconstruction using the first k
+ * codebooks"; the number of active codebooks is a deployment parameter):
+ *
+ *     W_m[o, g*8 + e] = s[o] * sum_{k<m} C_k[ b_k[o, g] ][e]         (Sec. 3.2 and Sec. 5)
+ *     y[t, o]         = sum_i x[t, i] * W_m[o, i]                     (Sec. 2.2, Y = W X)
+ *
+ * Conventions that hold for every entry point:
+ *   - All data pointers are DEVICE pointers, 16-byte aligned, owned by the caller. The
+ *     library allocates and frees nothing and keeps no pointer after a call returns.
+ *   - stream is a cudaStream_t passed as void* (NULL = the legacy default stream). All work
+ *     is enqueued asynchronously on it; no call synchronises unless its comment says so.
+ *   - Argument errors are detected on the host before anything is launched; the call then
+ *     returns a non-zero aq_status and the device is untouched. A failed launch returns
+ *     AQ_ERR_CUDA.
+ *   - Readings of points the paper leaves open: the scale multiplies the codebook sum of its
+ *     row (R1); a codebook is stored [2^B][g], codeword-contiguous (R2); books are numbered
+ *     0..M-1 and "prefix m" means books 0..m-1.
+ */
+#ifndef AQ_H
+#define AQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define AQ_ABI_VERSION 1
+
+typedef enum {
+    AQ_OK = 0,
+    AQ_ERR_INVALID_ARG = 1,   /* null pointer, m outside 1..M, bad sizes, bad dtype */
+    AQ_ERR_UNSUPPORTED = 2,   /* valid in principle but not implemented (e.g. g != 8) */
+    AQ_ERR_ALIGNMENT = 3,     /* a pointer is not 16-byte aligned */
+    AQ_ERR_CUDA = 4,          /* a CUDA launch or runtime call failed */
+    AQ_ERR_TIMEOUT = 5,       /* a bounded device-side wait gave up (reported via workspace) */
+    AQ_ERR_WORKSPACE = 6      /* workspace missing or smaller than the *_workspace_bytes query */
+} aq_status;
+
+typedef enum { AQ_F16 = 0, AQ_BF16 = 1, AQ_F32 = 2 } aq_dtype;
+
+/* Shape and storage types of one quantized layer (App. C lists the three stored parts:
+ * codebooks, codes, per-output-unit scales). */
+typedef struct aq_layout {
+    int32_t out_features;   /* d_out >= 0 */
+    int32_t in_features;    /* d_in >= 8, a multiple of group_size */
+    int32_t group_size;     /* g; only 8 is supported */
+    int32_t num_books;      /* M, 1..8 */
+    int32_t code_bits;      /* B; 8 (uint8 codes) or 16 (uint16 codes) */
+    int32_t book_dtype;     /* AQ_F16 or AQ_BF16: element type of the codebooks */
+    int32_t scale_dtype;    /* AQ_F16 or AQ_BF16: element type of the scales */
+} aq_layout;
+
+/* ABI version of the loaded library (AQ_ABI_VERSION). */
+int aq_abi_version(void);
+
+/* Static English text for a status code; never NULL. */
+const char* aq_status_string(int status);
+
+/* ---------------------------------------------------------------- packed code planes
+ * Codes are stored codebook-major ("planes"), so a prefix m reads only the first m planes:
+ *   rows_pad = d_out rounded up to 32; ng = d_in/8 groups, ng_pad = ng rounded up to 32;
+ *   S = ng_pad/32 slices of 32 groups. Plane k (k = 0..M-1) is rows_pad*ng_pad codes of
+ *   B/8 bytes each, laid out [slice][row][position] with 32 positions per (slice,row).
+ *   Position p of row o in slice s holds the code of group s*32 + ((p + o) mod 32): each
+ *   row's 32 codes of a slice are rotated by the row index, so 32 consecutive rows read a
+ *   position p together touch 32 different groups. Padding rows/groups hold code 0.
+ *   Plane k starts at byte k*aq_plane_bytes(); the first m planes are a contiguous prefix. */
+
+/* Bytes of one code plane; 0 if the layout is invalid. */
+size_t aq_plane_bytes(const aq_layout* layout);
+
+/* Bytes of the first m planes (m*aq_plane_bytes); 0 if the layout or m is invalid. */
+size_t aq_packed_bytes(const aq_layout* layout, int m);
+
+/* Pack natural codes into planes (the codes b_{i,j,m} of Sec. 3.2).
+ *   codes  : device, (d_out, d_in/8, M) row-major, uint8 (B = 8) or uint16 (B = 16);
+ *            code values must be < 2^B.
+ *   planes : device, aq_packed_bytes(layout, M) bytes, fully written (padding = 0). */
+aq_status aq_pack(const aq_layout* layout, const void* codes, void* planes, void* stream);
+
+/* ---------------------------------------------------------------- decode
+ * W_m written out densely (Sec. 5 partial reconstruction with the scale of R1).
+ * Bit-exact contract: for each element, acc = +0.0f; for k = 0..m-1: acc += (float)C_k[...][e]
+ * (fp32 adds, in that order); v = acc * (float)s[o] (one fp32 multiply); the output is v
+ * rounded once, to nearest-even, to book_dtype.
+ *   planes : device, at least the first m planes (aq_packed_bytes(layout, m) bytes)
+ *   books  : device, [M][2^B][8] of book_dtype (only the first m books are read)
+ *   scales : device, [d_out] of scale_dtype
+ *   w      : device, [d_out][d_in] of book_dtype, row-major. */
+aq_status aq_decode(const aq_layout* layout, int m, const void* planes, const void* books,
+                    const void* scales, void* w, void* stream);
+
+/* ---------------------------------------------------------------- GEMV (batch 1..16)
+ * y[t, o] = sum_i x[t, i] * W_m[o, i] for t < batch, accumulated in fp32. The kernel reads
+ * the first m planes once (HBM-bound at batch 1); 8-bit codebooks are staged on chip.
+ *   x         : device, [batch][d_in] of x_dtype (AQ_F16 or AQ_BF16), row-major
+ *   y         : device, [batch][d_out] of y_dtype (AQ_F16, AQ_BF16 or AQ_F32), row-major
+ *   workspace : device scratch of at least aq_gemv_workspace_bytes(layout, batch) bytes.
+ *               It must be zero-filled once before its first use (aq_workspace_init); every
+ *               call leaves it zeroed again. Calls that may overlap on the GPU must not
+ *               share a workspace.
+ * Accuracy: |y - y_exact| <= 1e-2*(1+|y_exact|) per element and relative Frobenius error
+ * <= 2e-3, with y_exact the fp64 product of the exactly widened stored values. */
+size_t aq_gemv_workspace_bytes(const aq_layout* layout, int batch);
+aq_status aq_gemv(const aq_layout* layout, int m, const void* planes, const void* books,
+                  const void* scales, const void* x, int x_dtype, int batch, void* y,
+                  int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
+
+/* ---------------------------------------------------------------- GEMM (prefill)
+ * Same product for many tokens: y[t, o] = sum_i x[t, i] * W_m[o, i], t < tokens. Decoded
+ * weight tiles are built in shared memory and multiplied on the tensor cores with fp32
+ * accumulation. Supported: code_bits = 8, book_dtype == x_dtype (f16 or bf16).
+ *   x : device, [tokens][d_in] of x_dtype;  y : device, [tokens][d_out] of y_dtype.
+ *   workspace : aq_gemm_workspace_bytes(layout, tokens) bytes, zero-filled before first use;
+ *               its first word receives a device-side status (see aq_workspace_status). */
+size_t aq_gemm_workspace_bytes(const aq_layout* layout, int tokens);
+aq_status aq_gemm(const aq_layout* layout, int m, const void* planes, const void* books,
+                  const void* scales, const void* x, int x_dtype, int tokens, void* y,
+                  int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
+
+/* ---------------------------------------------------------------- workspace helpers
+ * aq_workspace_init: enqueue a zero-fill of bytes at workspace (cudaMemsetAsync).
+ * aq_workspace_status: SYNCHRONISES stream, then returns the device-side status a kernel
+ * recorded in the workspace (AQ_OK if none) and clears it. */
+aq_status aq_workspace_init(void* workspace, size_t bytes, void* stream);
+aq_status aq_workspace_status(void* workspace, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AQ_H */

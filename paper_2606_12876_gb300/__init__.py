@@ -1,0 +1,166 @@
+"""Python binding of libaq, the GB300 multi-bitwidth additive-codebook library (include/aq.h).
+
+Argument marshalling only: every function forwards to the C entry point of the same name in
+libaq.so, passing device pointers of torch tensors and the current CUDA stream. All the
+arithmetic runs in the library's CUDA kernels; there is no Python or CPU fallback, and the
+functions raise if the library is missing.
+"""
+import ctypes
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libaq.so")
+
+AQ_OK, AQ_ERR_INVALID_ARG, AQ_ERR_UNSUPPORTED, AQ_ERR_ALIGNMENT = 0, 1, 2, 3
+AQ_ERR_CUDA, AQ_ERR_TIMEOUT, AQ_ERR_WORKSPACE = 4, 5, 6
+AQ_F16, AQ_BF16, AQ_F32 = 0, 1, 2
+DTYPES = {"f16": AQ_F16, "bf16": AQ_BF16, "f32": AQ_F32}
+TORCH_DTYPES = {AQ_F16: torch.float16, AQ_BF16: torch.bfloat16, AQ_F32: torch.float32}
+
+# Every entry point that include/aq.h declares.
+EXPORTS = ["aq_abi_version", "aq_status_string", "aq_plane_bytes", "aq_packed_bytes", "aq_pack",
+           "aq_decode", "aq_gemv_workspace_bytes", "aq_gemv", "aq_gemm_workspace_bytes",
+           "aq_gemm", "aq_workspace_init", "aq_workspace_status"]
+
+
+class AQError(RuntimeError):
+    def __init__(self, status, where):
+        self.status = status
+        super().__init__("%s failed: %s (status %d)" % (where, status_string(status), status))
+
+
+class Layout(ctypes.Structure):
+    """struct aq_layout."""
+    _fields_ = [("out_features", ctypes.c_int32), ("in_features", ctypes.c_int32),
+                ("group_size", ctypes.c_int32), ("num_books", ctypes.c_int32),
+                ("code_bits", ctypes.c_int32), ("book_dtype", ctypes.c_int32),
+                ("scale_dtype", ctypes.c_int32)]
+
+    @classmethod
+    def make(cls, out, inp, M, B=8, G=8, book_dtype="f16", scale_dtype="f16"):
+        return cls(out, inp, G, M, B, DTYPES[book_dtype], DTYPES[scale_dtype])
+
+
+_lib = None
+
+
+def lib():
+    """Load libaq.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError("libaq.so is not built; run __graft_entry__.build() or "
+                               "python paper_2606_12876_gb300/build.py")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, i32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+        lp = ctypes.POINTER(Layout)
+        sig = {
+            "aq_abi_version": (i32, []),
+            "aq_status_string": (ctypes.c_char_p, [i32]),
+            "aq_plane_bytes": (sz, [lp]),
+            "aq_packed_bytes": (sz, [lp, i32]),
+            "aq_pack": (i32, [lp, vp, vp, vp]),
+            "aq_decode": (i32, [lp, i32, vp, vp, vp, vp, vp]),
+            "aq_gemv_workspace_bytes": (sz, [lp, i32]),
+            "aq_gemv": (i32, [lp, i32, vp, vp, vp, vp, i32, i32, vp, i32, vp, sz, vp]),
+            "aq_gemm_workspace_bytes": (sz, [lp, i32]),
+            "aq_gemm": (i32, [lp, i32, vp, vp, vp, vp, i32, i32, vp, i32, vp, sz, vp]),
+            "aq_workspace_init": (i32, [vp, sz, vp]),
+            "aq_workspace_status": (i32, [vp, vp]),
+        }
+        for name, (res, args) in sig.items():
+            fn = getattr(L, name)
+            fn.restype, fn.argtypes = res, args
+        _lib = L
+    return _lib
+
+
+def status_string(status):
+    return lib().aq_status_string(int(status)).decode()
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(status, where):
+    if status != AQ_OK:
+        raise AQError(status, where)
+
+
+def abi_version():
+    return lib().aq_abi_version()
+
+
+def plane_bytes(layout):
+    return lib().aq_plane_bytes(ctypes.byref(layout))
+
+
+def packed_bytes(layout, m):
+    return lib().aq_packed_bytes(ctypes.byref(layout), m)
+
+
+def gemv_workspace_bytes(layout, batch):
+    return lib().aq_gemv_workspace_bytes(ctypes.byref(layout), batch)
+
+
+def gemm_workspace_bytes(layout, tokens):
+    return lib().aq_gemm_workspace_bytes(ctypes.byref(layout), tokens)
+
+
+def aq_pack(layout, codes, planes, stream=None):
+    _check(lib().aq_pack(ctypes.byref(layout), _ptr(codes), _ptr(planes), _stream(stream)),
+           "aq_pack")
+
+
+def aq_decode(layout, m, planes, books, scales, w, stream=None):
+    _check(lib().aq_decode(ctypes.byref(layout), m, _ptr(planes), _ptr(books), _ptr(scales),
+                           _ptr(w), _stream(stream)), "aq_decode")
+
+
+def aq_gemv(layout, m, planes, books, scales, x, x_dtype, batch, y, y_dtype, workspace,
+            workspace_bytes=None, stream=None):
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    _check(lib().aq_gemv(ctypes.byref(layout), m, _ptr(planes), _ptr(books), _ptr(scales),
+                         _ptr(x), x_dtype, batch, _ptr(y), y_dtype, _ptr(workspace),
+                         workspace_bytes, _stream(stream)), "aq_gemv")
+
+
+def aq_gemm(layout, m, planes, books, scales, x, x_dtype, tokens, y, y_dtype, workspace,
+            workspace_bytes=None, stream=None):
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    _check(lib().aq_gemm(ctypes.byref(layout), m, _ptr(planes), _ptr(books), _ptr(scales),
+                         _ptr(x), x_dtype, tokens, _ptr(y), y_dtype, _ptr(workspace),
+                         workspace_bytes, _stream(stream)), "aq_gemm")
+
+
+def aq_workspace_init(workspace, nbytes=None, stream=None):
+    if nbytes is None:
+        nbytes = workspace.numel() * workspace.element_size()
+    _check(lib().aq_workspace_init(_ptr(workspace), nbytes, _stream(stream)), "aq_workspace_init")
+
+
+def aq_workspace_status(workspace, stream=None):
+    """Synchronises the stream; returns the device-side status recorded in the workspace."""
+    return lib().aq_workspace_status(_ptr(workspace), _stream(stream))
+
+
+def workspace(nbytes, device="cuda"):
+    """A zero-filled workspace tensor of at least nbytes (16-byte aligned by the allocator)."""
+    return torch.zeros(max(16, (nbytes + 15) // 16 * 16), dtype=torch.uint8, device=device)

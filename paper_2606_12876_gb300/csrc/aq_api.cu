@@ -1,0 +1,197 @@
+// Host side of the C ABI declared in include/aq.h: argument validation, size queries and
+// dispatch to the kernel launchers. Nothing here allocates device memory.
+#include <mutex>
+
+#include "aq_internal.cuh"
+
+namespace aq {
+
+aq_status make_dims(const aq_layout* L, Dims* d) {
+    if (!L || !d) return AQ_ERR_INVALID_ARG;
+    if (L->out_features < 0 || L->in_features <= 0 || L->group_size <= 0 || L->num_books <= 0 ||
+        L->code_bits <= 0 || L->code_bits > 16)
+        return AQ_ERR_INVALID_ARG;
+    if (L->in_features % L->group_size) return AQ_ERR_INVALID_ARG;
+    if ((L->book_dtype != AQ_F16 && L->book_dtype != AQ_BF16) ||
+        (L->scale_dtype != AQ_F16 && L->scale_dtype != AQ_BF16))
+        return AQ_ERR_INVALID_ARG;
+    if (L->group_size != 8) return AQ_ERR_UNSUPPORTED;
+    if (L->code_bits != 8 && L->code_bits != 16) return AQ_ERR_UNSUPPORTED;
+    if (L->num_books > 8) return AQ_ERR_UNSUPPORTED;
+    d->out = L->out_features;
+    d->in = L->in_features;
+    d->G = L->group_size;
+    d->M = L->num_books;
+    d->B = L->code_bits;
+    d->book_dt = L->book_dtype;
+    d->scale_dt = L->scale_dtype;
+    d->ng = d->in / 8;
+    d->ng_pad = (d->ng + 31) / 32 * 32;
+    d->S = d->ng_pad / 32;
+    d->rows_pad = (int)(((long long)d->out + 31) / 32 * 32);
+    d->RBc = d->rows_pad / 32;
+    d->esz = d->B / 8;
+    d->plane_elems = (size_t)d->rows_pad * (size_t)d->ng_pad;
+    d->plane_bytes = d->plane_elems * d->esz;
+    return AQ_OK;
+}
+
+aq_status device_info(DeviceInfo* info) {
+    static std::mutex mu;
+    static DeviceInfo cache[64];
+    static bool have[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return AQ_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!have[dev]) {
+        DeviceInfo di{};
+        if (cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&di.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+                cudaSuccess)
+            return AQ_ERR_CUDA;
+        cache[dev] = di;
+        have[dev] = true;
+    }
+    *info = cache[dev];
+    return AQ_OK;
+}
+
+}  // namespace aq
+
+using aq::Dims;
+
+namespace {
+
+inline bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+inline cudaStream_t as_stream(void* s) { return (cudaStream_t)s; }
+
+aq_status check_m(const Dims& d, int m) { return (m < 1 || m > d.M) ? AQ_ERR_INVALID_ARG : AQ_OK; }
+
+aq_status check_ptrs(std::initializer_list<const void*> ps) {
+    for (const void* p : ps)
+        if (!p) return AQ_ERR_INVALID_ARG;
+    for (const void* p : ps)
+        if (!aligned16(p)) return AQ_ERR_ALIGNMENT;
+    return AQ_OK;
+}
+
+size_t gemv_ws_bytes(const Dims& d, int batch) {
+    return aq::ws_partial_offset(d) + (size_t)d.S * (size_t)batch * (size_t)d.rows_pad * 4;
+}
+
+}  // namespace
+
+extern "C" {
+
+int aq_abi_version(void) { return AQ_ABI_VERSION; }
+
+const char* aq_status_string(int status) {
+    switch (status) {
+        case AQ_OK: return "ok";
+        case AQ_ERR_INVALID_ARG: return "invalid argument";
+        case AQ_ERR_UNSUPPORTED: return "unsupported configuration";
+        case AQ_ERR_ALIGNMENT: return "pointer not 16-byte aligned";
+        case AQ_ERR_CUDA: return "CUDA error";
+        case AQ_ERR_TIMEOUT: return "device-side wait timed out";
+        case AQ_ERR_WORKSPACE: return "workspace missing or too small";
+        default: return "unknown status";
+    }
+}
+
+size_t aq_plane_bytes(const aq_layout* layout) {
+    Dims d;
+    return aq::make_dims(layout, &d) == AQ_OK ? d.plane_bytes : 0;
+}
+
+size_t aq_packed_bytes(const aq_layout* layout, int m) {
+    Dims d;
+    if (aq::make_dims(layout, &d) != AQ_OK || check_m(d, m) != AQ_OK) return 0;
+    return (size_t)m * d.plane_bytes;
+}
+
+aq_status aq_pack(const aq_layout* layout, const void* codes, void* planes, void* stream) {
+    Dims d;
+    aq_status st = aq::make_dims(layout, &d);
+    if (st != AQ_OK) return st;
+    if ((st = check_ptrs({planes})) != AQ_OK) return st;
+    if (d.out > 0 && (st = check_ptrs({codes})) != AQ_OK) return st;
+    return aq::launch_pack(d, codes, planes, as_stream(stream));
+}
+
+aq_status aq_decode(const aq_layout* layout, int m, const void* planes, const void* books,
+                    const void* scales, void* w, void* stream) {
+    Dims d;
+    aq_status st = aq::make_dims(layout, &d);
+    if (st != AQ_OK) return st;
+    if ((st = check_m(d, m)) != AQ_OK) return st;
+    if (d.out == 0) return AQ_OK;
+    if ((st = check_ptrs({planes, books, scales, w})) != AQ_OK) return st;
+    return aq::launch_decode(d, m, planes, books, scales, w, as_stream(stream));
+}
+
+size_t aq_gemv_workspace_bytes(const aq_layout* layout, int batch) {
+    Dims d;
+    if (aq::make_dims(layout, &d) != AQ_OK || batch < 0 || batch > 16) return 0;
+    return gemv_ws_bytes(d, batch < 1 ? 1 : batch);
+}
+
+aq_status aq_gemv(const aq_layout* layout, int m, const void* planes, const void* books,
+                  const void* scales, const void* x, int x_dtype, int batch, void* y,
+                  int y_dtype, void* workspace, size_t workspace_bytes, void* stream) {
+    Dims d;
+    aq_status st = aq::make_dims(layout, &d);
+    if (st != AQ_OK) return st;
+    if ((st = check_m(d, m)) != AQ_OK) return st;
+    if (batch < 0 || batch > 16) return AQ_ERR_INVALID_ARG;
+    if (x_dtype != AQ_F16 && x_dtype != AQ_BF16) return AQ_ERR_INVALID_ARG;
+    if (y_dtype != AQ_F16 && y_dtype != AQ_BF16 && y_dtype != AQ_F32) return AQ_ERR_INVALID_ARG;
+    if (batch == 0 || d.out == 0) return AQ_OK;
+    if ((st = check_ptrs({planes, books, scales, x, y})) != AQ_OK) return st;
+    if (!workspace || workspace_bytes < gemv_ws_bytes(d, batch)) return AQ_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;
+    return aq::launch_gemv(d, m, planes, books, scales, x, x_dtype, batch, y, y_dtype, workspace,
+                           as_stream(stream));
+}
+
+size_t aq_gemm_workspace_bytes(const aq_layout* layout, int tokens) {
+    Dims d;
+    if (aq::make_dims(layout, &d) != AQ_OK || tokens < 0) return 0;
+    return aq::kWsStatusBytes;
+}
+
+aq_status aq_gemm(const aq_layout* layout, int m, const void* planes, const void* books,
+                  const void* scales, const void* x, int x_dtype, int tokens, void* y,
+                  int y_dtype, void* workspace, size_t workspace_bytes, void* stream) {
+    Dims d;
+    aq_status st = aq::make_dims(layout, &d);
+    if (st != AQ_OK) return st;
+    if ((st = check_m(d, m)) != AQ_OK) return st;
+    if (tokens < 0) return AQ_ERR_INVALID_ARG;
+    (void)planes; (void)books; (void)scales; (void)x; (void)x_dtype; (void)y; (void)y_dtype;
+    (void)workspace; (void)workspace_bytes; (void)stream;
+    return AQ_ERR_UNSUPPORTED;
+}
+
+aq_status aq_workspace_init(void* workspace, size_t bytes, void* stream) {
+    if (!workspace) return AQ_ERR_INVALID_ARG;
+    if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;
+    return cudaMemsetAsync(workspace, 0, bytes, as_stream(stream)) == cudaSuccess ? AQ_OK
+                                                                                 : AQ_ERR_CUDA;
+}
+
+aq_status aq_workspace_status(void* workspace, void* stream) {
+    if (!workspace) return AQ_ERR_INVALID_ARG;
+    if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;
+    unsigned int word = 0;
+    const cudaStream_t st = as_stream(stream);
+    if (cudaMemcpyAsync(&word, workspace, 4, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess)
+        return AQ_ERR_CUDA;
+    if (word == 0) return AQ_OK;
+    if (cudaMemsetAsync(workspace, 0, 4, st) != cudaSuccess || cudaStreamSynchronize(st) != cudaSuccess)
+        return AQ_ERR_CUDA;
+    return (aq_status)word;
+}
+
+}  // extern "C"

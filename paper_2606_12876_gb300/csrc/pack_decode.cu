@@ -1,0 +1,154 @@
+// aq_pack and aq_decode kernels.
+//
+// Packing turns the natural code tensor b (Sec. 3.2: one B-bit index per output row, group
+// of 8 inputs and codebook) into codebook-major planes so that a prefix of m codebooks
+// (Sec. 5) is a prefix of the buffer. Decoding writes the partial reconstruction W_m densely.
+#include "aq_internal.cuh"
+
+namespace aq {
+namespace {
+
+// One thread per packed code. Output index = ((k*S + s)*rows_pad + o)*32 + p.
+template <typename CT>
+__global__ void pack_kernel(const CT* __restrict__ codes, CT* __restrict__ planes, int out,
+                            int ng, int M, int rows_pad, int S, size_t total) {
+    for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        const int p = (int)(idx & 31);
+        size_t rest = idx >> 5;
+        const int o = (int)(rest % rows_pad);
+        rest /= rows_pad;
+        const int s = (int)(rest % S);
+        const int k = (int)(rest / S);
+        const int g = s * 32 + ((p + o) & 31);
+        CT v = 0;
+        if (o < out && g < ng) v = codes[((size_t)o * ng + g) * M + k];
+        planes[idx] = v;
+    }
+}
+
+constexpr int kDecWarps = 8;
+
+// Decode: each warp owns one 32-row block of one slice. Lane L stages its own row's codes
+// for the m planes in shared memory, then the warp walks the 32 rows with lane L producing
+// group s*32+L of that row, so each output row segment is written as 512 contiguous bytes.
+// Bit-exact contract (aq.h): fp32 adds in book order from +0.0f, one fp32 multiply by the
+// scale, one round-to-nearest-even to the book type.
+template <int B, int BDT, int SDT>
+__global__ void __launch_bounds__(kDecWarps * 32)
+decode_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
+              const uint16_t* __restrict__ scales, uint16_t* __restrict__ w, int m, int out,
+              int in, int ng, int rows_pad, int RBc, size_t plane_bytes) {
+    constexpr int ESZ = B / 8;                       // bytes per code
+    constexpr int UNIT = 32 * ESZ;                   // bytes of one (row, slice) unit
+    extern __shared__ __align__(16) unsigned char smem[];
+    uint16_t* books_s = (uint16_t*)smem;             // B = 8: [m][256][8]
+    const size_t books_bytes = (B == 8) ? (size_t)m * 256 * 8 * 2 : 0;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    unsigned char* codes_s = smem + books_bytes + (size_t)warp * m * 32 * UNIT;
+
+    if constexpr (B == 8) {
+        const uint4* src = (const uint4*)books;
+        uint4* dst = (uint4*)books_s;
+        for (int i = threadIdx.x; i < m * 256; i += blockDim.x) dst[i] = src[i];
+    }
+    const int s = blockIdx.y;
+    const int rb = blockIdx.x * kDecWarps + warp;
+    const bool active = rb < RBc;
+    if (active) {
+        const int o = rb * 32 + lane;
+        for (int k = 0; k < m; ++k) {
+            const uint4* src =
+                (const uint4*)(planes + k * plane_bytes + ((size_t)s * rows_pad + o) * UNIT);
+            uint4* dst = (uint4*)(codes_s + ((size_t)k * 32 + lane) * UNIT);
+#pragma unroll
+            for (int q = 0; q < UNIT / 16; ++q) dst[q] = ld_stream_v4(src + q);
+        }
+    }
+    __syncthreads();
+    if (!active) return;
+
+    const int g = s * 32 + lane;
+    for (int r = 0; r < 32; ++r) {
+        const int o = rb * 32 + r;
+        if (o >= out) break;
+        const float sc = bits_to_f32<SDT>(scales[o]);
+        const int p = (lane - r) & 31;               // position of group `lane` in row o
+        float acc[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[e] = 0.0f;
+        for (int k = 0; k < m; ++k) {
+            uint32_t code;
+            if constexpr (B == 8) code = codes_s[((size_t)k * 32 + r) * UNIT + p];
+            else code = ((const uint16_t*)(codes_s + ((size_t)k * 32 + r) * UNIT))[p];
+            uint4 cw;
+            if constexpr (B == 8) cw = ((const uint4*)books_s)[k * 256 + code];
+            else cw = __ldg((const uint4*)books + ((size_t)k << 16) + code);
+            float c[8];
+            unpack8<BDT>(cw, c);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[e] = __fadd_rn(acc[e], c[e]);
+        }
+        if (g < ng) {
+            uint32_t pk[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t lo = f32_to_bits<BDT>(__fmul_rn(acc[2 * i], sc));
+                const uint32_t hi = f32_to_bits<BDT>(__fmul_rn(acc[2 * i + 1], sc));
+                pk[i] = lo | (hi << 16);
+            }
+            *(uint4*)(w + (size_t)o * in + (size_t)g * 8) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        }
+    }
+}
+
+template <int B, int BDT, int SDT>
+aq_status run_decode(const Dims& d, int m, const void* planes, const void* books,
+                     const void* scales, void* w, cudaStream_t st) {
+    const size_t smem = (B == 8 ? (size_t)m * 4096 : 0) + (size_t)kDecWarps * m * 32 * 32 * (B / 8);
+    auto kern = decode_kernel<B, BDT, SDT>;
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+        return AQ_ERR_CUDA;
+    dim3 grid((d.RBc + kDecWarps - 1) / kDecWarps, d.S);
+    kern<<<grid, kDecWarps * 32, smem, st>>>((const uint8_t*)planes, (const uint16_t*)books,
+                                             (const uint16_t*)scales, (uint16_t*)w, m, d.out,
+                                             d.in, d.ng, d.rows_pad, d.RBc, d.plane_bytes);
+    return cudaGetLastError() == cudaSuccess ? AQ_OK : AQ_ERR_CUDA;
+}
+
+}  // namespace
+
+aq_status launch_pack(const Dims& d, const void* codes, void* planes, cudaStream_t st) {
+    const size_t total = (size_t)d.M * d.plane_elems;
+    if (total == 0) return AQ_OK;
+    const int threads = 256;
+    const size_t want = (total + threads - 1) / threads;
+    const int blocks = (int)(want < 65535 * 16 ? want : 65535 * 16);
+    if (d.esz == 1)
+        pack_kernel<uint8_t><<<blocks, threads, 0, st>>>((const uint8_t*)codes, (uint8_t*)planes,
+                                                         d.out, d.ng, d.M, d.rows_pad, d.S, total);
+    else
+        pack_kernel<uint16_t><<<blocks, threads, 0, st>>>((const uint16_t*)codes,
+                                                          (uint16_t*)planes, d.out, d.ng, d.M,
+                                                          d.rows_pad, d.S, total);
+    return cudaGetLastError() == cudaSuccess ? AQ_OK : AQ_ERR_CUDA;
+}
+
+aq_status launch_decode(const Dims& d, int m, const void* planes, const void* books,
+                        const void* scales, void* w, cudaStream_t st) {
+    if (d.out == 0) return AQ_OK;
+    const int key = (d.B == 16) * 4 + (d.book_dt == AQ_BF16) * 2 + (d.scale_dt == AQ_BF16);
+    switch (key) {
+        case 0: return run_decode<8, AQ_F16, AQ_F16>(d, m, planes, books, scales, w, st);
+        case 1: return run_decode<8, AQ_F16, AQ_BF16>(d, m, planes, books, scales, w, st);
+        case 2: return run_decode<8, AQ_BF16, AQ_F16>(d, m, planes, books, scales, w, st);
+        case 3: return run_decode<8, AQ_BF16, AQ_BF16>(d, m, planes, books, scales, w, st);
+        case 4: return run_decode<16, AQ_F16, AQ_F16>(d, m, planes, books, scales, w, st);
+        case 5: return run_decode<16, AQ_F16, AQ_BF16>(d, m, planes, books, scales, w, st);
+        case 6: return run_decode<16, AQ_BF16, AQ_F16>(d, m, planes, books, scales, w, st);
+        default: return run_decode<16, AQ_BF16, AQ_BF16>(d, m, planes, books, scales, w, st);
+    }
+}
+
+}  // namespace aq

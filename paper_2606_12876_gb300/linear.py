@@ -1,0 +1,112 @@
+"""AQLinear: one additive-codebook linear layer resident on the GPU, served at any prefix m.
+
+The layer is stored once (AQLMFormat(C, b, s) of Alg. 1: M codebooks, codes, per-row scales)
+and evaluated with the first m codebooks chosen per call (Sec. 5). Device memory comes from
+torch; all work is done by libaq through the binding in this package.
+"""
+import numpy as np
+import torch
+
+from . import (AQ_BF16, AQ_F16, AQ_F32, DTYPES, TORCH_DTYPES, Layout, aq_decode, aq_gemm,
+               aq_gemv, aq_pack, gemm_workspace_bytes, gemv_workspace_bytes, packed_bytes,
+               workspace)
+
+
+def _u16_to_device(a, device):
+    a = np.ascontiguousarray(a, dtype=np.uint16)
+    return torch.from_numpy(a.view(np.int16)).to(device)
+
+
+class AQLinear:
+    """Packed planes, codebooks and scales of one layer on `device`.
+
+    books: [M][2^B][8] fp16/bf16 bit patterns (uint16); codes: (out, in/8, M) uint8/uint16;
+    scales: [out] bit patterns. The natural codes are packed on the GPU by aq_pack.
+    """
+
+    def __init__(self, books, codes, scales, book_dtype="f16", scale_dtype="f16",
+                 device="cuda", keep_codes=False):
+        out, ng, M = codes.shape
+        B = 8 if codes.dtype == np.uint8 else 16
+        self.layout = Layout.make(out, ng * 8, M, B=B, book_dtype=book_dtype,
+                                  scale_dtype=scale_dtype)
+        self.out, self.inp, self.M, self.B = out, ng * 8, M, B
+        self.device = torch.device(device)
+        self.book_dtype, self.scale_dtype = book_dtype, scale_dtype
+        self.books = _u16_to_device(books, self.device)
+        self.scales = _u16_to_device(scales, self.device)
+        codes_t = torch.from_numpy(np.ascontiguousarray(codes).view(
+            np.int8 if B == 8 else np.int16)).to(self.device)
+        self.planes = torch.empty(packed_bytes(self.layout, M), dtype=torch.uint8,
+                                  device=self.device)
+        aq_pack(self.layout, codes_t, self.planes)
+        self.codes = codes_t if keep_codes else None
+        self._ws = {}
+
+    @classmethod
+    def from_layer(cls, layer, device="cuda", keep_codes=False):
+        """From a workloads.make_layer() dict."""
+        return cls(layer["books"], layer["codes"], layer["scales"], layer["book_dtype"],
+                   layer["scale_dtype"], device, keep_codes)
+
+    def planes_prefix(self, m):
+        """The first m planes: the only code bytes a prefix-m call reads."""
+        return self.planes[: packed_bytes(self.layout, m)]
+
+    def _workspace(self, kind, n):
+        nbytes = (gemv_workspace_bytes if kind == "gemv" else gemm_workspace_bytes)(self.layout, n)
+        key = (kind, torch.cuda.current_stream(self.device).cuda_stream)
+        ws = self._ws.get(key)
+        if ws is None or ws.numel() < nbytes:
+            ws = workspace(nbytes, self.device)
+            self._ws[key] = ws
+        return ws
+
+    def decode(self, m, out=None):
+        """Dense W_m [out][in] in the book dtype (bit-exact contract of aq.h)."""
+        if out is None:
+            out = torch.empty(self.out, self.inp, dtype=TORCH_DTYPES[DTYPES[self.book_dtype]],
+                              device=self.device)
+        aq_decode(self.layout, m, self.planes, self.books, self.scales, out)
+        return out
+
+    def gemv(self, x, m, y=None, y_dtype=None):
+        """y = x W_m^T for x of shape [batch <= 16, in]."""
+        xd = _dtype_code(x.dtype)
+        yd = xd if y_dtype is None else y_dtype
+        batch = x.shape[0]
+        if y is None:
+            y = torch.empty(batch, self.out, dtype=TORCH_DTYPES[yd], device=self.device)
+        ws = self._workspace("gemv", batch)
+        aq_gemv(self.layout, m, self.planes, self.books, self.scales, x, xd, batch, y, yd, ws)
+        return y
+
+    def gemm(self, x, m, y=None, y_dtype=None):
+        """y = x W_m^T for x of shape [tokens, in] on the tensor cores."""
+        xd = _dtype_code(x.dtype)
+        yd = xd if y_dtype is None else y_dtype
+        tokens = x.shape[0]
+        if y is None:
+            y = torch.empty(tokens, self.out, dtype=TORCH_DTYPES[yd], device=self.device)
+        ws = self._workspace("gemm", tokens)
+        aq_gemm(self.layout, m, self.planes, self.books, self.scales, x, xd, tokens, y, yd, ws)
+        return y
+
+    def __call__(self, x, m):
+        return self.gemv(x, m) if x.shape[0] <= 16 else self.gemm(x, m)
+
+
+def _dtype_code(dt):
+    if dt == torch.float16:
+        return AQ_F16
+    if dt == torch.bfloat16:
+        return AQ_BF16
+    if dt == torch.float32:
+        return AQ_F32
+    raise TypeError("unsupported activation dtype %s" % dt)
+
+
+def x_to_device(x_bits, x_dtype, device="cuda"):
+    """Activation bit patterns (uint16, from workloads.make_x) -> device tensor of x_dtype."""
+    t = _u16_to_device(x_bits, device)
+    return t.view(torch.float16 if x_dtype == "f16" else torch.bfloat16)

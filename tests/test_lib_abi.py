@@ -1,0 +1,127 @@
+"""The C-ABI library without a GPU: it loads, exports what include/aq.h declares, answers size
+queries that agree with the oracle's packed layout, and rejects bad arguments on the host
+(no compute call is made here)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import aq_testutil
+import oracle
+import paper_2606_12876_gb300 as aq
+import workloads
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "aq.h")
+FAKE = 1 << 20          # an aligned non-null address; never dereferenced by these tests
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    aq_testutil.ensure_built()
+
+
+def header_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:aq_status|size_t|int|const char\*)\s+(aq_\w+)\s*\(",
+                                 text, flags=re.M)))
+
+
+def test_every_declared_symbol_is_exported():
+    names = header_functions()
+    assert len(names) >= 12
+    L = ctypes.CDLL(aq.LIB_PATH)
+    for n in names:
+        assert hasattr(L, n), n
+    assert sorted(aq.EXPORTS) == names
+
+
+def test_version_and_status_strings():
+    assert aq.abi_version() == 1
+    for s in range(7):
+        assert aq.status_string(s) and aq.status_string(s) != "unknown status"
+    assert aq.status_string(99) == "unknown status"
+
+
+@pytest.mark.parametrize("out,inp,M,B", [(1, 8, 1, 8), (37, 560, 3, 8), (64, 256, 4, 8),
+                                          (50, 136, 2, 16), (4096, 4096, 4, 8)])
+def test_packed_sizes_match_oracle_layout(out, inp, M, B):
+    L = aq.Layout.make(out, inp, M, B=B)
+    layer = dict(out=out, **{"in": inp}, G=8, M=M, B=B,
+                 codes=np.zeros((out, inp // 8, M), np.uint8 if B == 8 else np.uint16))
+    total = oracle.pack(layer).size
+    assert aq.plane_bytes(L) * M == total
+    for m in range(1, M + 1):
+        assert aq.packed_bytes(L, m) == m * aq.plane_bytes(L)
+    assert aq.packed_bytes(L, 0) == 0 and aq.packed_bytes(L, M + 1) == 0
+
+
+def test_gemv_workspace_covers_partials():
+    L = aq.Layout.make(4096, 4096, 4)
+    # 16 slices x batch x 4096 rows of fp32 partials, plus status and counters
+    assert aq.gemv_workspace_bytes(L, 1) >= 16 * 4096 * 4
+    assert aq.gemv_workspace_bytes(L, 16) >= 16 * 16 * 4096 * 4
+    assert aq.gemv_workspace_bytes(L, 17) == 0
+
+
+def _lay(**kw):
+    base = dict(out=64, inp=256, M=4, B=8, G=8, book_dtype="f16", scale_dtype="f16")
+    base.update(kw)
+    return aq.Layout.make(**base)
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(G=4), aq.AQ_ERR_UNSUPPORTED), (dict(B=4), aq.AQ_ERR_UNSUPPORTED),
+    (dict(B=17), aq.AQ_ERR_INVALID_ARG), (dict(M=9), aq.AQ_ERR_UNSUPPORTED),
+    (dict(M=0), aq.AQ_ERR_INVALID_ARG), (dict(inp=260), aq.AQ_ERR_INVALID_ARG),
+    (dict(inp=0), aq.AQ_ERR_INVALID_ARG), (dict(out=-1), aq.AQ_ERR_INVALID_ARG),
+])
+def test_layout_rejected(kw, status):
+    L = _lay(**kw)
+    assert aq.plane_bytes(L) == 0
+    rc = aq.lib().aq_decode(ctypes.byref(L), 1, FAKE, FAKE, FAKE, FAKE, None)
+    assert rc == status
+
+
+def test_bad_dtype_rejected():
+    L = _lay()
+    L.book_dtype = 7
+    assert aq.lib().aq_decode(ctypes.byref(L), 1, FAKE, FAKE, FAKE, FAKE, None) == aq.AQ_ERR_INVALID_ARG
+
+
+def _gemv(L, m=1, planes=FAKE, x=FAKE, x_dt=aq.AQ_F16, batch=1, y=FAKE, y_dt=aq.AQ_F16,
+          ws=FAKE, ws_bytes=None):
+    if ws_bytes is None:
+        ws_bytes = aq.gemv_workspace_bytes(L, max(1, min(batch, 16)))
+    return aq.lib().aq_gemv(ctypes.byref(L), m, planes, FAKE, FAKE, x, x_dt, batch, y, y_dt, ws,
+                            ws_bytes, None)
+
+
+def test_gemv_argument_errors():
+    L = _lay()
+    assert _gemv(L, m=0) == aq.AQ_ERR_INVALID_ARG
+    assert _gemv(L, m=5) == aq.AQ_ERR_INVALID_ARG
+    assert _gemv(L, batch=17) == aq.AQ_ERR_INVALID_ARG
+    assert _gemv(L, batch=-1) == aq.AQ_ERR_INVALID_ARG
+    assert _gemv(L, x_dt=aq.AQ_F32) == aq.AQ_ERR_INVALID_ARG
+    assert _gemv(L, y_dt=9) == aq.AQ_ERR_INVALID_ARG
+    assert _gemv(L, planes=None) == aq.AQ_ERR_INVALID_ARG
+    assert _gemv(L, x=FAKE + 2) == aq.AQ_ERR_ALIGNMENT
+    assert _gemv(L, ws=None) == aq.AQ_ERR_WORKSPACE
+    assert _gemv(L, ws_bytes=aq.gemv_workspace_bytes(L, 1) - 4) == aq.AQ_ERR_WORKSPACE
+    # empty work is a successful no-op that touches nothing
+    assert _gemv(L, batch=0, planes=None, x=None, y=None, ws=None) == aq.AQ_OK
+    assert _gemv(_lay(out=0), planes=None, x=None, y=None, ws=None) == aq.AQ_OK
+
+
+def test_decode_and_pack_argument_errors():
+    L = _lay()
+    lib = aq.lib()
+    assert lib.aq_decode(ctypes.byref(L), 0, FAKE, FAKE, FAKE, FAKE, None) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_decode(ctypes.byref(L), 1, FAKE, None, FAKE, FAKE, None) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_decode(ctypes.byref(L), 1, FAKE, FAKE, FAKE + 8, FAKE, None) == aq.AQ_ERR_ALIGNMENT
+    assert lib.aq_pack(ctypes.byref(L), None, FAKE, None) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_pack(None, FAKE, FAKE, None) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_workspace_init(None, 16, None) == aq.AQ_ERR_INVALID_ARG
