@@ -65,6 +65,10 @@ int aq_abi_version(void);
 /* Static English text for a status code; never NULL. */
 const char* aq_status_string(int status);
 
+/* Text of the last CUDA failure seen by this thread inside the library (the call that
+ * failed, the CUDA error name and message), or "" if none. Valid until the next call. */
+const char* aq_last_error(void);
+
 /* ---------------------------------------------------------------- packed code planes
  * Codes are stored codebook-major ("planes"), so a prefix m reads only the first m planes:
  *   rows_pad = d_out rounded up to 32; ng = d_in/8 groups, ng_pad = ng rounded up to 32;
@@ -104,10 +108,14 @@ aq_status aq_decode(const aq_layout* layout, int m, const void* planes, const vo
  * the first m planes once (HBM-bound at batch 1); 8-bit codebooks are staged on chip.
  *   x         : device, [batch][d_in] of x_dtype (AQ_F16 or AQ_BF16), row-major
  *   y         : device, [batch][d_out] of y_dtype (AQ_F16, AQ_BF16 or AQ_F32), row-major
- *   workspace : device scratch of at least aq_gemv_workspace_bytes(layout, batch) bytes.
- *               It must be zero-filled once before its first use (aq_workspace_init); every
- *               call leaves it zeroed again. Calls that may overlap on the GPU must not
- *               share a workspace.
+ *   workspace : device scratch of at least aq_gemv_workspace_bytes(layout, batch) bytes:
+ *               a status word, one completion counter per 32 output rows and fp32 partial
+ *               sums (one per 256-input slice, token and row). Zero-fill it once before its
+ *               first use (aq_workspace_init); every call leaves it ready for the next one.
+ *               Calls that may overlap on the GPU must not share a workspace.
+ * One kernel is enqueued, with programmatic dependent launch; it waits for the preceding
+ * grid before reading memory. The slices of each row are summed in a fixed order, so the
+ * result does not depend on scheduling.
  * Accuracy: |y - y_exact| <= 1e-2*(1+|y_exact|) per element and relative Frobenius error
  * <= 2e-3, with y_exact the fp64 product of the exactly widened stored values. */
 size_t aq_gemv_workspace_bytes(const aq_layout* layout, int batch);

@@ -20,7 +20,7 @@ DTYPES = {"f16": AQ_F16, "bf16": AQ_BF16, "f32": AQ_F32}
 TORCH_DTYPES = {AQ_F16: torch.float16, AQ_BF16: torch.bfloat16, AQ_F32: torch.float32}
 
 # Every entry point that include/aq.h declares.
-EXPORTS = ["aq_abi_version", "aq_status_string", "aq_plane_bytes", "aq_packed_bytes", "aq_pack",
+EXPORTS = ["aq_abi_version", "aq_status_string", "aq_last_error", "aq_plane_bytes", "aq_packed_bytes", "aq_pack",
            "aq_decode", "aq_gemv_workspace_bytes", "aq_gemv", "aq_gemm_workspace_bytes",
            "aq_gemm", "aq_workspace_init", "aq_workspace_status"]
 
@@ -28,7 +28,10 @@ EXPORTS = ["aq_abi_version", "aq_status_string", "aq_plane_bytes", "aq_packed_by
 class AQError(RuntimeError):
     def __init__(self, status, where):
         self.status = status
-        super().__init__("%s failed: %s (status %d)" % (where, status_string(status), status))
+        msg = "%s failed: %s (status %d)" % (where, status_string(status), status)
+        if status == AQ_ERR_CUDA:
+            msg += ": " + lib().aq_last_error().decode()
+        super().__init__(msg)
 
 
 class Layout(ctypes.Structure):
@@ -59,6 +62,7 @@ def lib():
         sig = {
             "aq_abi_version": (i32, []),
             "aq_status_string": (ctypes.c_char_p, [i32]),
+            "aq_last_error": (ctypes.c_char_p, []),
             "aq_plane_bytes": (sz, [lp]),
             "aq_packed_bytes": (sz, [lp, i32]),
             "aq_pack": (i32, [lp, vp, vp, vp]),

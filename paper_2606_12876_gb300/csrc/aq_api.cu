@@ -1,5 +1,6 @@
 // Host side of the C ABI declared in include/aq.h: argument validation, size queries and
 // dispatch to the kernel launchers. Nothing here allocates device memory.
+#include <cstdio>
 #include <mutex>
 
 #include "aq_internal.cuh"
@@ -36,19 +37,33 @@ aq_status make_dims(const aq_layout* L, Dims* d) {
     return AQ_OK;
 }
 
+namespace {
+thread_local char g_last_error[256] = "";
+}
+
+aq_status cuda_fail(cudaError_t e, const char* what) {
+    snprintf(g_last_error, sizeof(g_last_error), "%s: %s (%s)", what, cudaGetErrorName(e),
+             cudaGetErrorString(e));
+    return AQ_ERR_CUDA;
+}
+
 aq_status device_info(DeviceInfo* info) {
     static std::mutex mu;
     static DeviceInfo cache[64];
     static bool have[64] = {};
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return AQ_ERR_CUDA;
+    if (cudaError_t e = cudaGetDevice(&dev); e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= 64) return AQ_ERR_UNSUPPORTED;
     std::lock_guard<std::mutex> lock(mu);
     if (!have[dev]) {
         DeviceInfo di{};
-        if (cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-            cudaDeviceGetAttribute(&di.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
-                cudaSuccess)
-            return AQ_ERR_CUDA;
+        if (cudaError_t e = cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, dev);
+            e != cudaSuccess)
+            return cuda_fail(e, "cudaDeviceGetAttribute");
+        if (cudaError_t e = cudaDeviceGetAttribute(&di.smem_optin,
+                                                   cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+            e != cudaSuccess)
+            return cuda_fail(e, "cudaDeviceGetAttribute");
         cache[dev] = di;
         have[dev] = true;
     }
@@ -85,6 +100,8 @@ size_t gemv_ws_bytes(const Dims& d, int batch) {
 extern "C" {
 
 int aq_abi_version(void) { return AQ_ABI_VERSION; }
+
+const char* aq_last_error(void) { return aq::g_last_error; }
 
 const char* aq_status_string(int status) {
     switch (status) {
@@ -176,8 +193,7 @@ aq_status aq_gemm(const aq_layout* layout, int m, const void* planes, const void
 aq_status aq_workspace_init(void* workspace, size_t bytes, void* stream) {
     if (!workspace) return AQ_ERR_INVALID_ARG;
     if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;
-    return cudaMemsetAsync(workspace, 0, bytes, as_stream(stream)) == cudaSuccess ? AQ_OK
-                                                                                 : AQ_ERR_CUDA;
+    return aq::cuda_ok(cudaMemsetAsync(workspace, 0, bytes, as_stream(stream)), "cudaMemsetAsync");
 }
 
 aq_status aq_workspace_status(void* workspace, void* stream) {
@@ -185,12 +201,13 @@ aq_status aq_workspace_status(void* workspace, void* stream) {
     if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;
     unsigned int word = 0;
     const cudaStream_t st = as_stream(stream);
-    if (cudaMemcpyAsync(&word, workspace, 4, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
-        cudaStreamSynchronize(st) != cudaSuccess)
-        return AQ_ERR_CUDA;
-    if (word == 0) return AQ_OK;
-    if (cudaMemsetAsync(workspace, 0, 4, st) != cudaSuccess || cudaStreamSynchronize(st) != cudaSuccess)
-        return AQ_ERR_CUDA;
+    aq_status rc = aq::cuda_ok(cudaMemcpyAsync(&word, workspace, 4, cudaMemcpyDeviceToHost, st),
+                               "cudaMemcpyAsync");
+    if (rc == AQ_OK) rc = aq::cuda_ok(cudaStreamSynchronize(st), "cudaStreamSynchronize");
+    if (rc != AQ_OK || word == 0) return rc;
+    rc = aq::cuda_ok(cudaMemsetAsync(workspace, 0, 4, st), "cudaMemsetAsync");
+    if (rc == AQ_OK) rc = aq::cuda_ok(cudaStreamSynchronize(st), "cudaStreamSynchronize");
+    if (rc != AQ_OK) return rc;
     return (aq_status)word;
 }
 

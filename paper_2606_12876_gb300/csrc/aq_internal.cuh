@@ -33,11 +33,20 @@ struct DeviceInfo {
 };
 aq_status device_info(DeviceInfo* info);
 
-// Workspace layout shared by the split-K kernels: [status 256 B][counters][partials].
+// Workspace layout of the split-K GEMV:
+//   [status word, 256 B][one u32 completion counter per 32-row block][fp32 partials
+//   [S][batch][rows_pad]]. Counters start at zero and are returned to zero by each call.
 constexpr size_t kWsStatusBytes = 256;
 inline size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 inline size_t ws_counter_bytes(const Dims& d) { return round_up((size_t)d.RBc * 4, 256); }
 inline size_t ws_partial_offset(const Dims& d) { return kWsStatusBytes + ws_counter_bytes(d); }
+
+// Records a failed CUDA call (thread-local text for aq_last_error) and returns AQ_ERR_CUDA.
+aq_status cuda_fail(cudaError_t e, const char* what);
+// AQ_OK if e is cudaSuccess, else cuda_fail(e, what).
+inline aq_status cuda_ok(cudaError_t e, const char* what) {
+    return e == cudaSuccess ? AQ_OK : cuda_fail(e, what);
+}
 
 // ---- launchers (each returns AQ_OK or AQ_ERR_CUDA; arguments are already validated) ----
 aq_status launch_pack(const Dims& d, const void* codes, void* planes, cudaStream_t st);
@@ -85,6 +94,14 @@ __device__ __forceinline__ uint4 ld_stream_v4(const void* p) {
     return r;
 }
 
+// 32-bit shared-window address of a pointer into shared memory, and plain shared loads and
+// stores through it (no generic-address conversion per access).
+__device__ __forceinline__ float lds_f32(uint32_t addr) {
+    float v;
+    asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+    return v;
+}
+
 // Byte permute (PTX prmt, generic mode): selector nibbles pick bytes of {b:a}; a nibble
 // with bit 3 set replicates the sign bit of the picked byte.
 __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
@@ -93,38 +110,155 @@ __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
     return d;
 }
 
-// Split-K epilogue shared by the GEMV kernels: the CTA that finishes last for a row chunk
-// sums the per-slice partials in slice order (deterministic), applies the row scale and
-// stores y. Counters are left at zero for the next call.
-template <int SDT>
-__device__ __forceinline__ void splitk_finish(unsigned int* counters, const float* partials,
-                                              const uint16_t* scales, void* y, int y_dt,
-                                              int out, int rows_pad, int S, int batch,
-                                              int chunk, int row0, int row1) {
-    __shared__ int s_last;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        __threadfence();
-        const unsigned prev = atomicAdd(&counters[chunk], 1u);
-        s_last = (prev == (unsigned)(S - 1));
+// ---- shared-memory barriers, bulk copies and programmatic dependent launch (sm_90+) -------
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+                 : "memory");
+}
+
+// Make barrier initialisation visible to the async (TMA) proxy and the other threads.
+__device__ __forceinline__ void mbar_fence_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Every spin-wait in this library is bounded: after kSpinLimit polls (well over a second with
+// the back-off) the wait gives up and the caller records AQ_ERR_TIMEOUT instead of hanging.
+constexpr uint32_t kSpinLimit = 1u << 22;
+
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+    for (uint32_t i = 0; i < kSpinLimit; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (i >= 4096) __nanosleep(128);
     }
-    __syncthreads();
-    if (!s_last) return;
-    __threadfence();
-    const int r1 = min(row1, out);
-    const int nrows = r1 - row0;
-    for (int idx = threadIdx.x; idx < nrows * batch; idx += blockDim.x) {
-        const int t = idx / nrows;
-        const int r = row0 + (idx - t * nrows);
-        float sum = 0.0f;
-        for (int s = 0; s < S; ++s) sum += __ldcg(partials + ((size_t)s * batch + t) * rows_pad + r);
-        const float v = sum * bits_to_f32<SDT>(scales[r]);
-        const size_t yi = (size_t)t * out + r;
-        if (y_dt == AQ_F32) ((float*)y)[yi] = v;
-        else if (y_dt == AQ_F16) ((uint16_t*)y)[yi] = f32_to_bits<AQ_F16>(v);
-        else ((uint16_t*)y)[yi] = f32_to_bits<AQ_BF16>(v);
+    return false;
+}
+
+// Record a device-side failure in the workspace status word (first error wins).
+__device__ __forceinline__ void record_status(unsigned int* status, unsigned int code) {
+    if (status) atomicCAS(status, 0u, code);
+}
+
+// 1-D bulk copy global -> shared (TMA engine), completing on an mbarrier transaction count.
+// dst, src 16-byte aligned; bytes a multiple of 16.
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes,
+                                         uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// Programmatic dependent launch: wait for the preceding grid's results / allow the next grid
+// to start launching. Both are no-ops when the launch has no programmatic dependency.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Named barrier over a subset of the CTA's warps.
+__device__ __forceinline__ void named_barrier(int id, int threads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+
+// Packed fp32 pair FMA (one instruction for two lanes of work): d = a * b + c.
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+    unsigned long long ar = *(unsigned long long*)&a, br = *(unsigned long long*)&b,
+                       cr = *(unsigned long long*)&c, dr;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(dr) : "l"(ar), "l"(br), "l"(cr));
+    return *(float2*)&dr;
+}
+
+// ---- split-K completion ------------------------------------------------------------------
+//
+// A work item is (slice s, 32-row block rb); its fp32 partial sums for the block's rows (and
+// every token) sit in partials[s][t][row]. When a CTA has written all its items it counts
+// each item on the block's counter; whoever brings a counter to S (all slices done) sums the
+// S partials of that block in slice order, applies the row scale (R1: s[o] multiplies the
+// codebook sum, so it factors out of the dot product), stores y and resets the counter.
+// The outcome does not depend on which CTA finishes last. Every thread of the CTA must call
+// this with the same n_items (it contains CTA-wide barriers).
+constexpr int kFinishMax = 1024;  // items counted per round (>= the largest CTA size used)
+
+template <int SDT, typename ItemRb>
+__device__ __forceinline__ void finish_items(long long n_items, ItemRb item_rb,
+                                             unsigned int* __restrict__ counters,
+                                             const float* __restrict__ partials,
+                                             const uint16_t* __restrict__ scales, void* y,
+                                             int y_dt, int out, int rows_pad, int S, int batch) {
+    __shared__ int s_list[kFinishMax];
+    __shared__ int s_n;
+    const int tid = threadIdx.x;
+    const size_t stride = (size_t)batch * rows_pad;
+    __threadfence();                       // this thread's partial stores are visible GPU-wide
+    for (long long base = 0; base < n_items; base += blockDim.x) {
+        __syncthreads();
+        if (tid == 0) s_n = 0;
+        __syncthreads();
+        const long long j = base + tid;
+        if (j < n_items) {
+            const int rb = item_rb(j);
+            if (atomicAdd(&counters[rb], 1u) == (unsigned)(S - 1)) s_list[atomicAdd(&s_n, 1)] = rb;
+        }
+        __syncthreads();
+        __threadfence();                   // order the counter reads before the partial reads
+        // One (row, token) per thread, all of its S loads issued before the sums: the whole
+        // finalisation of a CTA costs about one memory round trip.
+        const int n = s_n;
+        const long long total = (long long)n * 32 * batch;
+        for (long long w = tid; w < total; w += blockDim.x) {
+            const int t = (int)(w % batch);
+            const long long e = w / batch;
+            const int rb = s_list[e >> 5];
+            const int r = rb * 32 + (int)(e & 31);
+            const float* p = partials + (size_t)t * rows_pad + r;
+            float sum = 0.0f;
+            int sl = 0;
+            for (; sl + 16 <= S; sl += 16) {
+                float v[16];
+#pragma unroll
+                for (int q = 0; q < 16; ++q) v[q] = __ldcg(p + (size_t)(sl + q) * stride);
+#pragma unroll
+                for (int q = 0; q < 16; ++q) sum += v[q];
+            }
+            for (; sl < S; ++sl) sum += __ldcg(p + (size_t)sl * stride);
+            if (r < out) {
+                const float v = sum * bits_to_f32<SDT>(scales[r]);
+                const size_t yi = (size_t)t * out + r;
+                if (y_dt == AQ_F32) ((float*)y)[yi] = v;
+                else if (y_dt == AQ_F16) ((uint16_t*)y)[yi] = f32_to_bits<AQ_F16>(v);
+                else ((uint16_t*)y)[yi] = f32_to_bits<AQ_BF16>(v);
+            }
+        }
+        __syncthreads();
+        for (int e = tid; e < n; e += blockDim.x) counters[s_list[e]] = 0u;
     }
-    if (threadIdx.x == 0) counters[chunk] = 0u;
 }
 
 }  // namespace aq

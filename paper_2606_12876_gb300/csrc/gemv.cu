@@ -1,147 +1,299 @@
 // aq_gemv: y = x * W_m^T for 1..16 tokens, W_m the prefix-m additive reconstruction
 // (Sec. 3.2 group sums, restricted to the first m codebooks as in Sec. 5; Y = W X of Sec. 2.2).
 //
-// Work split (split-K): the grid is (row chunks) x (slices of 32 groups = 256 inputs). Each
-// CTA reads the first m code planes of its (slice, rows) region once, writes one fp32
-// partial per (row, token), and the last CTA of a row chunk sums the slices in order, scales
-// the row (R1: s[o] multiplies the codebook sum, so it factors out of the dot product) and
-// stores y.
+// Work split (split-K): the input dimension is cut into slices of 32 groups (256 inputs).
+// A work item is (slice, 32-row block). Each item reads the first m code planes of its rows
+// once and writes one fp32 partial per (row, token). When all slices of a 32-row block are
+// written, the CTA that counted the last one sums them in slice order (deterministic), scales
+// the rows and stores y (finish_items).
 //
-// Two kernels:
+// Two product kernels:
 //  * gemv_lut (B = 8, one token, m <= 4). By linearity, x_g . (sum_k C_k[b_k]) =
-//    sum_k T_k[g][b_k] with T_k[g][j] = x_g . C_k[j]. The CTA builds T for its 32 groups and
-//    m books in shared memory (32 KiB per book), then every code byte costs one shared-memory
-//    lookup and one fp32 add. Lane L owns row 32*rb+L; because each row's 32 codes are stored
+//    sum_k T_k[g][b_k] with T_k[g][j] = x_g . C_k[j]. A persistent CTA (one per SM) walks a
+//    contiguous range of work items; for each slice it builds T for the 32 groups and m books
+//    in shared memory (32 KiB per book), then every code byte costs one shared-memory lookup
+//    and one fp32 add. Lane L owns row 32*rb+L; because each row's 32 codes are stored
 //    rotated by the row index, at step p all 32 lanes look up 32 different groups, i.e. 32
 //    different banks, so the lookups are conflict-free and no cross-lane reduction is needed.
+//    One producer warp streams the code planes into a shared-memory ring with TMA bulk copies
+//    (the CTA's rows of a slice are contiguous in every plane), overlapping HBM reads with
+//    the table build and the lookups of the eight consumer warps.
 //  * gemv_direct (any B, 1..16 tokens). Decode each group in fp32 (sum of m codewords), then
 //    multiply by the tokens' 8 activations. Lane L owns row 32*rb+L and walks the 32 groups
 //    of the slice in a common order, so the activation loads are warp-uniform broadcasts.
+#include <map>
 #include <mutex>
+#include <tuple>
 
 #include "aq_internal.cuh"
 
 namespace aq {
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kWarps = kThreads / 32;
-
 // ------------------------------------------------------------------ LUT kernel (B = 8, b = 1)
 
-// Table layout: pairs of books share 256-byte rows, T[k/2][j][k%2][32 groups] (fp32), so the
-// byte offset of entry (k, j, g) is (k/2)*65536 + j*256 + (k%2)*128 + g*4 and j*256 + g*4 is
-// produced from a code byte by one prmt.
-template <int MM, int BDT, int XDT, int SDT>
-__global__ void __launch_bounds__(kThreads)
+constexpr int kCons = 16;                         // consumer warps (one 32-row block each per stage)
+constexpr int kLutThreads = (kCons + 1) * 32;     // + one producer warp
+constexpr int kStageRb = 16;                      // 32-row blocks per stage: a 16 KiB plane copy
+constexpr int kSlot = kStageRb * 1024;            // one ring slot = one plane of one stage
+constexpr int kSlots = 8;                         // largest ring depth (128 KiB)
+constexpr int kXSlices = 8;                       // activation slices staged up front
+constexpr int kTBytes = 65536;                    // table of one book pair
+constexpr int kLutMaxM = 8;
+
+// Shared memory: [T 64 KiB][codebooks m x 4 KiB][activations 8 x 512 B][ring][barriers]
+inline size_t lut_smem_bytes(int m, int slots) {
+    return (size_t)kTBytes + (size_t)m * 4096 + kXSlices * 512 + (size_t)slots * kSlot +
+           2 * kSlots * 8;
+}
+
+// The m books are processed in passes of at most two (pass p: books 2p, 2p+1), so the table
+// never exceeds 64 KiB: T[j][k%2][32 groups] (fp32), entry (k, j, g) at byte
+// j*256 + (k%2)*128 + g*4; j*256 + g*4 is produced from a code byte by one prmt.
+//
+// A CTA owns the items [i0, i1) (item = slice * RBc + 32-row block). In every pass it walks
+// them in stages of up to 16 items that never cross a slice. For each stage and each book of
+// the pass the producer warp copies the stage's rows of that book's plane into one ring slot
+// with a TMA bulk copy (16 KiB; the CTA's rows of a slice are contiguous in every plane), and
+// consumer warp w looks up item w of the stage. A row's sum over the pass's books stays in a
+// register; pass 0 stores it as the fp32 partial and later passes add to it. The codebooks
+// and the activations of the CTA's first slices are requested before any code.
+template <int BDT, int XDT, int SDT>
+__global__ void __launch_bounds__(kLutThreads, 1)
 gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
                 const uint16_t* __restrict__ x, const uint16_t* __restrict__ scales,
-                float* __restrict__ partials, unsigned int* __restrict__ counters, void* y,
-                int y_dt, int out, int ng, int rows_pad, int S, int RBc, int rb_per_chunk,
-                size_t plane_bytes) {
-    constexpr int NP = (MM + 1) / 2;
-    extern __shared__ __align__(16) unsigned char smem[];
-    unsigned char* T = smem;                                   // NP * 64 KiB
-    float* Cf = (float*)(smem + NP * 65536);                   // [MM][256][8] fp32
+                float* __restrict__ partials, unsigned int* __restrict__ counters,
+                unsigned int* __restrict__ status, void* y, int y_dt, int m, int out, int in,
+                int ng, int rows_pad, int RBc, int S, long long total_items, size_t plane_bytes,
+                int nslots, int cps) {
+    extern __shared__ __align__(128) unsigned char smem[];
+    unsigned char* T = smem;
+    uint4* Cb = (uint4*)(smem + kTBytes);                          // [m][256] codewords
+    unsigned char* xs = smem + kTBytes + (size_t)m * 4096;         // [kXSlices][256] activations
+    unsigned char* ring = xs + kXSlices * 512;                     // nslots x 16 KiB
+    uint64_t* full = (uint64_t*)(ring + (size_t)nslots * kSlot);
+    uint64_t* empty = full + kSlots;
+    __shared__ volatile int s_abort;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int s = blockIdx.y, chunk = blockIdx.x;
-
-    // Stage the first MM codebooks as fp32.
-    for (int i = tid; i < MM * 256; i += kThreads) {
-        const uint4 v = __ldg((const uint4*)books + i);
-        float f[8];
-        unpack8<BDT>(v, f);
-        float4* d = (float4*)(Cf + (size_t)i * 8);
-        d[0] = make_float4(f[0], f[1], f[2], f[3]);
-        d[1] = make_float4(f[4], f[5], f[6], f[7]);
+    // Item range of this CTA: slice-aligned (cps CTAs per slice) or balanced over the grid.
+    long long i0, i1;
+    if (cps > 0) {
+        const int s = blockIdx.x / cps, c = blockIdx.x % cps;
+        i0 = (long long)s * RBc + (long long)c * RBc / cps;
+        i1 = (long long)s * RBc + (long long)(c + 1) * RBc / cps;
+    } else {
+        i0 = (long long)blockIdx.x * total_items / gridDim.x;
+        i1 = (long long)(blockIdx.x + 1) * total_items / gridDim.x;
     }
-    // Activations of group s*32+lane (zero for padding groups).
-    float xv[8];
-    {
-        const int g = s * 32 + lane;
-        if (g < ng) {
-            unpack8<XDT>(__ldg((const uint4*)x + g), xv);
-        } else {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) xv[e] = 0.0f;
+    const int s_first = (int)(i0 / RBc);
+    const int npass = (m + 1) / 2;
+
+    if (tid == 0) {
+        for (int d = 0; d < nslots; ++d) {
+            mbar_init(&full[d], 1);
+            mbar_init(&empty[d], kCons);
         }
+        mbar_fence_init();
+        s_abort = 0;
+    }
+    pdl_wait();                 // inputs may come from the preceding kernel in the stream
+
+    // Codebooks and activations are requested first (into registers); the producer starts
+    // its copies only after every thread has issued these loads (the barrier below).
+    // (consumer threads only: they are the ones that store the codebooks below)
+    uint4 cb_r[4];
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+        const int i = tid + r * kCons * 32;
+        cb_r[r] = (tid < kCons * 32 && i < m * 256) ? __ldg((const uint4*)books + i)
+                                                      : make_uint4(0u, 0u, 0u, 0u);
+    }
+    uint2 x_r = make_uint2(0u, 0u);
+    if (tid < kXSlices * 64) {
+        const int col = (s_first + (tid >> 6)) * 256 + (tid & 63) * 4;
+        if (col < in) x_r = __ldg((const uint2*)(x + col));
     }
     __syncthreads();
 
-    // T_k[j][lane] = x_{s*32+lane} . C_k[j]
-    for (int j = warp; j < 256; j += kWarps) {
-#pragma unroll
-        for (int k = 0; k < MM; ++k) {
-            const float4 c0 = *(const float4*)(Cf + ((size_t)k * 256 + j) * 8);
-            const float4 c1 = *(const float4*)(Cf + ((size_t)k * 256 + j) * 8 + 4);
-            float t = xv[0] * c0.x;
-            t = fmaf(xv[1], c0.y, t);
-            t = fmaf(xv[2], c0.z, t);
-            t = fmaf(xv[3], c0.w, t);
-            t = fmaf(xv[4], c1.x, t);
-            t = fmaf(xv[5], c1.y, t);
-            t = fmaf(xv[6], c1.z, t);
-            t = fmaf(xv[7], c1.w, t);
-            *(float*)(T + (k >> 1) * 65536 + j * 256 + (k & 1) * 128 + lane * 4) = t;
-        }
-    }
-    __syncthreads();
+    // Stage sequence shared by the producer and the consumers: pass, then items in order,
+    // cut at slice boundaries and at 16 items; one ring slot per (stage, book of the pass).
+    auto stage_len = [&](long long it) {
+        const long long slice_end = (it / RBc + 1) * RBc;
+        return (int)min((long long)kStageRb, min(i1, slice_end) - it);
+    };
 
-    // goff[q] byte i = 4 * group-in-slice read at position 4q+i by this lane: (4q+i+lane) mod 32.
-    uint32_t goff[8];
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-        uint32_t v = 0;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) v |= (uint32_t)(((4 * q + i + lane) & 31) * 4) << (8 * i);
-        goff[q] = v;
-    }
-
-    const int rb0 = chunk * rb_per_chunk;
-    const int rb1 = min(rb0 + rb_per_chunk, RBc);
-    for (int rb = rb0 + warp; rb < rb1; rb += kWarps) {
-        const int o = rb * 32 + lane;
-        uint4 cw[MM][2];
-#pragma unroll
-        for (int k = 0; k < MM; ++k) {
-            const uint8_t* src = planes + k * plane_bytes + ((size_t)s * rows_pad + o) * 32;
-            cw[k][0] = ld_stream_v4(src);
-            cw[k][1] = ld_stream_v4(src + 16);
+    if (warp == kCons) {
+        // ---- producer (lane 0 issues; the warp stays converged for the final barriers)
+        if (lane == 0) {
+            int q = 0;
+            for (int pass = 0; pass < npass; ++pass) {
+                const int mp = min(2, m - 2 * pass);
+                for (long long it = i0; it < i1;) {
+                    const int n = stage_len(it);
+                    const size_t src =
+                        ((size_t)(it / RBc) * rows_pad + (size_t)(it % RBc) * 32) * 32;
+                    for (int k = 0; k < mp; ++k, ++q) {
+                        const int slot = q % nslots;
+                        if (s_abort) break;
+                        if (q >= nslots && !mbar_wait(&empty[slot], ((q / nslots) - 1) & 1)) {
+                            record_status(status, AQ_ERR_TIMEOUT);
+                            s_abort = 1;
+                            break;
+                        }
+                        mbar_arrive_expect_tx(&full[slot], (uint32_t)(n * 1024));
+                        bulk_g2s(ring + (size_t)slot * kSlot,
+                                 planes + (size_t)(2 * pass + k) * plane_bytes + src,
+                                 (uint32_t)(n * 1024), &full[slot]);
+                    }
+                    it += n;
+                }
+            }
+            // No copy may be in flight when the CTA exits (bounded wait on the last slots).
+            for (int j = max(0, q - nslots); j < q; ++j) mbar_wait(&full[j % nslots], (j / nslots) & 1);
         }
-        float acc = 0.0f;
+        __syncwarp();
+    } else {
+        // ---- consumers
 #pragma unroll
-        for (int k = 0; k < MM; ++k) {
-            const unsigned char* Tk = T + (k >> 1) * 65536 + (k & 1) * 128;
-            const uint32_t wd[8] = {cw[k][0].x, cw[k][0].y, cw[k][0].z, cw[k][0].w,
-                                    cw[k][1].x, cw[k][1].y, cw[k][1].z, cw[k][1].w};
+        for (int r = 0; r < 4; ++r) {
+            const int i = tid + r * kCons * 32;
+            if (i < m * 256) Cb[i] = cb_r[r];
+        }
+        if (tid < kXSlices * 64) *(uint2*)(xs + (tid >> 6) * 512 + (tid & 63) * 8) = x_r;
+        named_barrier(1, kCons * 32);   // staged codebooks and activations visible to all consumers
+
+        // goff[q] byte i = 4 * group-in-slice read at position 4q+i by this lane.
+        uint32_t goff[8];
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                // byte0 = goff byte i, byte1 = code byte i, bytes 2-3 = sign of goff byte (0)
-                acc += *(const float*)(Tk + prmt(wd[q], goff[q], 0xCC04u));
-                acc += *(const float*)(Tk + prmt(wd[q], goff[q], 0xDD15u));
-                acc += *(const float*)(Tk + prmt(wd[q], goff[q], 0xEE26u));
-                acc += *(const float*)(Tk + prmt(wd[q], goff[q], 0xFF37u));
+        for (int q = 0; q < 8; ++q) {
+            uint32_t v = 0;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) v |= (uint32_t)(((4 * q + i + lane) & 31) * 4) << (8 * i);
+            goff[q] = v;
+        }
+
+        int q = 0;
+        for (int pass = 0; pass < npass; ++pass) {
+            const int mp = min(2, m - 2 * pass);
+            int cur_s = -1;
+            for (long long it = i0; it < i1;) {
+                const int n = stage_len(it);
+                const int s = (int)(it / RBc), rb = (int)(it % RBc);
+                if (s != cur_s) {
+                    // Table of the pass's books for slice s. Lane L = 8*ph + gq computes groups
+                    // 4gq..4gq+3 for codewords j = 16*warp + ph + 4i: one 16-byte codeword read
+                    // serves four entries, stored as one 16-byte piece.
+                    const int ph = lane >> 3, gq = lane & 7, sl = s - s_first;
+                    float2 xv[4][4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int g = s * 32 + gq * 4 + u;
+                        uint4 xr = make_uint4(0u, 0u, 0u, 0u);
+                        if (sl < kXSlices) xr = *(const uint4*)(xs + sl * 512 + (gq * 4 + u) * 16);
+                        else if (g < ng) xr = __ldg((const uint4*)x + g);
+                        float f[8];
+                        unpack8<XDT>(xr, f);
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) xv[u][e] = make_float2(f[2 * e], f[2 * e + 1]);
+                    }
+                    named_barrier(1, kCons * 32);   // old table no longer read; Cb / xs staged
+                    for (int k = 0; k < mp; ++k) {
+                        const int kb = 2 * pass + k;
+                        unsigned char* Tk = T + k * 128 + gq * 16;
+                        uint4 cw[4];
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) cw[i] = Cb[kb * 256 + warp * 16 + ph + 4 * i];
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            float c[8];
+                            unpack8<BDT>(cw[i], c);
+                            float r[4];
+#pragma unroll
+                            for (int u = 0; u < 4; ++u) {
+                                float2 t = make_float2(xv[u][0].x * c[0], xv[u][0].y * c[1]);
+                                t = ffma2(xv[u][1], make_float2(c[2], c[3]), t);
+                                t = ffma2(xv[u][2], make_float2(c[4], c[5]), t);
+                                t = ffma2(xv[u][3], make_float2(c[6], c[7]), t);
+                                r[u] = t.x + t.y;
+                            }
+                            *(float4*)(Tk + (warp * 16 + ph + 4 * i) * 256) =
+                                make_float4(r[0], r[1], r[2], r[3]);
+                        }
+                    }
+                    named_barrier(1, kCons * 32);
+                    cur_s = s;
+                }
+                float part = 0.0f;
+                for (int k = 0; k < mp; ++k, ++q) {
+                    const int slot = q % nslots;
+                    bool ok = !s_abort;
+                    if (ok && !mbar_wait(&full[slot], (q / nslots) & 1)) {
+                        record_status(status, AQ_ERR_TIMEOUT);
+                        s_abort = 1;
+                        ok = false;
+                    }
+                    if (ok && warp < n) {
+                        // Lanes 4-7 of each group of eight read their two 16-byte halves in the
+                        // other order, which keeps the two reads free of bank conflicts.
+                        const uint4* src = (const uint4*)(ring + (size_t)slot * kSlot + warp * 1024 + lane * 32);
+                        const int c0 = (lane >> 2) & 1;
+                        const uint4 r0 = src[c0], r1 = src[c0 ^ 1];
+                        const uint4 a = c0 ? r1 : r0, b = c0 ? r0 : r1;
+                        const uint32_t wd[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+                        const uint32_t Tk = smem_u32(T) + k * 128;
+                        float acc[8];
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            uint32_t off[16];
+#pragma unroll
+                            for (int qq = 0; qq < 4; ++qq) {
+                                // byte0 = goff byte i, byte1 = code byte i, bytes 2-3 = sign of goff byte (0)
+                                const uint32_t w = wd[4 * h + qq], g = goff[4 * h + qq];
+                                off[4 * qq + 0] = prmt(w, g, 0xCC04u);
+                                off[4 * qq + 1] = prmt(w, g, 0xDD15u);
+                                off[4 * qq + 2] = prmt(w, g, 0xEE26u);
+                                off[4 * qq + 3] = prmt(w, g, 0xFF37u);
+                            }
+                            float v[16];
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) v[i] = lds_f32(Tk + off[i]);
+#pragma unroll
+                            for (int qq = 0; qq < 4; ++qq)
+                                acc[4 * h + qq] = (v[4 * qq] + v[4 * qq + 1]) + (v[4 * qq + 2] + v[4 * qq + 3]);
+                        }
+                        part += ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+                    }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&empty[slot]);
+                }
+                if (!s_abort && warp < n) {
+                    float* dst = partials + (size_t)s * rows_pad + (size_t)(rb + warp) * 32 + lane;
+                    if (pass > 0) part += *dst;     // this thread wrote it in the previous pass
+                    *dst = part;
+                }
+                it += n;
             }
         }
-        partials[(size_t)s * rows_pad + o] = acc;
     }
-    splitk_finish<SDT>(counters, partials, scales, y, y_dt, out, rows_pad, S, 1, chunk,
-                       rb0 * 32, rb1 * 32);
+    pdl_launch_dependents();
+    finish_items<SDT>(i1 - i0, [&](long long j) { return (int)((i0 + j) % RBc); }, counters,
+                      partials, scales, y, y_dt, out, rows_pad, S, 1);
 }
 
 // ------------------------------------------------------------------ direct kernel (any B, b <= 16)
 
 template <int NB, int B, int BDT, int SDT>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(256)
 gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
                    const uint16_t* __restrict__ x, int x_dt, const uint16_t* __restrict__ scales,
                    float* __restrict__ partials, unsigned int* __restrict__ counters, void* y,
-                   int y_dt, int m, int batch, int out, int in, int ng, int rows_pad, int S,
-                   int RBc, int rb_per_chunk, size_t plane_bytes) {
+                   int y_dt, int out, int m, int batch, int in, int rows_pad, int RBc, int S,
+                   int rb_per_chunk, size_t plane_bytes) {
     constexpr int ESZ = B / 8;
     constexpr int UNIT = 32 * ESZ;
-    extern __shared__ __align__(16) unsigned char smem[];
+    constexpr int kWarps = 8;
+    extern __shared__ __align__(128) unsigned char smem[];
     float* xs = (float*)smem;                                        // [NB][256]
     uint16_t* books_s = (uint16_t*)(smem + NB * 1024);               // B = 8: [m][256][8]
     const size_t books_bytes = (B == 8) ? (size_t)m * 4096 : 0;
@@ -149,7 +301,8 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
     unsigned char* codes_s = smem + NB * 1024 + books_bytes + (size_t)warp * m * 32 * UNIT;
     const int s = blockIdx.y, chunk = blockIdx.x;
 
-    for (int i = tid; i < NB * 256; i += kThreads) {
+    pdl_wait();
+    for (int i = tid; i < NB * 256; i += 256) {
         const int t = i >> 8, c = i & 255;
         const int col = s * 256 + c;
         float v = 0.0f;
@@ -157,7 +310,7 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
         xs[i] = v;
     }
     if constexpr (B == 8) {
-        for (int i = tid; i < m * 256; i += kThreads)
+        for (int i = tid; i < m * 256; i += 256)
             ((uint4*)books_s)[i] = __ldg((const uint4*)books + i);
     }
     __syncthreads();
@@ -214,123 +367,144 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
         for (int t = 0; t < NB; ++t)
             if (t < batch) partials[((size_t)s * batch + t) * rows_pad + o] = acc[t];
     }
-    splitk_finish<SDT>(counters, partials, scales, y, y_dt, out, rows_pad, S, batch, chunk,
-                       rb0 * 32, rb1 * 32);
+    pdl_launch_dependents();
+    finish_items<SDT>(max(rb1 - rb0, 0), [&](long long j) { return rb0 + (int)j; }, counters,
+                      partials, scales, y, y_dt, out, rows_pad, S, batch);
 }
 
 // ------------------------------------------------------------------ host side
 
-struct Grid {
-    int chunks, rb_per_chunk;
-};
-
-Grid plan_grid(const Dims& d, int sms, int ctas_per_sm) {
-    const int target = sms * (ctas_per_sm > 0 ? ctas_per_sm : 1);
-    int chunks = (target + d.S - 1) / d.S;
-    if (chunks < 1) chunks = 1;
-    if (chunks > d.RBc) chunks = d.RBc;
-    const int rbpc = (d.RBc + chunks - 1) / chunks;
-    return Grid{(d.RBc + rbpc - 1) / rbpc, rbpc};
+// Launch with the programmatic-stream-serialization attribute (PDL), so the kernel's CTAs may
+// become resident while the preceding kernel in the stream drains; every kernel launched this
+// way calls griddepcontrol.wait before it reads anything another kernel may have written.
+template <typename... KArgs, typename... Args>
+aq_status launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                     Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cuda_ok(cudaLaunchKernelEx(&cfg, kern, (KArgs)args...), "cudaLaunchKernelEx");
 }
 
 // Raises the kernel's dynamic shared-memory limit and returns its occupancy. Both are cached
 // per (kernel, device, slot), slot being the prefix m where the shared-memory size depends on
 // it, so the CUDA attribute calls happen once, before any stream capture that later calls
 // reuse.
-struct PrepCache {
-    std::mutex mu;
-    int occ[64][9] = {};
-};
-
 template <typename K>
-aq_status prepare(K kern, size_t smem, int slot, int* ctas_per_sm) {
-    static PrepCache cache;
+aq_status prepare(K kern, size_t smem, int threads, int slot, int* ctas_per_sm) {
+    static std::mutex mu;
+    static std::map<std::tuple<const void*, int, int>, int> cache;
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64 || slot < 0 || slot > 8)
-        return AQ_ERR_CUDA;
-    std::lock_guard<std::mutex> lock(cache.mu);
-    if (cache.occ[dev][slot] > 0) {
-        *ctas_per_sm = cache.occ[dev][slot];
+    if (cudaError_t e = cudaGetDevice(&dev); e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    const auto key = std::make_tuple((const void*)kern, dev, slot);
+    std::lock_guard<std::mutex> lock(mu);
+    if (auto it = cache.find(key); it != cache.end()) {
+        *ctas_per_sm = it->second;
         return AQ_OK;
     }
     DeviceInfo di;
-    if (device_info(&di) != AQ_OK) return AQ_ERR_CUDA;
+    if (aq_status e = device_info(&di); e != AQ_OK) return e;
     cudaFuncAttributes fa;
-    if (cudaFuncGetAttributes(&fa, kern) != cudaSuccess) return AQ_ERR_CUDA;
+    if (cudaError_t e = cudaFuncGetAttributes(&fa, kern); e != cudaSuccess)
+        return cuda_fail(e, "cudaFuncGetAttributes");
     const int dyn_max = di.smem_optin - (int)fa.sharedSizeBytes;
     if ((int)smem > dyn_max) return AQ_ERR_UNSUPPORTED;
     // Allow the largest size any slot of this kernel may need (the attribute is per kernel).
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn_max) !=
-        cudaSuccess)
-        return AQ_ERR_CUDA;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, kern, kThreads, smem) != cudaSuccess)
-        return AQ_ERR_CUDA;
+    if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             dyn_max);
+        e != cudaSuccess)
+        return cuda_fail(e, "cudaFuncSetAttribute");
+    // Every kernel of the library asks for the same (largest) shared-memory carve-out, so
+    // consecutive launches never force an SM to re-split its L1 / shared-memory storage.
+    if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                             (int)cudaSharedmemCarveoutMaxShared);
+        e != cudaSuccess)
+        return cuda_fail(e, "cudaFuncSetAttribute");
+    if (cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, kern, threads,
+                                                                      smem);
+        e != cudaSuccess)
+        return cuda_fail(e, "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
     if (*ctas_per_sm < 1) return AQ_ERR_UNSUPPORTED;
-    cache.occ[dev][slot] = *ctas_per_sm;
+    cache[key] = *ctas_per_sm;
     return AQ_OK;
 }
 
-template <int MM, int BDT, int XDT, int SDT>
-aq_status run_lut(const Dims& d, const void* planes, const void* books, const void* scales,
-                  const void* x, void* y, int y_dt, void* ws, cudaStream_t st) {
+struct GemvArgs {
+    const void *planes, *books, *scales, *x;
+    int x_dt, batch;
+    void* y;
+    int y_dt;
+    float* partials;
+    unsigned int* counters;
+    unsigned int* status;
+};
+
+template <int BDT, int XDT, int SDT>
+aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     DeviceInfo di;
-    if (device_info(&di) != AQ_OK) return AQ_ERR_CUDA;
-    const size_t smem = (size_t)((MM + 1) / 2) * 65536 + (size_t)MM * 8192;
-    auto kern = gemv_lut_kernel<MM, BDT, XDT, SDT>;
+    if (aq_status e = device_info(&di); e != AQ_OK) return e;
+    auto kern = gemv_lut_kernel<BDT, XDT, SDT>;
+    // As many 16 KiB ring slots as fit next to the table, codebooks and activations (<= 8).
+    const size_t fixed = lut_smem_bytes(m, 0) + 8192;   // + static shared memory and slack
+    int nslots = di.smem_optin > (int)fixed ? (int)((di.smem_optin - fixed) / kSlot) : 0;
+    if (nslots > kSlots) nslots = kSlots;
+    if (nslots < 2) return AQ_ERR_UNSUPPORTED;
+    const size_t smem = lut_smem_bytes(m, nslots);
     int occ = 0;
-    if (aq_status e = prepare(kern, smem, 0, &occ); e != AQ_OK) return e;
-    const Grid g = plan_grid(d, di.sms, occ);
-    unsigned int* counters = (unsigned int*)((char*)ws + kWsStatusBytes);
-    float* partials = (float*)((char*)ws + ws_partial_offset(d));
-    kern<<<dim3(g.chunks, d.S), kThreads, smem, st>>>(
-        (const uint8_t*)planes, (const uint16_t*)books, (const uint16_t*)x,
-        (const uint16_t*)scales, partials, counters, y, y_dt, d.out, d.ng, d.rows_pad, d.S,
-        d.RBc, g.rb_per_chunk, d.plane_bytes);
-    return cudaGetLastError() == cudaSuccess ? AQ_OK : AQ_ERR_CUDA;
+    if (aq_status e = prepare(kern, smem, kLutThreads, m, &occ); e != AQ_OK) return e;
+    const long long items = (long long)d.S * d.RBc;
+    // One CTA per SM. If whole slices per CTA keep at least 90% of the SMs busy, every CTA
+    // gets a single slice (one table build per book); otherwise items are balanced evenly
+    // and a CTA may span two slices.
+    int cps = di.sms / d.S;
+    if (cps > d.RBc) cps = d.RBc;
+    int grid;
+    if (cps >= 1 && (long long)cps * d.S * 10 >= (long long)di.sms * 9) {
+        grid = cps * d.S;
+    } else {
+        cps = 0;
+        grid = (int)(items < di.sms ? items : di.sms);
+    }
+    return launch_pdl(kern, dim3(grid), dim3(kLutThreads), smem, st, (const uint8_t*)a.planes,
+                      (const uint16_t*)a.books, (const uint16_t*)a.x, (const uint16_t*)a.scales,
+                      a.partials, a.counters, a.status, a.y, a.y_dt, m, d.out, d.in, d.ng,
+                      d.rows_pad, d.RBc, d.S, items, d.plane_bytes, nslots, cps);
 }
 
 template <int NB, int B, int BDT, int SDT>
-aq_status run_direct(const Dims& d, int m, const void* planes, const void* books,
-                     const void* scales, const void* x, int x_dt, int batch, void* y, int y_dt,
-                     void* ws, cudaStream_t st) {
+aq_status run_direct(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     DeviceInfo di;
-    if (device_info(&di) != AQ_OK) return AQ_ERR_CUDA;
+    if (aq_status e = device_info(&di); e != AQ_OK) return e;
     const size_t smem = (size_t)NB * 1024 + (B == 8 ? (size_t)m * 4096 : 0) +
-                        (size_t)kWarps * m * 32 * 32 * (B / 8);
+                        (size_t)8 * m * 32 * 32 * (B / 8);
     auto kern = gemv_direct_kernel<NB, B, BDT, SDT>;
     int occ = 0;
-    if (aq_status e = prepare(kern, smem, m, &occ); e != AQ_OK) return e;
-    const Grid g = plan_grid(d, di.sms, occ);
-    unsigned int* counters = (unsigned int*)((char*)ws + kWsStatusBytes);
-    float* partials = (float*)((char*)ws + ws_partial_offset(d));
-    kern<<<dim3(g.chunks, d.S), kThreads, smem, st>>>(
-        (const uint8_t*)planes, (const uint16_t*)books, (const uint16_t*)x, x_dt,
-        (const uint16_t*)scales, partials, counters, y, y_dt, m, batch, d.out, d.in, d.ng,
-        d.rows_pad, d.S, d.RBc, g.rb_per_chunk, d.plane_bytes);
-    return cudaGetLastError() == cudaSuccess ? AQ_OK : AQ_ERR_CUDA;
-}
-
-template <int BDT, int XDT, int SDT>
-aq_status dispatch_lut(const Dims& d, int m, const void* planes, const void* books,
-                       const void* scales, const void* x, void* y, int y_dt, void* ws,
-                       cudaStream_t st) {
-    switch (m) {
-        case 1: return run_lut<1, BDT, XDT, SDT>(d, planes, books, scales, x, y, y_dt, ws, st);
-        case 2: return run_lut<2, BDT, XDT, SDT>(d, planes, books, scales, x, y, y_dt, ws, st);
-        case 3: return run_lut<3, BDT, XDT, SDT>(d, planes, books, scales, x, y, y_dt, ws, st);
-        default: return run_lut<4, BDT, XDT, SDT>(d, planes, books, scales, x, y, y_dt, ws, st);
-    }
+    if (aq_status e = prepare(kern, smem, 256, m, &occ); e != AQ_OK) return e;
+    const int target = di.sms * occ;
+    int chunks = (target + d.S - 1) / d.S;
+    chunks = chunks < 1 ? 1 : (chunks > d.RBc ? d.RBc : chunks);
+    const int rbpc = (d.RBc + chunks - 1) / chunks;
+    chunks = (d.RBc + rbpc - 1) / rbpc;
+    return launch_pdl(kern, dim3(chunks, d.S), dim3(256), smem, st, (const uint8_t*)a.planes,
+                      (const uint16_t*)a.books, (const uint16_t*)a.x, a.x_dt,
+                      (const uint16_t*)a.scales, a.partials, a.counters, a.y, a.y_dt, d.out, m,
+                      a.batch, d.in, d.rows_pad, d.RBc, d.S, rbpc, d.plane_bytes);
 }
 
 template <int B, int BDT, int SDT>
-aq_status dispatch_direct(const Dims& d, int m, const void* planes, const void* books,
-                          const void* scales, const void* x, int x_dt, int batch, void* y,
-                          int y_dt, void* ws, cudaStream_t st) {
-    if (batch <= 1) return run_direct<1, B, BDT, SDT>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
-    if (batch <= 2) return run_direct<2, B, BDT, SDT>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
-    if (batch <= 4) return run_direct<4, B, BDT, SDT>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
-    if (batch <= 8) return run_direct<8, B, BDT, SDT>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
-    return run_direct<16, B, BDT, SDT>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
+aq_status dispatch_direct(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
+    if (a.batch <= 1) return run_direct<1, B, BDT, SDT>(d, m, a, st);
+    if (a.batch <= 2) return run_direct<2, B, BDT, SDT>(d, m, a, st);
+    if (a.batch <= 4) return run_direct<4, B, BDT, SDT>(d, m, a, st);
+    if (a.batch <= 8) return run_direct<8, B, BDT, SDT>(d, m, a, st);
+    return run_direct<16, B, BDT, SDT>(d, m, a, st);
 }
 
 }  // namespace
@@ -339,30 +513,31 @@ aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* book
                       const void* scales, const void* x, int x_dt, int batch, void* y,
                       int y_dt, void* ws, cudaStream_t st) {
     if (d.out == 0 || batch == 0) return AQ_OK;
-    const bool bb = d.book_dt == AQ_BF16, sb = d.scale_dt == AQ_BF16, xb = x_dt == AQ_BF16;
-    if (d.B == 8 && batch == 1 && m <= 4) {
-        const int key = bb * 4 + xb * 2 + sb;
-        switch (key) {
-            case 0: return dispatch_lut<AQ_F16, AQ_F16, AQ_F16>(d, m, planes, books, scales, x, y, y_dt, ws, st);
-            case 1: return dispatch_lut<AQ_F16, AQ_F16, AQ_BF16>(d, m, planes, books, scales, x, y, y_dt, ws, st);
-            case 2: return dispatch_lut<AQ_F16, AQ_BF16, AQ_F16>(d, m, planes, books, scales, x, y, y_dt, ws, st);
-            case 3: return dispatch_lut<AQ_F16, AQ_BF16, AQ_BF16>(d, m, planes, books, scales, x, y, y_dt, ws, st);
-            case 4: return dispatch_lut<AQ_BF16, AQ_F16, AQ_F16>(d, m, planes, books, scales, x, y, y_dt, ws, st);
-            case 5: return dispatch_lut<AQ_BF16, AQ_F16, AQ_BF16>(d, m, planes, books, scales, x, y, y_dt, ws, st);
-            case 6: return dispatch_lut<AQ_BF16, AQ_BF16, AQ_F16>(d, m, planes, books, scales, x, y, y_dt, ws, st);
-            default: return dispatch_lut<AQ_BF16, AQ_BF16, AQ_BF16>(d, m, planes, books, scales, x, y, y_dt, ws, st);
+    GemvArgs a{planes, books, scales, x, x_dt, batch, y, y_dt,
+               (float*)((char*)ws + ws_partial_offset(d)),
+               (unsigned int*)((char*)ws + kWsStatusBytes), (unsigned int*)ws};
+    const int bb = d.book_dt == AQ_BF16, xb = x_dt == AQ_BF16, sb = d.scale_dt == AQ_BF16;
+    if (d.B == 8 && batch == 1 && m <= kLutMaxM) {
+        switch (bb * 4 + xb * 2 + sb) {
+            case 0: return run_lut<AQ_F16, AQ_F16, AQ_F16>(d, m, a, st);
+            case 1: return run_lut<AQ_F16, AQ_F16, AQ_BF16>(d, m, a, st);
+            case 2: return run_lut<AQ_F16, AQ_BF16, AQ_F16>(d, m, a, st);
+            case 3: return run_lut<AQ_F16, AQ_BF16, AQ_BF16>(d, m, a, st);
+            case 4: return run_lut<AQ_BF16, AQ_F16, AQ_F16>(d, m, a, st);
+            case 5: return run_lut<AQ_BF16, AQ_F16, AQ_BF16>(d, m, a, st);
+            case 6: return run_lut<AQ_BF16, AQ_BF16, AQ_F16>(d, m, a, st);
+            default: return run_lut<AQ_BF16, AQ_BF16, AQ_BF16>(d, m, a, st);
         }
     }
-    const int key = (d.B == 16) * 4 + bb * 2 + sb;
-    switch (key) {
-        case 0: return dispatch_direct<8, AQ_F16, AQ_F16>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
-        case 1: return dispatch_direct<8, AQ_F16, AQ_BF16>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
-        case 2: return dispatch_direct<8, AQ_BF16, AQ_F16>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
-        case 3: return dispatch_direct<8, AQ_BF16, AQ_BF16>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
-        case 4: return dispatch_direct<16, AQ_F16, AQ_F16>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
-        case 5: return dispatch_direct<16, AQ_F16, AQ_BF16>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
-        case 6: return dispatch_direct<16, AQ_BF16, AQ_F16>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
-        default: return dispatch_direct<16, AQ_BF16, AQ_BF16>(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
+    switch ((d.B == 16) * 4 + bb * 2 + sb) {
+        case 0: return dispatch_direct<8, AQ_F16, AQ_F16>(d, m, a, st);
+        case 1: return dispatch_direct<8, AQ_F16, AQ_BF16>(d, m, a, st);
+        case 2: return dispatch_direct<8, AQ_BF16, AQ_F16>(d, m, a, st);
+        case 3: return dispatch_direct<8, AQ_BF16, AQ_BF16>(d, m, a, st);
+        case 4: return dispatch_direct<16, AQ_F16, AQ_F16>(d, m, a, st);
+        case 5: return dispatch_direct<16, AQ_F16, AQ_BF16>(d, m, a, st);
+        case 6: return dispatch_direct<16, AQ_BF16, AQ_F16>(d, m, a, st);
+        default: return dispatch_direct<16, AQ_BF16, AQ_BF16>(d, m, a, st);
     }
 }
 

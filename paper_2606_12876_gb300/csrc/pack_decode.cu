@@ -107,14 +107,16 @@ aq_status run_decode(const Dims& d, int m, const void* planes, const void* books
                      const void* scales, void* w, cudaStream_t st) {
     const size_t smem = (B == 8 ? (size_t)m * 4096 : 0) + (size_t)kDecWarps * m * 32 * 32 * (B / 8);
     auto kern = decode_kernel<B, BDT, SDT>;
-    if (smem > 48 * 1024 &&
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
-        return AQ_ERR_CUDA;
+    if (smem > 48 * 1024)
+        if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)smem);
+            e != cudaSuccess)
+            return cuda_fail(e, "cudaFuncSetAttribute");
     dim3 grid((d.RBc + kDecWarps - 1) / kDecWarps, d.S);
     kern<<<grid, kDecWarps * 32, smem, st>>>((const uint8_t*)planes, (const uint16_t*)books,
                                              (const uint16_t*)scales, (uint16_t*)w, m, d.out,
                                              d.in, d.ng, d.rows_pad, d.RBc, d.plane_bytes);
-    return cudaGetLastError() == cudaSuccess ? AQ_OK : AQ_ERR_CUDA;
+    return cuda_ok(cudaGetLastError(), "kernel launch");
 }
 
 }  // namespace
@@ -132,7 +134,7 @@ aq_status launch_pack(const Dims& d, const void* codes, void* planes, cudaStream
         pack_kernel<uint16_t><<<blocks, threads, 0, st>>>((const uint16_t*)codes,
                                                           (uint16_t*)planes, d.out, d.ng, d.M,
                                                           d.rows_pad, d.S, total);
-    return cudaGetLastError() == cudaSuccess ? AQ_OK : AQ_ERR_CUDA;
+    return cuda_ok(cudaGetLastError(), "kernel launch");
 }
 
 aq_status launch_decode(const Dims& d, int m, const void* planes, const void* books,
