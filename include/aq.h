@@ -123,6 +123,28 @@ aq_status aq_gemv(const aq_layout* layout, int m, const void* planes, const void
                   const void* scales, const void* x, int x_dtype, int batch, void* y,
                   int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
 
+/* ---------------------------------------------------------------- GEMV without a workspace
+ * (This entry point has no counterpart in the paper.) The GEMV of aq_gemv for callers that
+ * cannot allocate device memory when they run a layer, and so cannot pass a workspace: for
+ * example a plugin inside a host program that owns all device memory and offers no
+ * allocator, or a serving loop that must not allocate after start-up because an allocation
+ * can synchronise the device or fail under memory pressure. Nothing is allocated: the scratch
+ * comes from a fixed AQ_STATIC_SCRATCH_BYTES buffer that the library holds, as a device
+ * array, on every GPU that loads it, until the process exits.
+ *   - Arguments and results are those of aq_gemv (same checks, same status codes).
+ *   - Returns AQ_ERR_WORKSPACE when aq_gemv_workspace_bytes(layout, batch) is larger than
+ *     AQ_STATIC_SCRATCH_BYTES; use aq_gemv with a workspace for such sizes.
+ *   - The first call on a device looks up the buffer's device address; make that first call
+ *     on each device before capturing any stream on it.
+ *   - Each call enqueues a clear of the buffer's status word and counters, then the GEMV.
+ *   - Every call on a device shares the one buffer, which keeps the last call's contents:
+ *     calls that may overlap on the GPU (other streams, other host threads) race on it and
+ *     must be ordered by the caller. */
+#define AQ_STATIC_SCRATCH_BYTES ((size_t)4 << 20)
+aq_status aq_gemv_static_scratch(const aq_layout* layout, int m, const void* planes,
+                                 const void* books, const void* scales, const void* x,
+                                 int x_dtype, int batch, void* y, int y_dtype, void* stream);
+
 /* ---------------------------------------------------------------- GEMM (prefill)
  * Same product for many tokens: y[t, o] = sum_i x[t, i] * W_m[o, i], t < tokens. Decoded
  * weight tiles are built in shared memory and multiplied on the tensor cores with fp32

@@ -22,7 +22,7 @@ TORCH_DTYPES = {AQ_F16: torch.float16, AQ_BF16: torch.bfloat16, AQ_F32: torch.fl
 # Every entry point that include/aq.h declares.
 EXPORTS = ["aq_abi_version", "aq_status_string", "aq_last_error", "aq_plane_bytes", "aq_packed_bytes", "aq_pack",
            "aq_decode", "aq_gemv_workspace_bytes", "aq_gemv", "aq_gemm_workspace_bytes",
-           "aq_gemm", "aq_workspace_init", "aq_workspace_status"]
+           "aq_gemm", "aq_workspace_init", "aq_workspace_status", "aq_gemv_static_scratch"]
 
 
 class AQError(RuntimeError):
@@ -73,6 +73,7 @@ def lib():
             "aq_gemm": (i32, [lp, i32, vp, vp, vp, vp, i32, i32, vp, i32, vp, sz, vp]),
             "aq_workspace_init": (i32, [vp, sz, vp]),
             "aq_workspace_status": (i32, [vp, vp]),
+            "aq_gemv_static_scratch": (i32, [lp, i32, vp, vp, vp, vp, i32, i32, vp, i32, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -152,6 +153,14 @@ def aq_gemm(layout, m, planes, books, scales, x, x_dtype, tokens, y, y_dtype, wo
     _check(lib().aq_gemm(ctypes.byref(layout), m, _ptr(planes), _ptr(books), _ptr(scales),
                          _ptr(x), x_dtype, tokens, _ptr(y), y_dtype, _ptr(workspace),
                          workspace_bytes, _stream(stream)), "aq_gemm")
+
+
+def aq_gemv_static_scratch(layout, m, planes, books, scales, x, x_dtype, batch, y, y_dtype,
+                           stream=None):
+    """aq_gemv without a workspace: scratch comes from the library's fixed device buffer."""
+    _check(lib().aq_gemv_static_scratch(ctypes.byref(layout), m, _ptr(planes), _ptr(books),
+                                        _ptr(scales), _ptr(x), x_dtype, batch, _ptr(y), y_dtype,
+                                        _stream(stream)), "aq_gemv_static_scratch")
 
 
 def aq_workspace_init(workspace, nbytes=None, stream=None):

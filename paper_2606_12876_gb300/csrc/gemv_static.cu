@@ -1,0 +1,67 @@
+// aq_gemv_static_scratch: the GEMV of aq_gemv for callers that cannot allocate device memory.
+//
+// Some callers cannot call cudaMalloc when they run a layer: a plugin inside a host program
+// that owns every byte of device memory and offers no allocator, a serving loop that must not
+// allocate after start-up (an allocation can synchronise the device or fail under memory
+// pressure), or code whose device footprint has to be fixed and known in advance. They cannot
+// provide the workspace that aq_gemv needs either. This entry point takes that scratch
+// (status word, completion counters, per-slice partial sums) from a fixed buffer that lives
+// in this file as a device array, so a call allocates nothing.
+#include <mutex>
+
+#include "aq_internal.cuh"
+
+namespace {
+
+// The fixed scratch buffer. Being a file-scope device array, it is created on every GPU that
+// loads this library and stays there until the process exits.
+constexpr size_t kStaticScratchBytes = AQ_STATIC_SCRATCH_BYTES;
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+// In host code, g_static_scratch names a host-side stand-in, not the device buffer; the device
+// address is looked up once per device (with that device current) and cached here.
+std::mutex g_mu;
+void* g_scratch_addr[64] = {};
+
+aq_status static_scratch_address(void** out) {
+    int dev = 0;
+    if (cudaError_t e = cudaGetDevice(&dev); e != cudaSuccess) return aq::cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= 64) return AQ_ERR_UNSUPPORTED;
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (!g_scratch_addr[dev]) {
+        void* p = nullptr;
+        if (cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch); e != cudaSuccess)
+            return aq::cuda_fail(e, "cudaGetSymbolAddress");
+        g_scratch_addr[dev] = p;
+    }
+    *out = g_scratch_addr[dev];
+    return AQ_OK;
+}
+
+}  // namespace
+
+extern "C" aq_status aq_gemv_static_scratch(const aq_layout* layout, int m, const void* planes,
+                                            const void* books, const void* scales,
+                                            const void* x, int x_dtype, int batch, void* y,
+                                            int y_dtype, void* stream) {
+    // Same argument checks as aq_gemv: run them with no workspace. Any answer other than
+    // "workspace missing" (an argument error, or success for empty work) is final.
+    const aq_status pre = aq_gemv(layout, m, planes, books, scales, x, x_dtype, batch, y,
+                                  y_dtype, nullptr, 0, stream);
+    if (pre != AQ_ERR_WORKSPACE) return pre;
+
+    const size_t need = aq_gemv_workspace_bytes(layout, batch);
+    if (need == 0 || need > kStaticScratchBytes) return AQ_ERR_WORKSPACE;  // beyond the fixed buffer
+    aq::Dims d;
+    if (aq_status e = aq::make_dims(layout, &d); e != AQ_OK) return e;
+
+    void* scratch = nullptr;
+    if (aq_status e = static_scratch_address(&scratch); e != AQ_OK) return e;
+    // The buffer keeps whatever the previous call left; the status word and the counters
+    // must start at zero, so clear them (the partial sums are always written before read).
+    if (cudaError_t e = cudaMemsetAsync(scratch, 0, aq::ws_partial_offset(d), (cudaStream_t)stream);
+        e != cudaSuccess)
+        return aq::cuda_fail(e, "cudaMemsetAsync");
+    return aq_gemv(layout, m, planes, books, scales, x, x_dtype, batch, y, y_dtype, scratch,
+                   kStaticScratchBytes, stream);
+}
