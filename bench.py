@@ -47,6 +47,26 @@ def layer_bytes(out, inp, m, B=8, G=8, batch=1, xsize=2, ysize=2):
             + batch * inp * xsize + batch * out * ysize)
 
 
+def profiled_traffic(workload, m):
+    """DRAM bytes per launch measured by ncu (profiles/gemv_lut_traffic.txt), or None when the
+    kernel sources changed since that capture."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "gemv_lut_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    h = hashlib.sha256()
+    for f in ("gemv.cu", "aq_internal.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2606_12876_gb300", "csrc", f), "rb").read())
+    rec, traffic = None, None
+    for line in open(path):
+        parts = line.split()
+        if len(parts) == 2 and parts[0] == "source_hash":
+            rec = parts[1]
+        elif len(parts) == 4 and parts[0] == workload and parts[1] == "m=%d" % m:
+            traffic = int(parts[3])
+    return traffic if rec == h.hexdigest()[:16] else None
+
+
 def dist_env():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -315,7 +335,8 @@ def own_arm(args):
             "roofline": {
                 "bound": "hbm", "kernel": "gemv_lut_kernel m=%d" % dom["m"],
                 "achieved": dom["GB_s"], "peak": hbm_peak, "unit": "GB/s",
-                "frac": round(dom["GB_s"] / hbm_peak, 4), "traffic": None,
+                "frac": round(dom["GB_s"] / hbm_peak, 4),
+                "traffic": profiled_traffic(WORKLOAD, dom["m"]),
                 "peak_source": peak_src},
             "cpu_baseline": cpu,
             "e2e": e2e,
