@@ -38,6 +38,7 @@ def parse():
     ap.add_argument("--impl", default="own", choices=["own", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-gemm", action="store_true")
     return ap.parse_args()
 
 
@@ -173,6 +174,51 @@ def reference_arm(args):
     print(json.dumps(line), flush=True)
 
 
+def measure_gemm(dev, stream, peaks, reps=5):
+    """Prefill GEMM on the 70B up-projection shape (4096 tokens, 8192 -> 28672, M = 4 bf16
+    books, bf16 activations) for every prefix m, next to a dense bf16 torch.matmul of the same
+    shape. Inputs (64 MB activations, 28-112 MB codes) exceed L2."""
+    import torch
+    import paper_2606_12876_gb300 as aq
+    from paper_2606_12876_gb300.linear import AQLinear, x_to_device
+    import workloads
+    name = "llama70b_up_prefill"
+    (_, layer), = list(workloads.config_layers(name))
+    tokens, out, inp = 4096, layer["out"], layer["in"]
+    lin = AQLinear.from_layer(layer, device=dev)
+    x = x_to_device(workloads.config_x(name, tokens, inp), "bf16", dev)
+    y = torch.empty(tokens, out, dtype=torch.bfloat16, device=dev)
+    flops = 2.0 * tokens * out * inp
+    peak = peaks.get("bf16_tflops", 1900.0)
+
+    def timed(fn):
+        with torch.cuda.stream(stream):
+            fn()
+            torch.cuda.synchronize(dev)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(reps):
+                fn()
+            e1.record()
+        torch.cuda.synchronize(dev)
+        return e0.elapsed_time(e1) / reps
+
+    rows = []
+    for m in (1, 2, 3, 4):
+        ms = timed(lambda: lin.gemm(x, m, y=y))
+        tf = flops / (ms * 1e-3) / 1e12
+        rows.append({"m": m, "ms": round(ms, 4), "TFLOP_s": round(tf, 1),
+                     "frac_bf16_peak": round(tf / peak, 4)})
+    wd = torch.randn(out, inp, device=dev, dtype=torch.bfloat16)
+    dense_ms = timed(lambda: torch.matmul(x, wd.t()))
+    del wd
+    return {"workload": name, "tokens": tokens, "out": out, "in": inp, "M": 4,
+            "compute": "fp16 tcgen05 MMA, fp32 accumulation, weights decoded in shared memory",
+            "per_m": rows, "dense_bf16_torch_ms": round(dense_ms, 4),
+            "dense_bf16_TFLOP_s": round(flops / (dense_ms * 1e-3) / 1e12, 1),
+            "peak_TFLOP_s": peak, "peak_source": "measured" if "bf16_tflops" in peaks else "fallback"}
+
+
 def own_arm(args):
     import numpy as np
     import torch
@@ -206,6 +252,13 @@ def own_arm(args):
     copies = [lin.planes.clone() for _ in range(ncopies)]
     bytes_m = {m: layer_bytes(out, inp, m) for m in ms}
     bytes_step = sum(bytes_m.values())
+
+    peaks = {}
+    ppath = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(ppath):
+        peaks = json.load(open(ppath))
+    hbm_peak = peaks.get("hbm_gbs", 6800.0)
+    peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
 
     stream = torch.cuda.Stream(device=dev)
 
@@ -270,12 +323,6 @@ def own_arm(args):
         per_m_us[m] = time_graph(g) * 1e3 / args.steps
         del g
 
-    peaks = {}
-    ppath = os.path.join(ROOT, "MEASURED_PEAKS.json")
-    if os.path.exists(ppath):
-        peaks = json.load(open(ppath))
-    hbm_peak = peaks.get("hbm_gbs", 6800.0)
-    peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
 
     per_m = []
     for m in ms:
@@ -312,6 +359,8 @@ def own_arm(args):
                "d2h_bytes_per_step": y_host.numel() * 2,
                "api": "paper_2606_12876_gb300.aq_gemv (ctypes -> libaq.so), eager"}
 
+    gemm = None if args.no_gemm else measure_gemm(dev, stream, peaks)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
@@ -332,6 +381,7 @@ def own_arm(args):
                        "l2": "rotating %d weight copies (%d x %.1f MB >= 3x L2 %.0f MB)" % (
                            ncopies, ncopies, pbytes / 1e6, l2 / 1e6)},
             "per_m": per_m,
+            "gemm": gemm,
             "roofline": {
                 "bound": "hbm", "kernel": "gemv_lut_kernel m=%d" % dom["m"],
                 "achieved": dom["GB_s"], "peak": hbm_peak, "unit": "GB/s",

@@ -147,11 +147,17 @@ aq_status aq_gemv_static_scratch(const aq_layout* layout, int m, const void* pla
 
 /* ---------------------------------------------------------------- GEMM (prefill)
  * Same product for many tokens: y[t, o] = sum_i x[t, i] * W_m[o, i], t < tokens. Decoded
- * weight tiles are built in shared memory and multiplied on the tensor cores with fp32
- * accumulation. Supported: code_bits = 8, book_dtype == x_dtype (f16 or bf16).
- *   x : device, [tokens][d_in] of x_dtype;  y : device, [tokens][d_out] of y_dtype.
- *   workspace : aq_gemm_workspace_bytes(layout, tokens) bytes, zero-filled before first use;
- *               its first word receives a device-side status (see aq_workspace_status). */
+ * weight tiles are built in shared memory and multiplied on the tcgen05 tensor cores with
+ * fp32 accumulation in tensor memory; W_m is never written to HBM. The MMA operands are fp16:
+ * each decoded weight (fp32 sum of the m codewords) is rounded once to fp16, and bf16
+ * activations are first copied to fp16 in the workspace (exact for |x| in fp16's normal
+ * range; values beyond +-65504 saturate). Supported: code_bits = 8, m <= 4.
+ *   x : device, [tokens][d_in] of x_dtype (AQ_F16 or AQ_BF16); y : device, [tokens][d_out]
+ *       of y_dtype (AQ_F16, AQ_BF16 or AQ_F32).
+ *   workspace : aq_gemm_workspace_bytes(layout, tokens) bytes (a status word and room for the
+ *               fp16 activation copy), zero-filled before first use; its first word receives a
+ *               device-side status (see aq_workspace_status).
+ * Accuracy: as aq_gemv for fp32 outputs; fp16/bf16 outputs add one rounding of y. */
 size_t aq_gemm_workspace_bytes(const aq_layout* layout, int tokens);
 aq_status aq_gemm(const aq_layout* layout, int m, const void* planes, const void* books,
                   const void* scales, const void* x, int x_dtype, int tokens, void* y,

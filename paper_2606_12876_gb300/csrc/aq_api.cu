@@ -91,6 +91,11 @@ aq_status check_ptrs(std::initializer_list<const void*> ps) {
     return AQ_OK;
 }
 
+// GEMM workspace: status word, then room for an fp16 copy of bf16 activations.
+size_t gemm_ws_bytes(const Dims& d, int tokens) {
+    return aq::kWsStatusBytes + (size_t)tokens * (size_t)d.in * 2;
+}
+
 size_t gemv_ws_bytes(const Dims& d, int batch) {
     return aq::ws_partial_offset(d) + (size_t)d.S * (size_t)batch * (size_t)d.rows_pad * 4;
 }
@@ -174,7 +179,7 @@ aq_status aq_gemv(const aq_layout* layout, int m, const void* planes, const void
 size_t aq_gemm_workspace_bytes(const aq_layout* layout, int tokens) {
     Dims d;
     if (aq::make_dims(layout, &d) != AQ_OK || tokens < 0) return 0;
-    return aq::kWsStatusBytes;
+    return gemm_ws_bytes(d, tokens);
 }
 
 aq_status aq_gemm(const aq_layout* layout, int m, const void* planes, const void* books,
@@ -185,9 +190,14 @@ aq_status aq_gemm(const aq_layout* layout, int m, const void* planes, const void
     if (st != AQ_OK) return st;
     if ((st = check_m(d, m)) != AQ_OK) return st;
     if (tokens < 0) return AQ_ERR_INVALID_ARG;
-    (void)planes; (void)books; (void)scales; (void)x; (void)x_dtype; (void)y; (void)y_dtype;
-    (void)workspace; (void)workspace_bytes; (void)stream;
-    return AQ_ERR_UNSUPPORTED;
+    if (x_dtype != AQ_F16 && x_dtype != AQ_BF16) return AQ_ERR_INVALID_ARG;
+    if (y_dtype != AQ_F16 && y_dtype != AQ_BF16 && y_dtype != AQ_F32) return AQ_ERR_INVALID_ARG;
+    if (tokens == 0 || d.out == 0) return AQ_OK;
+    if ((st = check_ptrs({planes, books, scales, x, y})) != AQ_OK) return st;
+    if (!workspace || workspace_bytes < gemm_ws_bytes(d, tokens)) return AQ_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;
+    return aq::launch_gemm(d, m, planes, books, scales, x, x_dtype, tokens, y, y_dtype, workspace,
+                           as_stream(stream));
 }
 
 aq_status aq_workspace_init(void* workspace, size_t bytes, void* stream) {

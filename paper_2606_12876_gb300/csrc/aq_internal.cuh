@@ -55,6 +55,9 @@ aq_status launch_decode(const Dims& d, int m, const void* planes, const void* bo
 aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* books,
                       const void* scales, const void* x, int x_dt, int batch, void* y,
                       int y_dt, void* ws, cudaStream_t st);
+aq_status launch_gemm(const Dims& d, int m, const void* planes, const void* books,
+                      const void* scales, const void* x, int x_dt, int tokens, void* y, int y_dt,
+                      void* ws, cudaStream_t st);
 
 // ---- device helpers ---------------------------------------------------------------------
 template <int DT>
