@@ -39,6 +39,10 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-gemm", action="store_true")
+    ap.add_argument("--gemm-tokens", type=int, default=4096,
+                    help="tokens of the prefill GEMM case (smaller values: profiling runs)")
+    ap.add_argument("--skip-gemv", action="store_true",
+                    help="only the GEMM case (profiling runs; prints no bench line)")
     return ap.parse_args()
 
 
@@ -174,7 +178,7 @@ def reference_arm(args):
     print(json.dumps(line), flush=True)
 
 
-def measure_gemm(dev, stream, peaks, reps=5):
+def measure_gemm(dev, stream, peaks, reps=5, tokens=4096):
     """Prefill GEMM on the 70B up-projection shape (4096 tokens, 8192 -> 28672, M = 4 bf16
     books, bf16 activations) for every prefix m, next to a dense bf16 torch.matmul of the same
     shape. Inputs (64 MB activations, 28-112 MB codes) exceed L2."""
@@ -184,7 +188,7 @@ def measure_gemm(dev, stream, peaks, reps=5):
     import workloads
     name = "llama70b_up_prefill"
     (_, layer), = list(workloads.config_layers(name))
-    tokens, out, inp = 4096, layer["out"], layer["in"]
+    out, inp = layer["out"], layer["in"]
     lin = AQLinear.from_layer(layer, device=dev)
     x = x_to_device(workloads.config_x(name, tokens, inp), "bf16", dev)
     y = torch.empty(tokens, out, dtype=torch.bfloat16, device=dev)
@@ -261,6 +265,10 @@ def own_arm(args):
     peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
 
     stream = torch.cuda.Stream(device=dev)
+    if args.skip_gemv:
+        g = measure_gemm(dev, stream, peaks, tokens=args.gemm_tokens)
+        print(json.dumps({"gemm_only": g}), flush=True)
+        return
 
     def call(i, m):
         aq.aq_gemv(L, m, copies[i % ncopies], lin.books, lin.scales, x, aq.AQ_F16, 1, ys[m],
@@ -359,7 +367,7 @@ def own_arm(args):
                "d2h_bytes_per_step": y_host.numel() * 2,
                "api": "paper_2606_12876_gb300.aq_gemv (ctypes -> libaq.so), eager"}
 
-    gemm = None if args.no_gemm else measure_gemm(dev, stream, peaks)
+    gemm = None if args.no_gemm else measure_gemm(dev, stream, peaks, tokens=args.gemm_tokens)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
