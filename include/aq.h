@@ -57,7 +57,17 @@ typedef struct aq_layout {
     int32_t code_bits;      /* B; 8 (uint8 codes) or 16 (uint16 codes) */
     int32_t book_dtype;     /* AQ_F16 or AQ_BF16: element type of the codebooks */
     int32_t scale_dtype;    /* AQ_F16 or AQ_BF16: element type of the scales */
+    int32_t flags;          /* 0 or AQ_LAYOUT_STATIC_WEIGHTS */
 } aq_layout;
+
+/* Layout flag: the layer's codes, codebooks and scales are not written by any kernel that
+ * may still be running when a GEMV or GEMM call on them starts (in inference they are written
+ * once, then only read). A call may then begin reading them - prefetching the first code
+ * stages into L2 and staging the codebooks - before the kernel that precedes it on the stream
+ * has finished, which overlaps that traffic with the preceding kernel's tail. Activations are
+ * always read only after the preceding kernel has finished. Without the flag (0) every read
+ * waits for the preceding kernel. */
+#define AQ_LAYOUT_STATIC_WEIGHTS 1
 
 /* ABI version of the loaded library (AQ_ABI_VERSION). */
 int aq_abi_version(void);

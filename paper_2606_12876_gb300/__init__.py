@@ -16,6 +16,7 @@ LIB_PATH = os.path.join(_PKG, "libaq.so")
 AQ_OK, AQ_ERR_INVALID_ARG, AQ_ERR_UNSUPPORTED, AQ_ERR_ALIGNMENT = 0, 1, 2, 3
 AQ_ERR_CUDA, AQ_ERR_TIMEOUT, AQ_ERR_WORKSPACE = 4, 5, 6
 AQ_F16, AQ_BF16, AQ_F32 = 0, 1, 2
+AQ_LAYOUT_STATIC_WEIGHTS = 1
 DTYPES = {"f16": AQ_F16, "bf16": AQ_BF16, "f32": AQ_F32}
 TORCH_DTYPES = {AQ_F16: torch.float16, AQ_BF16: torch.bfloat16, AQ_F32: torch.float32}
 
@@ -39,11 +40,11 @@ class Layout(ctypes.Structure):
     _fields_ = [("out_features", ctypes.c_int32), ("in_features", ctypes.c_int32),
                 ("group_size", ctypes.c_int32), ("num_books", ctypes.c_int32),
                 ("code_bits", ctypes.c_int32), ("book_dtype", ctypes.c_int32),
-                ("scale_dtype", ctypes.c_int32)]
+                ("scale_dtype", ctypes.c_int32), ("flags", ctypes.c_int32)]
 
     @classmethod
-    def make(cls, out, inp, M, B=8, G=8, book_dtype="f16", scale_dtype="f16"):
-        return cls(out, inp, G, M, B, DTYPES[book_dtype], DTYPES[scale_dtype])
+    def make(cls, out, inp, M, B=8, G=8, book_dtype="f16", scale_dtype="f16", flags=0):
+        return cls(out, inp, G, M, B, DTYPES[book_dtype], DTYPES[scale_dtype], flags)
 
 
 _lib = None

@@ -26,6 +26,8 @@ aq_status make_dims(const aq_layout* L, Dims* d) {
     d->B = L->code_bits;
     d->book_dt = L->book_dtype;
     d->scale_dt = L->scale_dtype;
+    if (L->flags & ~AQ_LAYOUT_STATIC_WEIGHTS) return AQ_ERR_INVALID_ARG;
+    d->flags = L->flags;
     d->ng = d->in / 8;
     d->ng_pad = (d->ng + 31) / 32 * 32;
     d->S = d->ng_pad / 32;

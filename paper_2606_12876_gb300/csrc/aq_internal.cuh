@@ -14,6 +14,7 @@ namespace aq {
 // Derived sizes of a validated layout (see the packed-plane description in aq.h).
 struct Dims {
     int out, in, G, M, B, book_dt, scale_dt;
+    int flags;     // AQ_LAYOUT_* bits
     int ng;        // groups per row, in/8
     int ng_pad;    // ng rounded up to 32
     int S;         // slices of 32 groups
@@ -176,6 +177,12 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
         ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
         : "memory");
+}
+
+// Prefetch `bytes` of global memory into L2 (no data returned to the SM). src 16-byte
+// aligned, bytes a multiple of 16.
+__device__ __forceinline__ void prefetch_l2(const void* src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
 }
 
 // Programmatic dependent launch: wait for the preceding grid's results / allow the next grid

@@ -65,7 +65,7 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                 float* __restrict__ partials, unsigned int* __restrict__ counters,
                 unsigned int* __restrict__ status, void* y, int y_dt, int m, int out, int in,
                 int ng, int rows_pad, int RBc, int S, long long total_items, size_t plane_bytes,
-                int nslots, int cps) {
+                int nslots, int cps, int static_weights) {
     extern __shared__ __align__(128) unsigned char smem[];
     unsigned char* T = smem;
     uint4* Cb = (uint4*)(smem + kTBytes);                          // [m][256] codewords
@@ -97,18 +97,40 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
         mbar_fence_init();
         s_abort = 0;
     }
-    pdl_wait();                 // inputs may come from the preceding kernel in the stream
-
     // Codebooks and activations are requested first (into registers); the producer starts
     // its copies only after every thread has issued these loads (the barrier below).
     // (consumer threads only: they are the ones that store the codebooks below)
     uint4 cb_r[4];
+    auto load_books = [&]() {
 #pragma unroll
-    for (int r = 0; r < 4; ++r) {
-        const int i = tid + r * kCons * 32;
-        cb_r[r] = (tid < kCons * 32 && i < m * 256) ? __ldg((const uint4*)books + i)
-                                                      : make_uint4(0u, 0u, 0u, 0u);
+        for (int r = 0; r < 4; ++r) {
+            const int i = tid + r * kCons * 32;
+            cb_r[r] = (tid < kCons * 32 && i < m * 256) ? __ldg((const uint4*)books + i)
+                                                          : make_uint4(0u, 0u, 0u, 0u);
+        }
+    };
+    if (static_weights) {
+        // The weights are read-only while calls run (AQ_LAYOUT_STATIC_WEIGHTS): stage the
+        // codebooks and pull the first code stages of this CTA into L2 before waiting for the
+        // preceding kernel, so that traffic overlaps its tail.
+        load_books();
+        if (warp == kCons && lane == 0) {
+            uint32_t budget = 96 * 1024;
+            for (int k = 0; k < m && budget > 0; ++k)
+                for (long long it = i0; it < i1 && budget > 0;) {
+                    const long long seg_end = min(i1, (it / RBc + 1) * RBc);
+                    uint32_t bytes = (uint32_t)((seg_end - it) * 1024);
+                    if (bytes > budget) bytes = budget;
+                    prefetch_l2(planes + (size_t)k * plane_bytes +
+                                    ((size_t)(it / RBc) * rows_pad + (size_t)(it % RBc) * 32) * 32,
+                                bytes);
+                    budget -= bytes;
+                    it = seg_end;
+                }
+        }
     }
+    pdl_wait();                 // inputs may come from the preceding kernel in the stream
+    if (!static_weights) load_books();
     uint2 x_r = make_uint2(0u, 0u);
     if (tid < kXSlices * 64) {
         const int col = (s_first + (tid >> 6)) * 256 + (tid & 63) * 4;
@@ -475,7 +497,8 @@ aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     return launch_pdl(kern, dim3(grid), dim3(kLutThreads), smem, st, (const uint8_t*)a.planes,
                       (const uint16_t*)a.books, (const uint16_t*)a.x, (const uint16_t*)a.scales,
                       a.partials, a.counters, a.status, a.y, a.y_dt, m, d.out, d.in, d.ng,
-                      d.rows_pad, d.RBc, d.S, items, d.plane_bytes, nslots, cps);
+                      d.rows_pad, d.RBc, d.S, items, d.plane_bytes, nslots, cps,
+                      (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0);
 }
 
 template <int NB, int B, int BDT, int SDT>

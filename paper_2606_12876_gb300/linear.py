@@ -7,7 +7,8 @@ torch; all work is done by libaq through the binding in this package.
 import numpy as np
 import torch
 
-from . import (AQ_BF16, AQ_F16, AQ_F32, DTYPES, TORCH_DTYPES, Layout, aq_decode, aq_gemm,
+from . import (AQ_BF16, AQ_F16, AQ_F32, AQ_LAYOUT_STATIC_WEIGHTS, DTYPES, TORCH_DTYPES, Layout,
+               aq_decode, aq_gemm,
                aq_gemv, aq_pack, gemm_workspace_bytes, gemv_workspace_bytes, packed_bytes,
                workspace)
 
@@ -21,7 +22,9 @@ class AQLinear:
     """Packed planes, codebooks and scales of one layer on `device`.
 
     books: [M][2^B][8] fp16/bf16 bit patterns (uint16); codes: (out, in/8, M) uint8/uint16;
-    scales: [out] bit patterns. The natural codes are packed on the GPU by aq_pack.
+    scales: [out] bit patterns. The natural codes are packed on the GPU by aq_pack. After
+    packing the stream is synchronised and the layout is marked AQ_LAYOUT_STATIC_WEIGHTS: the
+    layer's weights are read-only from then on, so calls may prefetch them early.
     """
 
     def __init__(self, books, codes, scales, book_dtype="f16", scale_dtype="f16",
@@ -40,6 +43,8 @@ class AQLinear:
         self.planes = torch.empty(packed_bytes(self.layout, M), dtype=torch.uint8,
                                   device=self.device)
         aq_pack(self.layout, codes_t, self.planes)
+        torch.cuda.current_stream(self.device).synchronize()
+        self.layout.flags = AQ_LAYOUT_STATIC_WEIGHTS
         self.codes = codes_t if keep_codes else None
         self._ws = {}
 

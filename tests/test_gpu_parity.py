@@ -175,3 +175,18 @@ def test_gemv_prefix_buffer_only():
         y = torch.empty(1, 200, dtype=torch.float32, device="cuda")
         aq.aq_gemv(lin.layout, m, prefix, lin.books, lin.scales, x, aq.AQ_F16, 1, y, aq.AQ_F32, ws)
         U.assert_product_close(U.to_f64(y), oracle.product_exact(layer, x_bits, "f16", m))
+
+
+def test_gemv_static_weights_flag_gives_same_result():
+    """AQ_LAYOUT_STATIC_WEIGHTS only lets the kernel read the weights earlier; the result is
+    bit-identical with and without it."""
+    layer = _layer(2000, 4096, 4, 8, "f16", seed=12)
+    lin = AQLinear.from_layer(layer)
+    assert lin.layout.flags == aq.AQ_LAYOUT_STATIC_WEIGHTS
+    x = x_to_device(workloads.make_x(1, 4096, "f16", seed=5), "f16")
+    for m in (1, 3, 4):
+        a = lin.gemv(x, m).clone()
+        lin.layout.flags = 0
+        b = lin.gemv(x, m).clone()
+        lin.layout.flags = aq.AQ_LAYOUT_STATIC_WEIGHTS
+        assert torch.equal(a, b), m
