@@ -2,20 +2,28 @@
 // (the prefix-m additive reconstruction of Sec. 3.2 / Sec. 5) decoded tile by tile into shared
 // memory and never written to HBM.
 //
-// Tile: 512 tokens x 128 output rows, K in steps of 64 inputs (one 128-byte swizzle row of
-// 16-bit values). The four 128x128 fp32 accumulators fill the 512 columns of tensor memory, so
-// every decoded weight tile feeds 512 tokens. Roles (12 warps):
+// A cluster of two CTAs (one CTA pair, one CTA per SM) computes a 512-token x 256-row tile with
+// pair MMAs (tcgen05.mma.cta_group::2, M = 256 tokens, N = 256 rows, K = 16): each CTA holds
+// 128 tokens of every A block and decodes its own 128 of the 256 weight rows, and the MMA
+// reads both halves of both operands, so every SM supplies half the operand bytes of what a
+// single-CTA MMA of the same work would read from its shared memory. Shared-memory bandwidth is
+// what the decoders' codeword gathers compete for, so this is the main point of the pair.
+// Each CTA's tensor memory holds its 128 tokens x 256 rows for two token blocks (512 columns).
+// Roles (12 warps per CTA):
 //   warp 0      TMA producer: activation tiles (2-D tensor map, 128-byte swizzle, two
-//               256-token boxes per stage) and, once per 256-input slice, the slice's code rows
-//               of the first m planes (1-D bulk copies; a tile's rows of a slice are contiguous
+//               128-token boxes per stage) and, once per 256-input slice, this CTA's code rows
+//               of the first m planes (1-D bulk copies; a CTA's rows of a slice are contiguous
 //               in every plane).
-//   warp 1      allocates tensor memory; lane 0 issues tcgen05.mma (4 token blocks x 4 K=16
-//               steps per stage) and commits stage-release / accumulator-ready barriers.
+//   warp 1      allocates the pair's tensor memory (together with the peer's warp 1). In the
+//               leader CTA (rank 0) lane 0 issues the pair MMAs (2 token blocks x 4 K=16 steps
+//               per stage) and commits stage-release / accumulator-ready barriers to both
+//               CTAs. In the peer CTA lane 0 relays "stage ready" (its activation copies landed,
+//               its decoders wrote its weight half) to the leader with a remote mbarrier arrive.
 //   warps 4-11  decoders: each thread owns one weight row and four groups of every stage; it
-//               sums the m codewords in fp32 (book order), rounds once to the book type and
-//               writes the 16-byte group into the B tile in the UMMA K-major 128-byte-swizzle
-//               layout. Afterwards the same warps are the epilogue: tcgen05.ld from tensor
-//               memory, times the row scale (R1), round, store.
+//               sums the m codewords in fp32 (book order), rounds once to fp16 and writes the
+//               16-byte group into the B tile in the UMMA K-major 128-byte-swizzle layout.
+//               Afterwards the same warps are the epilogue: tcgen05.ld from tensor memory,
+//               times the row scale (R1), round, store.
 // Operands are fp16 (kind::f16, fp32 accumulation): the summed weights are rounded once to
 // fp16 (about 2^-11 relative), which keeps the product inside the stated per-element bound;
 // bf16 activations are first converted to fp16 into the workspace (exact for normal-range
@@ -32,32 +40,42 @@
 namespace aq {
 namespace {
 
-constexpr int kBM = 128;                      // tokens per MMA
-constexpr int kMT = 4;                        // token blocks per tile (512 tokens)
-constexpr int kBN = 128;                      // output rows per tile
+constexpr int kBM = 128;                      // tokens per CTA per MMA (M = 256 per pair)
+constexpr int kAcc = 2;                       // token blocks (accumulators) per CTA
+constexpr int kPairTokens = 2 * kAcc * kBM;   // 512 tokens per pair tile
+constexpr int kRows = 128;                    // weight rows decoded by one CTA
+constexpr int kBN = 2 * kRows;                // weight rows per pair tile (N of the MMA)
 constexpr int kBK = 64;                       // inputs per stage
-constexpr int kStages = 2;
+constexpr int kStagesA = 4;                   // activation ring (TMA)
+constexpr int kStagesB = 3;                   // decoded-weight ring
 constexpr int kGemmThreads = 384;
 constexpr int kDecWarp0 = 4, kDecWarps = 8;
 constexpr int kGemmMaxM = 4;
 
-constexpr int kAStage = kMT * kBM * 128;      // 64 KiB
-constexpr int kBStage = kBN * 128;            // 16 KiB
-constexpr int kCodeBuf = kGemmMaxM * kBN * 32;   // one slice of codes, all planes (16 KiB)
+constexpr int kABlock = kBM * 128;            // one 128-token x 64-input block (16 KiB)
+constexpr int kAStage = kAcc * kABlock;       // 32 KiB
+constexpr int kBStage = kRows * 128;          // 16 KiB
+constexpr int kCodeBuf = kGemmMaxM * kRows * 32;   // one slice of codes, all planes (16 KiB)
 
-// Shared-memory map (offsets from a 1024-byte aligned base).
+// Shared-memory map (offsets from a 1024-byte aligned base; identical in both CTAs of a pair,
+// which the pair MMA relies on: it reads the peer's operands at the same offsets).
 constexpr int kOffA = 0;
-constexpr int kOffB = kOffA + kStages * kAStage;
-constexpr int kOffCodes = kOffB + kStages * kBStage;
+constexpr int kOffB = kOffA + kStagesA * kAStage;
+constexpr int kOffCodes = kOffB + kStagesB * kBStage;
 constexpr int kOffBooks = kOffCodes + 2 * kCodeBuf;
 constexpr int kOffScale = kOffBooks + kGemmMaxM * 4096;
 constexpr int kOffBar = kOffScale + kBN * 4;
-constexpr int kNumBars = 3 * kStages + 4 + 1;   // full_a, full_b, empty, codes_full[2], codes_empty[2], acc
+// full_a, empty_a (per A stage), full_b, empty_b, peer_ready (per B stage), codes_full[2],
+// codes_empty[2], acc_full
+constexpr int kNumBars = 2 * kStagesA + 3 * kStagesB + 4 + 1;
 constexpr int kOffTmem = kOffBar + kNumBars * 8;
-constexpr int kSmemUsed = kOffTmem + 16;
-constexpr int kGemmSmem = kSmemUsed + 1024;     // slack for aligning the base to 1024 bytes
+constexpr int kOffAbort = kOffTmem + 16;
+// The kernel has no static shared memory, so its dynamic shared memory starts on a 1024-byte
+// boundary (checked at run time: the 128-byte swizzled tiles need it).
+constexpr int kGemmSmem = kOffAbort + 16;
+static_assert(kGemmSmem <= 227 * 1024, "shared memory map exceeds the per-CTA limit");
 
-// ---- tcgen05 / TMA helpers (PTX) -----------------------------------------------------------
+// ---- tcgen05 / TMA / cluster helpers (PTX) --------------------------------------------------
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int c0, int c1,
                                             uint64_t* bar) {
@@ -68,6 +86,49 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
         : "memory");
 }
 
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// Address, in the cluster shared window, of the variable at local address `addr` in CTA `rank`.
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+
+// Arrive on an mbarrier of another CTA of the cluster. The data it announces lives in the
+// arriving CTA's own shared memory (written there by its TMA copies and its decoders, which
+// this thread has already waited for), so the arrive orders those writes at CTA scope, the
+// usual form of a cross-CTA pipeline signal; a cluster-scope release costs this thread about
+// half a microsecond per stage, which alone exceeds a stage's MMA time.
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+// Bounded wait with cluster-scope acquire (for phases completed by another CTA's arrivals).
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity) {
+    for (uint32_t i = 0; i < kSpinLimit; ++i) {
+        uint32_t ok;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+            " selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(ok)
+            : "r"(smem_u32(bar)), "r"(parity)
+            : "memory");
+        if (ok) return true;
+        if (i >= 4096) __nanosleep(128);
+    }
+    return false;
+}
+
+// All threads of both CTAs (release / acquire at cluster scope); callable from divergent code.
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+
 // UMMA shared-memory descriptor: K-major operand, 128-byte swizzle, 8-row atoms 1024 bytes
 // apart (SBO), version 1, leading offset unused (16 bytes).
 __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr) {
@@ -75,19 +136,24 @@ __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr) {
            ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
 
-__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                         uint32_t idesc, uint32_t accumulate) {
+// Pair MMA: D[256 x N] (+)= A[256 x 16] * B[N x 16]^T, A and D split by rows across the pair,
+// B split by rows (N) across the pair; issued by one thread of the leader CTA.
+__device__ __forceinline__ void umma_f16_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                              uint32_t idesc, uint32_t accumulate) {
     asm volatile(
         "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+        " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
         "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
 
-__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+// Arrive on the barrier at local offset `bar` in both CTAs of the pair once every prior pair
+// MMA of this thread has completed.
+__device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
+    const uint16_t mask = 0x3;
     asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-            smem_u32(bar))
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+        " [%0], %1;" ::"r"(smem_u32(bar)), "h"(mask)
         : "memory");
 }
 
@@ -125,6 +191,73 @@ __device__ __forceinline__ uint32_t pack2(float lo, float hi, int dt) {
     return *(uint32_t*)&h;
 }
 
+// Shared-memory accesses through 32-bit shared-window addresses. lds128 is for data that no
+// thread writes while it may be read (codebooks): the compiler may reorder it freely.
+// lds128_ordered stays after the barrier wait that precedes it.
+__device__ __forceinline__ uint4 lds128(uint32_t a) {
+    uint4 v;
+    asm("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ uint4 lds128_ordered(uint32_t a) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a) : "memory");
+    return v;
+}
+__device__ __forceinline__ void sts128(uint32_t a, uint4 v) {
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z),
+                 "r"(v.w)
+                 : "memory");
+}
+
+// Two fp32 additions in one instruction (each lane rounded to nearest, as a scalar add).
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+    unsigned long long ar, br, dr;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(ar) : "f"(a.x), "f"(a.y));
+    asm("mov.b64 %0, {%1, %2};" : "=l"(br) : "f"(b.x), "f"(b.y));
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(dr) : "l"(ar), "l"(br));
+    float2 d;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(dr));
+    return d;
+}
+
+// One 32-bit word of a codeword (two 16-bit values, low half first) -> two floats.
+template <int BDT>
+__device__ __forceinline__ float2 widen2(uint32_t w) {
+    if constexpr (BDT == AQ_BF16) return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+    else return make_float2(__half2float(__ushort_as_half((unsigned short)(w & 0xffffu))),
+                            __half2float(__ushort_as_half((unsigned short)(w >> 16))));
+}
+
+__device__ __forceinline__ uint32_t f16x2(float2 v) {   // {lo, hi} -> packed fp16 pair, RN
+    uint32_t h;
+    asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(h) : "f"(v.y), "f"(v.x));
+    return h;
+}
+
+// Decoded group (eight fp16 weights): sum of the MB codewords in fp32, in book order, rounded
+// once to fp16. code[k] is the group's code in plane k; book k starts at books + k*4096.
+template <int BDT, int MB>
+__device__ __forceinline__ uint4 decode_group(uint32_t books, const uint32_t (&code)[MB]) {
+    const uint4 c0 = lds128(books + (code[0] << 4));
+    if constexpr (MB == 1 && BDT == AQ_F16) {
+        return c0;   // one fp16 codeword: widening to fp32 and rounding back is exact
+    } else {
+        float2 a0 = widen2<BDT>(c0.x), a1 = widen2<BDT>(c0.y), a2 = widen2<BDT>(c0.z),
+               a3 = widen2<BDT>(c0.w);
+#pragma unroll
+        for (int k = 1; k < MB; ++k) {
+            const uint4 ck = lds128(books + ((uint32_t)k << 12) + (code[k] << 4));
+            a0 = add2(a0, widen2<BDT>(ck.x));
+            a1 = add2(a1, widen2<BDT>(ck.y));
+            a2 = add2(a2, widen2<BDT>(ck.z));
+            a3 = add2(a3, widen2<BDT>(ck.w));
+        }
+        return make_uint4(f16x2(a0), f16x2(a1), f16x2(a2), f16x2(a3));
+    }
+}
+
 // Bounded wait that gives up at once after a failure anywhere in the CTA.
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort,
                                               unsigned int* status) {
@@ -135,38 +268,60 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
     return false;
 }
 
-template <int BDT>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+// One instantiation per book type and prefix length MB (= m): the decoders' code holds exactly
+// the lookups of that prefix.
+template <int BDT, int MB>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ planes,
             const uint16_t* __restrict__ books, const uint16_t* __restrict__ scales, void* y,
-            int y_dt, int scale_dt, unsigned int* __restrict__ status, int m, int tokens, int out,
+            int y_dt, int scale_dt, unsigned int* __restrict__ status, int tokens, int out,
             int in, int ng, int rows_pad, size_t plane_bytes) {
-    extern __shared__ unsigned char smem_raw[];
-    unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    extern __shared__ __align__(1024) unsigned char smem[];
     uint64_t* bars = (uint64_t*)(smem + kOffBar);
-    uint64_t* full_a = bars;
-    uint64_t* full_b = bars + kStages;
-    uint64_t* empty = bars + 2 * kStages;
-    uint64_t* codes_full = bars + 3 * kStages;
+    uint64_t* full_a = bars;                    // this CTA's activation copies landed
+    uint64_t* empty_a = bars + kStagesA;        // the pair MMAs reading the A stage completed
+    uint64_t* full_b = bars + 2 * kStagesA;     // this CTA's decoders wrote its weight half
+    uint64_t* empty_b = full_b + kStagesB;      // the pair MMAs reading the B stage completed
+    uint64_t* peer_ready = empty_b + kStagesB;  // (leader) the peer's A and B stages are ready
+    uint64_t* codes_full = peer_ready + kStagesB;
     uint64_t* codes_empty = codes_full + 2;
     uint64_t* acc_full = codes_empty + 2;
     uint32_t* tmem_slot = (uint32_t*)(smem + kOffTmem);
     float* scale_s = (float*)(smem + kOffScale);
-    const uint4* books_s = (const uint4*)(smem + kOffBooks);
-    __shared__ volatile int s_abort;
+    uint4* books_s = (uint4*)(smem + kOffBooks);
+    constexpr int m = MB;
+    volatile int& s_abort = *(volatile int*)(smem + kOffAbort);
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int n0 = blockIdx.x * kBN;          // first output row of the tile
-    const int t0 = blockIdx.y * (kMT * kBM);  // first token of the tile
-    const int nk = (in + kBK - 1) / kBK;      // K steps
-    const int nsl = (nk + 3) / 4;             // 256-input slices
-    const int rows_valid = min(kBN, rows_pad - n0);   // packed rows present (multiple of 32)
+    const uint32_t rank = cluster_rank();       // 0: leader (issues the MMAs), 1: peer
+    const int n0 = (blockIdx.x >> 1) * kBN;     // first output row of the pair tile
+    const int r0 = n0 + (int)rank * kRows;      // first row decoded by this CTA
+    const int t0 = blockIdx.y * kPairTokens;    // first token of the pair tile
+    const int nk = (in + kBK - 1) / kBK;        // K steps
+    const int nsl = (nk + 3) / 4;               // 256-input slices
+    const int rows_valid = max(0, min(kRows, rows_pad - r0));   // packed rows present (x32)
+    // Pairs that run at the same time share their token tile; if they all walked K in the same
+    // order they would request the same activation lines from L2 at the same moment. Each
+    // pair therefore starts at its own 256-input slice and wraps around (only the fp32
+    // accumulation order differs). Every role walks the slices in this order; `it` counts
+    // stages in processing order and drives the ring.
+    const int rot = (blockIdx.x >> 1) % nsl;
 
+    // Same answer in both CTAs of the pair (identical layouts), so both leave before any
+    // cluster-wide step.
+    if (smem_u32(smem) & 1023u) {
+        if (tid == 0) record_status(status, AQ_ERR_ALIGNMENT);
+        return;
+    }
     if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < kStagesA; ++s) {
             mbar_init(&full_a[s], 1);             // producer arrival + TMA bytes
+            mbar_init(&empty_a[s], 1);            // the leader's multicast commit
+        }
+        for (int s = 0; s < kStagesB; ++s) {
             mbar_init(&full_b[s], kDecWarps);     // one arrival per decoder warp
-            mbar_init(&empty[s], 1);              // tcgen05.commit
+            mbar_init(&empty_b[s], 1);            // the leader's multicast commit
+            mbar_init(&peer_ready[s], 1);         // the peer's relay arrival
         }
         for (int c = 0; c < 2; ++c) {
             mbar_init(&codes_full[c], 1);
@@ -176,14 +331,14 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
         mbar_fence_init();
         s_abort = 0;
     }
-    if (warp == 1) {   // tensor memory: 512 columns = four 128x128 fp32 accumulators
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
+    if (warp == 1) {   // tensor memory of the pair: 512 columns in each CTA, allocated jointly
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
                          smem_u32(tmem_slot))
                      : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
     }
     tc_fence_before();
-    __syncthreads();
+    cluster_sync();    // barriers of both CTAs initialised before any cross-CTA arrival
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     pdl_wait();
@@ -193,80 +348,112 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
         if (lane == 0) {
             asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&xmap) : "memory");
             int issued_a = 0, issued_c = 0;
-            for (int ks = 0; ks < nk && !s_abort; ++ks) {
-                const int st = ks % kStages;
-                if (ks % 4 == 0) {                        // codes of slice ks/4
-                    const int sl = ks / 4, cb = sl & 1;
-                    if (sl >= 2 && !wait_or_abort(&codes_empty[cb], ((sl >> 1) - 1) & 1, &s_abort, status))
-                        break;
-                    mbar_arrive_expect_tx(&codes_full[cb], (uint32_t)(m * rows_valid * 32));
-                    for (int k = 0; k < m; ++k)
-                        bulk_g2s(smem + kOffCodes + cb * kCodeBuf + k * (kBN * 32),
-                                 planes + (size_t)k * plane_bytes + ((size_t)sl * rows_pad + n0) * 32,
-                                 (uint32_t)(rows_valid * 32), &codes_full[cb]);
-                    ++issued_c;
-                }
-                if (ks >= kStages &&
-                    !wait_or_abort(&empty[st], ((ks / kStages) - 1) & 1, &s_abort, status))
+            bool stop = false;
+            for (int js = 0; js < nsl && !stop; ++js) {
+                const int sl = rot + js < nsl ? rot + js : rot + js - nsl;
+                const int cb = js & 1;                    // codes of slice sl
+                if (js >= 2 && !wait_or_abort(&codes_empty[cb], ((js >> 1) - 1) & 1, &s_abort, status))
                     break;
-                mbar_arrive_expect_tx(&full_a[st], (uint32_t)kAStage);
-                unsigned char* a = smem + kOffA + st * kAStage;
-                tma_load_2d(a, &xmap, ks * kBK, t0, &full_a[st]);
-                tma_load_2d(a + kAStage / 2, &xmap, ks * kBK, t0 + 2 * kBM, &full_a[st]);
-                ++issued_a;
+                mbar_arrive_expect_tx(&codes_full[cb], (uint32_t)(m * rows_valid * 32));
+                if (rows_valid > 0)
+                    for (int k = 0; k < m; ++k)
+                        bulk_g2s(smem + kOffCodes + cb * kCodeBuf + k * (kRows * 32),
+                                 planes + (size_t)k * plane_bytes + ((size_t)sl * rows_pad + r0) * 32,
+                                 (uint32_t)(rows_valid * 32), &codes_full[cb]);
+                ++issued_c;
+                const int nj = min(4, nk - sl * 4);
+                for (int j = 0; j < nj; ++j) {
+                    const int it = issued_a, st = it % kStagesA;
+                    if (it >= kStagesA &&
+                        !wait_or_abort(&empty_a[st], ((it / kStagesA) - 1) & 1, &s_abort, status)) {
+                        stop = true;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&full_a[st], (uint32_t)kAStage);
+                    unsigned char* a = smem + kOffA + st * kAStage;
+#pragma unroll
+                    for (int i = 0; i < kAcc; ++i)
+                        tma_load_2d(a + i * kABlock, &xmap, (sl * 4 + j) * kBK,
+                                    t0 + i * 2 * kBM + (int)rank * kBM, &full_a[st]);
+                    ++issued_a;
+                }
             }
             // No copy may still be in flight when the CTA exits.
-            for (int j = max(0, issued_a - kStages); j < issued_a; ++j)
-                mbar_wait(&full_a[j % kStages], (j / kStages) & 1);
+            for (int j = max(0, issued_a - kStagesA); j < issued_a; ++j)
+                mbar_wait(&full_a[j % kStagesA], (j / kStagesA) & 1);
             for (int j = max(0, issued_c - 2); j < issued_c; ++j)
                 mbar_wait(&codes_full[j & 1], (j >> 1) & 1);
         }
     } else if (warp == 1) {
-        // ---------------- MMA issuer
-        if (lane == 0) {
+        if (lane == 0 && rank == 0) {
+            // ---------------- MMA issuer (leader)
             // kind::f16 instruction descriptor: fp32 accumulator, fp16 A and B, both K-major,
-            // N = 128, M = 128.
-            const uint32_t idesc = (1u << 4) | ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
-            for (int ks = 0; ks < nk; ++ks) {
-                const int st = ks % kStages;
-                const uint32_t par = (ks / kStages) & 1;
-                if (!wait_or_abort(&full_a[st], par, &s_abort, status)) break;
-                if (!wait_or_abort(&full_b[st], par, &s_abort, status)) break;
+            // N = 256, M = 256 (pair).
+            const uint32_t idesc = (1u << 4) | ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)((2 * kBM) >> 4) << 24);
+            for (int it = 0; it < nk; ++it) {
+                const int sa = it % kStagesA, sb = it % kStagesB;
+                const uint32_t pa = (it / kStagesA) & 1, pb = (it / kStagesB) & 1;
+                if (!wait_or_abort(&full_a[sa], pa, &s_abort, status)) break;
+                if (!wait_or_abort(&full_b[sb], pb, &s_abort, status)) break;
+                if (!mbar_wait_cluster(&peer_ready[sb], pb)) {
+                    record_status(status, AQ_ERR_TIMEOUT);
+                    s_abort = 1;
+                    break;
+                }
                 tc_fence_after();
-                const uint32_t a0 = smem_u32(smem + kOffA + st * kAStage);
-                const uint32_t b0 = smem_u32(smem + kOffB + st * kBStage);
+                const uint32_t a0 = smem_u32(smem + kOffA + sa * kAStage);
+                const uint32_t b0 = smem_u32(smem + kOffB + sb * kBStage);
 #pragma unroll
-                for (int i = 0; i < kMT; ++i)
+                for (int i = 0; i < kAcc; ++i)
 #pragma unroll
                     for (int kk = 0; kk < kBK / 16; ++kk)
-                        umma_f16(tmem + i * kBN, umma_desc_sw128(a0 + i * (kBM * 128) + kk * 32),
-                                 umma_desc_sw128(b0 + kk * 32), idesc, (ks > 0 || kk > 0) ? 1u : 0u);
-                umma_commit(&empty[st]);
+                        umma_f16_pair(tmem + i * kBN, umma_desc_sw128(a0 + i * kABlock + kk * 32),
+                                      umma_desc_sw128(b0 + kk * 32), idesc, (it > 0 || kk > 0) ? 1u : 0u);
+                umma_commit_pair(&empty_a[sa]);
+                umma_commit_pair(&empty_b[sb]);
             }
-            umma_commit(acc_full);
+            umma_commit_pair(acc_full);
+        } else if (lane == 0) {
+            // ---------------- relay (peer): this CTA's half of a stage is ready
+            const uint32_t leader_ready = map_to_rank(smem_u32(peer_ready), 0);
+            for (int it = 0; it < nk; ++it) {
+                const int sa = it % kStagesA, sb = it % kStagesB;
+                if (!wait_or_abort(&full_a[sa], (it / kStagesA) & 1, &s_abort, status)) break;
+                if (!wait_or_abort(&full_b[sb], (it / kStagesB) & 1, &s_abort, status)) break;
+                mbar_arrive_cluster(leader_ready + sb * 8);
+            }
         }
     } else if (warp >= kDecWarp0) {
         // ---------------- decoders, then epilogue
         const int dt = tid - kDecWarp0 * 32;        // 0..255
-        const int n = dt & (kBN - 1);               // tile row owned by this thread
+        const int n = dt & (kRows - 1);             // row of this CTA's half owned by the thread
         const int cs = dt >> 7;                     // groups 4cs..4cs+3 of every stage
-        const int row = n0 + n;
+        const int row = r0 + n;
         for (int i = dt; i < m * 256; i += kDecWarps * 32)
-            ((uint4*)books_s)[i] = __ldg((const uint4*)books + i);
-        if (dt < kBN) scale_s[dt] = (n0 + dt < out) ? bits_to_f32_rt(scales[n0 + dt], scale_dt) : 0.0f;
+            books_s[i] = __ldg((const uint4*)books + i);
+        for (int i = dt; i < kBN; i += kDecWarps * 32)
+            scale_s[i] = (n0 + i < out) ? bits_to_f32_rt(scales[n0 + i], scale_dt) : 0.0f;
         named_barrier(1, kDecWarps * 32);
 
         const int r = row & 31;                     // rotation of this row's codes
-        for (int sl = 0; sl < nsl; ++sl) {
-            const int cb = sl & 1;
-            uint32_t cw[kGemmMaxM][8];              // this row's 32 codes of the slice, per plane
-            const bool have = wait_or_abort(&codes_full[cb], (sl >> 1) & 1, &s_abort, status);
+        const int rw = r >> 2, rb = (r & 3) * 8;
+        const bool row_ok = row < out;
+        const uint32_t books_u = smem_u32(books_s);
+        const uint32_t b_tile = smem_u32(smem + kOffB) + (n >> 3) * 1024 + (n & 7) * 128;
+        int it = 0;                                 // stages decoded so far (ring position)
+        for (int js = 0; js < nsl; ++js) {
+            const int sl = rot + js < nsl ? rot + js : rot + js - nsl;
+            const int cb = js & 1;
+            // q[k][j]: the codes (one byte each) of groups 8j + 4cs .. 8j + 4cs + 3 of the
+            // slice in plane k; the front entry always belongs to the next stage.
+            uint32_t q[MB][4];
+            const bool have = wait_or_abort(&codes_full[cb], (js >> 1) & 1, &s_abort, status);
 #pragma unroll
-            for (int k = 0; k < kGemmMaxM; ++k) {
+            for (int k = 0; k < MB; ++k) {
                 uint32_t w[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-                if (have && k < m && n < rows_valid) {
-                    const uint4* src = (const uint4*)(smem + kOffCodes + cb * kCodeBuf + k * (kBN * 32) + n * 32);
-                    const uint4 lo = src[0], hi = src[1];
+                if (have && n < rows_valid) {
+                    const uint32_t src = smem_u32(smem + kOffCodes + cb * kCodeBuf + k * (kRows * 32) + n * 32);
+                    const uint4 lo = lds128_ordered(src), hi = lds128_ordered(src + 16);
                     w[0] = lo.x; w[1] = lo.y; w[2] = lo.z; w[3] = lo.w;
                     w[4] = hi.x; w[5] = hi.y; w[6] = hi.z; w[7] = hi.w;
                 }
@@ -275,65 +462,49 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
                 // Word rotation V[i] = W[i - rw] as three conditional steps (rw is per thread,
                 // so no dynamically indexed register array), then the byte part with funnel
                 // shifts: out word i = bytes of V[i-1]:V[i] shifted left by 8*(r mod 4).
-                const int rw = r >> 2, rb = (r & 3) * 8;
-                uint32_t v[8];
+                uint32_t v[8], t[8];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) v[i] = w[i];
-                {
-                    uint32_t t[8];
+                for (int i = 0; i < 8; ++i) t[i] = (rw & 1) ? w[(i + 7) & 7] : w[i];
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) t[i] = (rw & 1) ? v[(i + 7) & 7] : v[i];
+                for (int i = 0; i < 8; ++i) v[i] = (rw & 2) ? t[(i + 6) & 7] : t[i];
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) v[i] = (rw & 2) ? t[(i + 6) & 7] : t[i];
+                for (int i = 0; i < 8; ++i) t[i] = (rw & 4) ? v[(i + 4) & 7] : v[i];
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) t[i] = (rw & 4) ? v[(i + 4) & 7] : v[i];
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) v[i] = t[i];
+                for (int j = 0; j < 4; ++j) {           // output word 2j + cs
+                    const uint32_t cur = cs ? t[2 * j + 1] : t[2 * j];
+                    const uint32_t prev = cs ? t[2 * j] : t[(2 * j + 7) & 7];
+                    q[k][j] = rb ? __funnelshift_l(prev, cur, rb) : cur;
                 }
-#pragma unroll
-                for (int i = 0; i < 8; ++i) cw[k][i] = rb ? __funnelshift_l(v[(i + 7) & 7], v[i], rb) : v[i];
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(&codes_empty[cb]);
 
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const int ks = sl * 4 + j;
-                if (ks >= nk) break;
-                const int st = ks % kStages;
-                if (ks >= kStages) wait_or_abort(&empty[st], ((ks / kStages) - 1) & 1, &s_abort, status);
-                unsigned char* bt = smem + kOffB + st * kBStage + (n >> 3) * 1024 + (n & 7) * 128;
+            const int nj = min(4, nk - sl * 4);
+#pragma unroll 1
+            for (int j = 0; j < nj; ++j) {
+                const int st = it % kStagesB;
+                if (it >= kStagesB) wait_or_abort(&empty_b[st], ((it / kStagesB) - 1) & 1, &s_abort, status);
+                const uint32_t bt = b_tile + st * kBStage;
+                const int g0 = sl * 32 + j * 8 + cs * 4;     // first group of the thread's four
 #pragma unroll
                 for (int cc = 0; cc < 4; ++cc) {
-                    const int c = cs * 4 + cc;                  // group within the stage
-                    const int g = sl * 32 + j * 8 + c;          // group within the row
-                    float acc[8];
+                    uint32_t code[MB];
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) acc[e] = 0.0f;
-#pragma unroll
-                    for (int k = 0; k < kGemmMaxM; ++k) {
-                        if (k < m) {
-                            // group j*8 + 4*cs + cc of the slice: word 2j + cs, byte cc
-                            const uint32_t word = cs ? cw[k][2 * j + 1] : cw[k][2 * j];
-                            const uint32_t code = (word >> (cc * 8)) & 0xffu;
-                            const uint4 q = books_s[k * 256 + code];
-                            float f[8];
-                            unpack8<BDT>(q, f);
-#pragma unroll
-                            for (int e = 0; e < 8; ++e) acc[e] += f[e];
-                        }
-                    }
-                    const bool valid = g < ng && row < out;
-                    uint4 o;
-                    o.x = valid ? pack2(acc[0], acc[1], AQ_F16) : 0u;
-                    o.y = valid ? pack2(acc[2], acc[3], AQ_F16) : 0u;
-                    o.z = valid ? pack2(acc[4], acc[5], AQ_F16) : 0u;
-                    o.w = valid ? pack2(acc[6], acc[7], AQ_F16) : 0u;
-                    *(uint4*)(bt + ((c ^ (n & 7)) << 4)) = o;
+                    for (int k = 0; k < MB; ++k) code[k] = (q[k][0] >> (cc * 8)) & 0xffu;
+                    uint4 o = decode_group<BDT, MB>(books_u, code);
+                    if (!(row_ok && g0 + cc < ng)) o = make_uint4(0u, 0u, 0u, 0u);
+                    sts128(bt + (((cs * 4 + cc) ^ (n & 7)) << 4), o);
                 }
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&full_b[st]);
+                ++it;
+#pragma unroll
+                for (int k = 0; k < MB; ++k) {
+                    q[k][0] = q[k][1];
+                    q[k][1] = q[k][2];
+                    q[k][2] = q[k][3];
+                }
             }
         }
 
@@ -346,39 +517,37 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
         const bool vec = (out & 7) == 0;
         if (ready) {
             const int q = warp & 3;                       // tensor-memory lane quarter
-            const int half = (warp - kDecWarp0) >> 2;     // token blocks 2*half, 2*half+1
-            for (int i = 2 * half; i < 2 * half + 2; ++i) {
-                const int t = t0 + i * kBM + q * 32 + lane;
-                for (int nc = 0; nc < kBN; nc += 32) {
-                    float v[32];
-                    tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + i * kBN + nc, v);
-                    if (t < tokens) {
-                        const size_t base = (size_t)t * out + n0 + nc;
-                        if (vec && n0 + nc + 32 <= out) {
-                            if (y_dt == AQ_F32) {
-                                float4* yp = (float4*)((float*)y + base);
+            const int i = (warp - kDecWarp0) >> 2;        // token block (accumulator)
+            const int t = t0 + i * 2 * kBM + (int)rank * kBM + q * 32 + lane;
+            for (int nc = 0; nc < kBN; nc += 32) {
+                float v[32];
+                tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + i * kBN + nc, v);
+                if (t < tokens) {
+                    const size_t base = (size_t)t * out + n0 + nc;
+                    if (vec && n0 + nc + 32 <= out) {
+                        if (y_dt == AQ_F32) {
+                            float4* yp = (float4*)((float*)y + base);
 #pragma unroll
-                                for (int e = 0; e < 32; e += 4)
-                                    yp[e / 4] = make_float4(v[e] * scale_s[nc + e], v[e + 1] * scale_s[nc + e + 1],
-                                                            v[e + 2] * scale_s[nc + e + 2], v[e + 3] * scale_s[nc + e + 3]);
-                            } else {
-                                uint4* yp = (uint4*)((uint16_t*)y + base);
-#pragma unroll
-                                for (int e = 0; e < 32; e += 8)
-                                    yp[e / 8] = make_uint4(pack2(v[e] * scale_s[nc + e], v[e + 1] * scale_s[nc + e + 1], y_dt),
-                                                           pack2(v[e + 2] * scale_s[nc + e + 2], v[e + 3] * scale_s[nc + e + 3], y_dt),
-                                                           pack2(v[e + 4] * scale_s[nc + e + 4], v[e + 5] * scale_s[nc + e + 5], y_dt),
-                                                           pack2(v[e + 6] * scale_s[nc + e + 6], v[e + 7] * scale_s[nc + e + 7], y_dt));
-                            }
+                            for (int e = 0; e < 32; e += 4)
+                                yp[e / 4] = make_float4(v[e] * scale_s[nc + e], v[e + 1] * scale_s[nc + e + 1],
+                                                        v[e + 2] * scale_s[nc + e + 2], v[e + 3] * scale_s[nc + e + 3]);
                         } else {
+                            uint4* yp = (uint4*)((uint16_t*)y + base);
 #pragma unroll
-                            for (int e = 0; e < 32; ++e) {
-                                if (n0 + nc + e < out) {
-                                    const float val = v[e] * scale_s[nc + e];
-                                    if (y_dt == AQ_F32) ((float*)y)[base + e] = val;
-                                    else if (y_dt == AQ_BF16) ((uint16_t*)y)[base + e] = f32_to_bits<AQ_BF16>(val);
-                                    else ((uint16_t*)y)[base + e] = f32_to_bits<AQ_F16>(val);
-                                }
+                            for (int e = 0; e < 32; e += 8)
+                                yp[e / 8] = make_uint4(pack2(v[e] * scale_s[nc + e], v[e + 1] * scale_s[nc + e + 1], y_dt),
+                                                       pack2(v[e + 2] * scale_s[nc + e + 2], v[e + 3] * scale_s[nc + e + 3], y_dt),
+                                                       pack2(v[e + 4] * scale_s[nc + e + 4], v[e + 5] * scale_s[nc + e + 5], y_dt),
+                                                       pack2(v[e + 6] * scale_s[nc + e + 6], v[e + 7] * scale_s[nc + e + 7], y_dt));
+                        }
+                    } else {
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) {
+                            if (n0 + nc + e < out) {
+                                const float val = v[e] * scale_s[nc + e];
+                                if (y_dt == AQ_F32) ((float*)y)[base + e] = val;
+                                else if (y_dt == AQ_BF16) ((uint16_t*)y)[base + e] = f32_to_bits<AQ_BF16>(val);
+                                else ((uint16_t*)y)[base + e] = f32_to_bits<AQ_F16>(val);
                             }
                         }
                     }
@@ -387,14 +556,18 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
         }
     }
 
-    // ---------------- teardown: release tensor memory once every reader is done
+    // ---------------- teardown
+    // The pair MMAs read both CTAs' shared memory and write both CTAs' tensor memory: the
+    // leader makes sure every MMA it issued has completed (the final commit always fires) and
+    // neither CTA leaves or frees tensor memory before the other is done with it.
+    if (warp == 1 && lane == 0 && rank == 0) mbar_wait(acc_full, 0);
     tc_fence_before();
-    __syncthreads();
+    cluster_sync();
     pdl_launch_dependents();
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem) : "memory");
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, 512;" ::"r"(tmem) : "memory");
     }
 }
 
@@ -454,21 +627,24 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
     std::memset(&map, 0, sizeof(map));
     const cuuint64_t dims[2] = {(cuuint64_t)d.in, (cuuint64_t)tokens};
     const cuuint64_t strides[1] = {(cuuint64_t)d.in * 2};
-    const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)(2 * kBM)};
+    const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)kBM};
     const cuuint32_t estr[2] = {1, 1};
     if (encode(&map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(x), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
         return AQ_ERR_CUDA;
 
-    auto kern = gemm_kernel<BDT>;
+    void (*kern)(const CUtensorMap, const uint8_t*, const uint16_t*, const uint16_t*, void*, int,
+                 int, unsigned int*, int, int, int, int, int, size_t) =
+        m == 1 ? gemm_kernel<BDT, 1> : m == 2 ? gemm_kernel<BDT, 2> : m == 3 ? gemm_kernel<BDT, 3>
+                                                                      : gemm_kernel<BDT, 4>;
     static std::mutex mu;
-    static bool attr_done[64] = {};
+    static bool attr_done[kGemmMaxM][64] = {};
     int dev = 0;
     if (cudaError_t e = cudaGetDevice(&dev); e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
     {
         std::lock_guard<std::mutex> lock(mu);
-        if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+        if (dev >= 0 && dev < 64 && !attr_done[m - 1][dev]) {
             if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
                 e != cudaSuccess)
                 return cuda_fail(e, "cudaFuncSetAttribute");
@@ -476,11 +652,12 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
                                                      (int)cudaSharedmemCarveoutMaxShared);
                 e != cudaSuccess)
                 return cuda_fail(e, "cudaFuncSetAttribute");
-            attr_done[dev] = true;
+            attr_done[m - 1][dev] = true;
         }
     }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((d.out + kBN - 1) / kBN, (tokens + kMT * kBM - 1) / (kMT * kBM));
+    // x: CTA pairs along the rows (cluster dimension 2), y: 512-token tiles
+    cfg.gridDim = dim3(2 * ((d.out + kBN - 1) / kBN), (tokens + kPairTokens - 1) / kPairTokens);
     cfg.blockDim = dim3(kGemmThreads);
     cfg.dynamicSmemBytes = kGemmSmem;
     cfg.stream = st;
@@ -491,7 +668,7 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
     cfg.numAttrs = 1;
     return cuda_ok(cudaLaunchKernelEx(&cfg, kern, map, (const uint8_t*)planes,
                                       (const uint16_t*)books, (const uint16_t*)scales, y, y_dt,
-                                      d.scale_dt, (unsigned int*)ws, m, tokens, d.out, d.in, d.ng,
+                                      d.scale_dt, (unsigned int*)ws, tokens, d.out, d.in, d.ng,
                                       d.rows_pad, d.plane_bytes),
                    "cudaLaunchKernelEx");
 }

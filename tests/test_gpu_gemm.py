@@ -2,7 +2,8 @@
 
 Same product tolerance as the GEMV (relative Frobenius <= 2e-3, per element
 <= 1e-2*(1+|y_ref|), against the oracle's fp64 product). Shapes cover several 512-token and
-128-row tiles, ragged token / row / input tails, fp16 and bf16 books and activations, all
+256-row pair tiles (including pairs whose second CTA has no rows), ragged token / row / input
+tails, fp16 and bf16 books and activations, all
 prefixes m <= 4 and all output types; the 70B up-projection prefill is checked on sampled
 token and row blocks that include the last ones.
 """
@@ -29,6 +30,7 @@ def gpu():
 SHAPES = [  # tokens, out, in, M, dtype
     (1, 128, 64, 1, "f16"), (128, 128, 256, 2, "bf16"), (700, 300, 520, 3, "bf16"),
     (512, 256, 512, 4, "f16"), (1030, 260, 1032, 4, "bf16"), (37, 1000, 8, 2, "f16"),
+    (600, 1288, 1032, 4, "bf16"),
 ]
 
 
