@@ -17,8 +17,11 @@
 //   warp 1      allocates the pair's tensor memory (together with the peer's warp 1). In the
 //               leader CTA (rank 0) lane 0 issues the pair MMAs (2 token blocks x 4 K=16 steps
 //               per stage) and commits stage-release / accumulator-ready barriers to both
-//               CTAs. In the peer CTA lane 0 relays "stage ready" (its activation copies landed,
-//               its decoders wrote its weight half) to the leader with a remote mbarrier arrive.
+//               CTAs; it waits on one barrier per stage. In the peer CTA lane 0 relays "stage
+//               ready" (its activation copies landed, its decoders wrote its weight half) to
+//               the leader with a remote mbarrier arrive.
+//   warp 2      (leader) lane 0 counts the leader's landed activation stages on the same
+//               stage barrier.
 //   warps 4-11  decoders: each thread owns one weight row and four groups of every stage; it
 //               sums the m codewords in fp32 (book order), rounds once to fp16 and writes the
 //               16-byte group into the B tile in the UMMA K-major 128-byte-swizzle layout.
@@ -65,7 +68,7 @@ constexpr int kOffCodes = kOffB + kStagesB * kBStage;
 constexpr int kOffBooks = kOffCodes + 2 * kCodeBuf;
 constexpr int kOffScale = kOffBooks + kGemmMaxM * 4096;
 constexpr int kOffBar = kOffScale + kBN * 4;
-// full_a, empty_a (per A stage), full_b, empty_b, peer_ready (per B stage), codes_full[2],
+// full_a, empty_a (per A stage), full_b, empty_b, ready (per B stage), codes_full[2],
 // codes_empty[2], acc_full
 constexpr int kNumBars = 2 * kStagesA + 3 * kStagesB + 4 + 1;
 constexpr int kOffTmem = kOffBar + kNumBars * 8;
@@ -282,8 +285,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
     uint64_t* empty_a = bars + kStagesA;        // the pair MMAs reading the A stage completed
     uint64_t* full_b = bars + 2 * kStagesA;     // this CTA's decoders wrote its weight half
     uint64_t* empty_b = full_b + kStagesB;      // the pair MMAs reading the B stage completed
-    uint64_t* peer_ready = empty_b + kStagesB;  // (leader) the peer's A and B stages are ready
-    uint64_t* codes_full = peer_ready + kStagesB;
+    // ready (leader only): both CTAs' A and B halves of the stage are in place. Arrivals: the
+    // leader's decoder warps, the leader's activation relay and the peer's relay.
+    uint64_t* ready = empty_b + kStagesB;
+    uint64_t* codes_full = ready + kStagesB;
     uint64_t* codes_empty = codes_full + 2;
     uint64_t* acc_full = codes_empty + 2;
     uint32_t* tmem_slot = (uint32_t*)(smem + kOffTmem);
@@ -319,9 +324,9 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
             mbar_init(&empty_a[s], 1);            // the leader's multicast commit
         }
         for (int s = 0; s < kStagesB; ++s) {
-            mbar_init(&full_b[s], kDecWarps);     // one arrival per decoder warp
+            mbar_init(&full_b[s], kDecWarps);     // (peer) one arrival per decoder warp
             mbar_init(&empty_b[s], 1);            // the leader's multicast commit
-            mbar_init(&peer_ready[s], 1);         // the peer's relay arrival
+            mbar_init(&ready[s], kDecWarps + 2);  // (leader) decoders + two relays
         }
         for (int c = 0; c < 2; ++c) {
             mbar_init(&codes_full[c], 1);
@@ -392,10 +397,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
             const uint32_t idesc = (1u << 4) | ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)((2 * kBM) >> 4) << 24);
             for (int it = 0; it < nk; ++it) {
                 const int sa = it % kStagesA, sb = it % kStagesB;
-                const uint32_t pa = (it / kStagesA) & 1, pb = (it / kStagesB) & 1;
-                if (!wait_or_abort(&full_a[sa], pa, &s_abort, status)) break;
-                if (!wait_or_abort(&full_b[sb], pb, &s_abort, status)) break;
-                if (!mbar_wait_cluster(&peer_ready[sb], pb)) {
+                if (s_abort || !mbar_wait_cluster(&ready[sb], (it / kStagesB) & 1)) {
                     record_status(status, AQ_ERR_TIMEOUT);
                     s_abort = 1;
                     break;
@@ -415,12 +417,26 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
             umma_commit_pair(acc_full);
         } else if (lane == 0) {
             // ---------------- relay (peer): this CTA's half of a stage is ready
-            const uint32_t leader_ready = map_to_rank(smem_u32(peer_ready), 0);
+            const uint32_t leader_ready = map_to_rank(smem_u32(ready), 0);
             for (int it = 0; it < nk; ++it) {
                 const int sa = it % kStagesA, sb = it % kStagesB;
                 if (!wait_or_abort(&full_a[sa], (it / kStagesA) & 1, &s_abort, status)) break;
                 if (!wait_or_abort(&full_b[sb], (it / kStagesB) & 1, &s_abort, status)) break;
                 mbar_arrive_cluster(leader_ready + sb * 8);
+            }
+        }
+    } else if (warp == 2) {
+        if (lane == 0 && rank == 0) {
+            // ---------------- activation relay (leader): its A stage landed
+            // The A ring is deeper than the stage barrier's ring, so before counting stage it
+            // the relay waits until the barrier's previous phase (stage it - kStagesB) is done.
+            for (int it = 0; it < nk; ++it) {
+                const int sa = it % kStagesA, sb = it % kStagesB;
+                if (it >= kStagesB &&
+                    !wait_or_abort(&ready[sb], ((it / kStagesB) - 1) & 1, &s_abort, status))
+                    break;
+                if (!wait_or_abort(&full_a[sa], (it / kStagesA) & 1, &s_abort, status)) break;
+                mbar_arrive(&ready[sb]);
             }
         }
     } else if (warp >= kDecWarp0) {
@@ -497,7 +513,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
                 }
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&full_b[st]);
+                if (lane == 0) mbar_arrive(rank == 0 ? &ready[st] : &full_b[st]);
                 ++it;
 #pragma unroll
                 for (int k = 0; k < MB; ++k) {
