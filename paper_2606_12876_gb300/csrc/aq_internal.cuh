@@ -141,26 +141,38 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
+// How long one try_wait may park the waiting thread (ns). The thread resumes as soon as the
+// phase completes; without a hint try_wait returns almost at once when the phase is still
+// open, and a waiting warp then spends issue slots polling that the working warps need.
+constexpr uint32_t kSuspendHintNs = 1u << 20;   // about 1 ms
+
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
         " selp.u32 %0, 1, 0, p;\n}\n"
         : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(kSuspendHintNs)
         : "memory");
     return ok != 0;
 }
 
-// Every spin-wait in this library is bounded: after kSpinLimit polls (well over a second with
-// the back-off) the wait gives up and the caller records AQ_ERR_TIMEOUT instead of hanging.
-constexpr uint32_t kSpinLimit = 1u << 22;
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Every wait in this library is bounded: after kWaitLimitNs of elapsed time it gives up and
+// the caller records AQ_ERR_TIMEOUT instead of hanging.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s
 
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-    for (uint32_t i = 0; i < kSpinLimit; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    do {
         if (mbar_try_wait(bar, parity)) return true;
-        if (i >= 4096) __nanosleep(128);
-    }
+    } while (global_ns() - t0 < kWaitLimitNs);
     return false;
 }
 
@@ -217,7 +229,7 @@ __device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
 constexpr int kFinishMax = 1024;  // items counted per round (>= the largest CTA size used)
 
 template <int SDT, typename ItemRb>
-__device__ __forceinline__ void finish_items(long long n_items, ItemRb item_rb,
+__device__ __forceinline__ void finish_items(int n_items, ItemRb item_rb,
                                              unsigned int* __restrict__ counters,
                                              const float* __restrict__ partials,
                                              const uint16_t* __restrict__ scales, void* y,
@@ -227,11 +239,11 @@ __device__ __forceinline__ void finish_items(long long n_items, ItemRb item_rb,
     const int tid = threadIdx.x;
     const size_t stride = (size_t)batch * rows_pad;
     __threadfence();                       // this thread's partial stores are visible GPU-wide
-    for (long long base = 0; base < n_items; base += blockDim.x) {
+    for (int base = 0; base < n_items; base += blockDim.x) {
         __syncthreads();
         if (tid == 0) s_n = 0;
         __syncthreads();
-        const long long j = base + tid;
+        const int j = base + tid;
         if (j < n_items) {
             const int rb = item_rb(j);
             if (atomicAdd(&counters[rb], 1u) == (unsigned)(S - 1)) s_list[atomicAdd(&s_n, 1)] = rb;
@@ -241,12 +253,12 @@ __device__ __forceinline__ void finish_items(long long n_items, ItemRb item_rb,
         // One (row, token) per thread, all of its S loads issued before the sums: the whole
         // finalisation of a CTA costs about one memory round trip.
         const int n = s_n;
-        const long long total = (long long)n * 32 * batch;
-        for (long long w = tid; w < total; w += blockDim.x) {
-            const int t = (int)(w % batch);
-            const long long e = w / batch;
+        const int total = n * 32 * batch;
+        for (int w = tid; w < total; w += blockDim.x) {
+            const int t = batch == 1 ? 0 : w % batch;
+            const int e = batch == 1 ? w : w / batch;
             const int rb = s_list[e >> 5];
-            const int r = rb * 32 + (int)(e & 31);
+            const int r = rb * 32 + (e & 31);
             const float* p = partials + (size_t)t * rows_pad + r;
             float sum = 0.0f;
             int sl = 0;

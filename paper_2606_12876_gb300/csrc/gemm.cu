@@ -113,17 +113,21 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
 
 // Bounded wait with cluster-scope acquire (for phases completed by another CTA's arrivals).
 __device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity) {
-    for (uint32_t i = 0; i < kSpinLimit; ++i) {
+    auto try_once = [&]() {
         uint32_t ok;
         asm volatile(
-            "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n"
             " selp.u32 %0, 1, 0, p;\n}\n"
             : "=r"(ok)
-            : "r"(smem_u32(bar)), "r"(parity)
+            : "r"(smem_u32(bar)), "r"(parity), "r"(kSuspendHintNs)
             : "memory");
-        if (ok) return true;
-        if (i >= 4096) __nanosleep(128);
-    }
+        return ok != 0;
+    };
+    if (try_once()) return true;
+    const uint64_t t0 = global_ns();
+    do {
+        if (try_once()) return true;
+    } while (global_ns() - t0 < kWaitLimitNs);
     return false;
 }
 

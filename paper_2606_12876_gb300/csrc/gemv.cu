@@ -64,7 +64,7 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                 const uint16_t* __restrict__ x, const uint16_t* __restrict__ scales,
                 float* __restrict__ partials, unsigned int* __restrict__ counters,
                 unsigned int* __restrict__ status, void* y, int y_dt, int m, int out, int in,
-                int ng, int rows_pad, int RBc, int S, long long total_items, size_t plane_bytes,
+                int ng, int rows_pad, int RBc, int S, int total_items, size_t plane_bytes,
                 int nslots, int cps, int static_weights) {
     extern __shared__ __align__(128) unsigned char smem[];
     unsigned char* T = smem;
@@ -77,16 +77,36 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     // Item range of this CTA: slice-aligned (cps CTAs per slice) or balanced over the grid.
-    long long i0, i1;
+    // Item indices fit in 32 bits (checked by the host); the per-stage bookkeeping below is
+    // incremental, without divisions (an integer division is a long instruction sequence).
+    int i0, i1;
     if (cps > 0) {
         const int s = blockIdx.x / cps, c = blockIdx.x % cps;
-        i0 = (long long)s * RBc + (long long)c * RBc / cps;
-        i1 = (long long)s * RBc + (long long)(c + 1) * RBc / cps;
+        i0 = s * RBc + c * RBc / cps;
+        i1 = s * RBc + (c + 1) * RBc / cps;
     } else {
-        i0 = (long long)blockIdx.x * total_items / gridDim.x;
-        i1 = (long long)(blockIdx.x + 1) * total_items / gridDim.x;
+        i0 = (int)((long long)blockIdx.x * total_items / gridDim.x);
+        i1 = (int)((long long)(blockIdx.x + 1) * total_items / gridDim.x);
     }
-    const int s_first = (int)(i0 / RBc);
+    const int s_first = i0 / RBc, rb_first = i0 - s_first * RBc;
+    // A walk over the CTA's items in stages: up to kStageRb items, never crossing a slice.
+    struct Walk {
+        int it, s, rb, n;
+    };
+    auto walk_start = [&]() {
+        Walk w{i0, s_first, rb_first, 0};
+        w.n = min(min(kStageRb, RBc - w.rb), i1 - w.it);
+        return w;
+    };
+    auto walk_next = [&](Walk& w) {
+        w.it += w.n;
+        w.rb += w.n;
+        if (w.rb == RBc) {
+            w.rb = 0;
+            ++w.s;
+        }
+        w.n = min(min(kStageRb, RBc - w.rb), i1 - w.it);
+    };
     const int npass = (m + 1) / 2;
 
     if (tid == 0) {
@@ -117,15 +137,12 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
         if (warp == kCons && lane == 0) {
             uint32_t budget = 96 * 1024;
             for (int k = 0; k < m && budget > 0; ++k)
-                for (long long it = i0; it < i1 && budget > 0;) {
-                    const long long seg_end = min(i1, (it / RBc + 1) * RBc);
-                    uint32_t bytes = (uint32_t)((seg_end - it) * 1024);
-                    if (bytes > budget) bytes = budget;
+                for (Walk w = walk_start(); w.it < i1 && budget > 0; walk_next(w)) {
+                    const uint32_t bytes = min((uint32_t)w.n * 1024u, budget);
                     prefetch_l2(planes + (size_t)k * plane_bytes +
-                                    ((size_t)(it / RBc) * rows_pad + (size_t)(it % RBc) * 32) * 32,
+                                    ((size_t)w.s * rows_pad + (size_t)w.rb * 32) * 32,
                                 bytes);
                     budget -= bytes;
-                    it = seg_end;
                 }
         }
     }
@@ -138,27 +155,22 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
     }
     __syncthreads();
 
-    // Stage sequence shared by the producer and the consumers: pass, then items in order,
-    // cut at slice boundaries and at 16 items; one ring slot per (stage, book of the pass).
-    auto stage_len = [&](long long it) {
-        const long long slice_end = (it / RBc + 1) * RBc;
-        return (int)min((long long)kStageRb, min(i1, slice_end) - it);
-    };
+    // Stage sequence shared by the producer and the consumers: pass, then the walk's stages;
+    // one ring slot per (stage, book of the pass).
 
     if (warp == kCons) {
         // ---- producer (lane 0 issues; the warp stays converged for the final barriers)
         if (lane == 0) {
-            int q = 0;
+            int q = 0, slot = 0;
+            uint32_t phase = 0;                 // parity of the slot's current use
             for (int pass = 0; pass < npass; ++pass) {
                 const int mp = min(2, m - 2 * pass);
-                for (long long it = i0; it < i1;) {
-                    const int n = stage_len(it);
-                    const size_t src =
-                        ((size_t)(it / RBc) * rows_pad + (size_t)(it % RBc) * 32) * 32;
+                for (Walk w = walk_start(); w.it < i1; walk_next(w)) {
+                    const int n = w.n;
+                    const size_t src = ((size_t)w.s * rows_pad + (size_t)w.rb * 32) * 32;
                     for (int k = 0; k < mp; ++k, ++q) {
-                        const int slot = q % nslots;
                         if (s_abort) break;
-                        if (q >= nslots && !mbar_wait(&empty[slot], ((q / nslots) - 1) & 1)) {
+                        if (q >= nslots && !mbar_wait(&empty[slot], phase ^ 1u)) {
                             record_status(status, AQ_ERR_TIMEOUT);
                             s_abort = 1;
                             break;
@@ -167,8 +179,11 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                         bulk_g2s(ring + (size_t)slot * kSlot,
                                  planes + (size_t)(2 * pass + k) * plane_bytes + src,
                                  (uint32_t)(n * 1024), &full[slot]);
+                        if (++slot == nslots) {
+                            slot = 0;
+                            phase ^= 1u;
+                        }
                     }
-                    it += n;
                 }
             }
             // No copy may be in flight when the CTA exits (bounded wait on the last slots).
@@ -195,13 +210,13 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
             goff[q] = v;
         }
 
-        int q = 0;
+        int slot = 0;
+        uint32_t phase = 0;                     // parity of the slot's current use
         for (int pass = 0; pass < npass; ++pass) {
             const int mp = min(2, m - 2 * pass);
             int cur_s = -1;
-            for (long long it = i0; it < i1;) {
-                const int n = stage_len(it);
-                const int s = (int)(it / RBc), rb = (int)(it % RBc);
+            for (Walk w = walk_start(); w.it < i1; walk_next(w)) {
+                const int n = w.n, s = w.s, rb = w.rb;
                 if (s != cur_s) {
                     // Table of the pass's books for slice s. Lane L = 8*ph + gq computes groups
                     // 4gq..4gq+3 for codewords j = 16*warp + ph + 4i: one 16-byte codeword read
@@ -247,10 +262,9 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                     cur_s = s;
                 }
                 float part = 0.0f;
-                for (int k = 0; k < mp; ++k, ++q) {
-                    const int slot = q % nslots;
+                for (int k = 0; k < mp; ++k) {
                     bool ok = !s_abort;
-                    if (ok && !mbar_wait(&full[slot], (q / nslots) & 1)) {
+                    if (ok && !mbar_wait(&full[slot], phase)) {
                         record_status(status, AQ_ERR_TIMEOUT);
                         s_abort = 1;
                         ok = false;
@@ -288,18 +302,21 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                     }
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&empty[slot]);
+                    if (++slot == nslots) {
+                        slot = 0;
+                        phase ^= 1u;
+                    }
                 }
                 if (!s_abort && warp < n) {
                     float* dst = partials + (size_t)s * rows_pad + (size_t)(rb + warp) * 32 + lane;
                     if (pass > 0) part += *dst;     // this thread wrote it in the previous pass
                     *dst = part;
                 }
-                it += n;
             }
         }
     }
     pdl_launch_dependents();
-    finish_items<SDT>(i1 - i0, [&](long long j) { return (int)((i0 + j) % RBc); }, counters,
+    finish_items<SDT>(i1 - i0, [&](int j) { return (i0 + j) % RBc; }, counters,
                       partials, scales, y, y_dt, out, rows_pad, S, 1);
 }
 
@@ -390,7 +407,7 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
             if (t < batch) partials[((size_t)s * batch + t) * rows_pad + o] = acc[t];
     }
     pdl_launch_dependents();
-    finish_items<SDT>(max(rb1 - rb0, 0), [&](long long j) { return rb0 + (int)j; }, counters,
+    finish_items<SDT>(max(rb1 - rb0, 0), [&](int j) { return rb0 + j; }, counters,
                       partials, scales, y, y_dt, out, rows_pad, S, batch);
 }
 
@@ -482,6 +499,7 @@ aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     int occ = 0;
     if (aq_status e = prepare(kern, smem, kLutThreads, m, &occ); e != AQ_OK) return e;
     const long long items = (long long)d.S * d.RBc;
+    if (items > 0x7fffffffLL) return AQ_ERR_UNSUPPORTED;   // item indices are 32-bit
     // One CTA per SM. If whole slices per CTA keep at least 90% of the SMs busy, every CTA
     // gets a single slice (one table build per book); otherwise items are balanced evenly
     // and a CTA may span two slices.
