@@ -398,7 +398,7 @@ def own_arm(args):
                 "peak_source": peak_src},
             "cpu_baseline": cpu,
             "e2e": e2e,
-            "gpu_launches": len(ms) * args.steps,
+            "gpu_launches": 2 * len(ms) * args.steps,   # product + split-K reduction per call
             "clocks": clk,
         }
         print(json.dumps(line), flush=True)

@@ -119,13 +119,15 @@ aq_status aq_decode(const aq_layout* layout, int m, const void* planes, const vo
  *   x         : device, [batch][d_in] of x_dtype (AQ_F16 or AQ_BF16), row-major
  *   y         : device, [batch][d_out] of y_dtype (AQ_F16, AQ_BF16 or AQ_F32), row-major
  *   workspace : device scratch of at least aq_gemv_workspace_bytes(layout, batch) bytes:
- *               a status word, one completion counter per 32 output rows and fp32 partial
- *               sums (one per 256-input slice, token and row). Zero-fill it once before its
+ *               a status word and fp32 partial sums (one per 256-input slice, token and
+ *               row). Zero-fill it once before its
  *               first use (aq_workspace_init); every call leaves it ready for the next one.
  *               Calls that may overlap on the GPU must not share a workspace.
- * One kernel is enqueued, with programmatic dependent launch; it waits for the preceding
- * grid before reading memory. The slices of each row are summed in a fixed order, so the
- * result does not depend on scheduling.
+ * Two kernels are enqueued, both with programmatic dependent launch: the product (fp32
+ * partial sums per 256-input slice into the workspace) and a split-K reduction that sums
+ * each row's partials, scales it and writes y. Each waits for the preceding grid before
+ * reading memory. The slices of each row are summed in a fixed order, so the result does
+ * not depend on scheduling.
  * Accuracy: |y - y_exact| <= 1e-2*(1+|y_exact|) per element and relative Frobenius error
  * <= 2e-3, with y_exact the fp64 product of the exactly widened stored values. */
 size_t aq_gemv_workspace_bytes(const aq_layout* layout, int batch);
@@ -146,7 +148,7 @@ aq_status aq_gemv(const aq_layout* layout, int m, const void* planes, const void
  *     AQ_STATIC_SCRATCH_BYTES; use aq_gemv with a workspace for such sizes.
  *   - The first call on a device looks up the buffer's device address; make that first call
  *     on each device before capturing any stream on it.
- *   - Each call enqueues a clear of the buffer's status word and counters, then the GEMV.
+ *   - Each call enqueues a clear of the buffer's status word, then the GEMV.
  *   - Every call on a device shares the one buffer, which keeps the last call's contents:
  *     calls that may overlap on the GPU (other streams, other host threads) race on it and
  *     must be ordered by the caller. */

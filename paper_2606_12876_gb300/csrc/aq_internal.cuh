@@ -34,13 +34,11 @@ struct DeviceInfo {
 };
 aq_status device_info(DeviceInfo* info);
 
-// Workspace layout of the split-K GEMV:
-//   [status word, 256 B][one u32 completion counter per 32-row block][fp32 partials
-//   [S][batch][rows_pad]]. Counters start at zero and are returned to zero by each call.
+// Workspace layout of the split-K GEMV: [status word, 256 B][fp32 partials
+// [units][batch][rows_pad]], written by the product kernel and read by the reduction.
 constexpr size_t kWsStatusBytes = 256;
 inline size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
-inline size_t ws_counter_bytes(const Dims& d) { return round_up((size_t)d.RBc * 4, 256); }
-inline size_t ws_partial_offset(const Dims& d) { return kWsStatusBytes + ws_counter_bytes(d); }
+inline size_t ws_partial_offset(const Dims&) { return kWsStatusBytes; }
 
 // Records a failed CUDA call (thread-local text for aq_last_error) and returns AQ_ERR_CUDA.
 aq_status cuda_fail(cudaError_t e, const char* what);
@@ -209,78 +207,23 @@ __device__ __forceinline__ void named_barrier(int id, int threads) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
+// Packed fp32 pair add (each lane rounded to nearest, as a scalar add): d = a + b.
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+    unsigned long long ar, br, dr;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(ar) : "f"(a.x), "f"(a.y));
+    asm("mov.b64 %0, {%1, %2};" : "=l"(br) : "f"(b.x), "f"(b.y));
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(dr) : "l"(ar), "l"(br));
+    float2 d;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(dr));
+    return d;
+}
+
 // Packed fp32 pair FMA (one instruction for two lanes of work): d = a * b + c.
 __device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
     unsigned long long ar = *(unsigned long long*)&a, br = *(unsigned long long*)&b,
                        cr = *(unsigned long long*)&c, dr;
     asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(dr) : "l"(ar), "l"(br), "l"(cr));
     return *(float2*)&dr;
-}
-
-// ---- split-K completion ------------------------------------------------------------------
-//
-// A work item is (slice s, 32-row block rb); its fp32 partial sums for the block's rows (and
-// every token) sit in partials[s][t][row]. When a CTA has written all its items it counts
-// each item on the block's counter; whoever brings a counter to S (all slices done) sums the
-// S partials of that block in slice order, applies the row scale (R1: s[o] multiplies the
-// codebook sum, so it factors out of the dot product), stores y and resets the counter.
-// The outcome does not depend on which CTA finishes last. Every thread of the CTA must call
-// this with the same n_items (it contains CTA-wide barriers).
-constexpr int kFinishMax = 1024;  // items counted per round (>= the largest CTA size used)
-
-template <int SDT, typename ItemRb>
-__device__ __forceinline__ void finish_items(int n_items, ItemRb item_rb,
-                                             unsigned int* __restrict__ counters,
-                                             const float* __restrict__ partials,
-                                             const uint16_t* __restrict__ scales, void* y,
-                                             int y_dt, int out, int rows_pad, int S, int batch) {
-    __shared__ int s_list[kFinishMax];
-    __shared__ int s_n;
-    const int tid = threadIdx.x;
-    const size_t stride = (size_t)batch * rows_pad;
-    __threadfence();                       // this thread's partial stores are visible GPU-wide
-    for (int base = 0; base < n_items; base += blockDim.x) {
-        __syncthreads();
-        if (tid == 0) s_n = 0;
-        __syncthreads();
-        const int j = base + tid;
-        if (j < n_items) {
-            const int rb = item_rb(j);
-            if (atomicAdd(&counters[rb], 1u) == (unsigned)(S - 1)) s_list[atomicAdd(&s_n, 1)] = rb;
-        }
-        __syncthreads();
-        __threadfence();                   // order the counter reads before the partial reads
-        // One (row, token) per thread, all of its S loads issued before the sums: the whole
-        // finalisation of a CTA costs about one memory round trip.
-        const int n = s_n;
-        const int total = n * 32 * batch;
-        for (int w = tid; w < total; w += blockDim.x) {
-            const int t = batch == 1 ? 0 : w % batch;
-            const int e = batch == 1 ? w : w / batch;
-            const int rb = s_list[e >> 5];
-            const int r = rb * 32 + (e & 31);
-            const float* p = partials + (size_t)t * rows_pad + r;
-            float sum = 0.0f;
-            int sl = 0;
-            for (; sl + 16 <= S; sl += 16) {
-                float v[16];
-#pragma unroll
-                for (int q = 0; q < 16; ++q) v[q] = __ldcg(p + (size_t)(sl + q) * stride);
-#pragma unroll
-                for (int q = 0; q < 16; ++q) sum += v[q];
-            }
-            for (; sl < S; ++sl) sum += __ldcg(p + (size_t)sl * stride);
-            if (r < out) {
-                const float v = sum * bits_to_f32<SDT>(scales[r]);
-                const size_t yi = (size_t)t * out + r;
-                if (y_dt == AQ_F32) ((float*)y)[yi] = v;
-                else if (y_dt == AQ_F16) ((uint16_t*)y)[yi] = f32_to_bits<AQ_F16>(v);
-                else ((uint16_t*)y)[yi] = f32_to_bits<AQ_BF16>(v);
-            }
-        }
-        __syncthreads();
-        for (int e = tid; e < n; e += blockDim.x) counters[s_list[e]] = 0u;
-    }
 }
 
 }  // namespace aq

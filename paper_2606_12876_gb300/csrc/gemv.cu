@@ -3,9 +3,10 @@
 //
 // Work split (split-K): the input dimension is cut into slices of 32 groups (256 inputs).
 // A work item is (slice, 32-row block). Each item reads the first m code planes of its rows
-// once and writes one fp32 partial per (row, token). When all slices of a 32-row block are
-// written, the CTA that counted the last one sums them in slice order (deterministic), scales
-// the rows and stores y (finish_items).
+// once and writes one fp32 partial per (row, token). A second, small kernel (splitk_reduce,
+// launched right behind with programmatic dependent launch, so its CTAs are already resident
+// when the product finishes) sums each row's partials in slice order (deterministic), scales
+// the row and stores y, with the rows spread evenly over the GPU.
 //
 // Two product kernels:
 //  * gemv_lut (B = 8, one token, m <= 4). By linearity, x_g . (sum_k C_k[b_k]) =
@@ -61,9 +62,7 @@ inline size_t lut_smem_bytes(int m, int slots) {
 template <int BDT, int XDT, int SDT>
 __global__ void __launch_bounds__(kLutThreads, 1)
 gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
-                const uint16_t* __restrict__ x, const uint16_t* __restrict__ scales,
-                float* __restrict__ partials, unsigned int* __restrict__ counters,
-                unsigned int* __restrict__ status, void* y, int y_dt, int m, int out, int in,
+                const uint16_t* __restrict__ x, float* __restrict__ partials, unsigned int* __restrict__ status, int m, int in,
                 int ng, int rows_pad, int RBc, int S, int total_items, size_t plane_bytes,
                 int nslots, int cps, int static_weights) {
     extern __shared__ __align__(128) unsigned char smem[];
@@ -147,6 +146,7 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
         }
     }
     pdl_wait();                 // inputs may come from the preceding kernel in the stream
+    pdl_launch_dependents();    // the split-K reduction may become resident (it waits for us)
     if (!static_weights) load_books();
     uint2 x_r = make_uint2(0u, 0u);
     if (tid < kXSlices * 64) {
@@ -200,13 +200,18 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
         if (tid < kXSlices * 64) *(uint2*)(xs + (tid >> 6) * 512 + (tid & 63) * 8) = x_r;
         named_barrier(1, kCons * 32);   // staged codebooks and activations visible to all consumers
 
-        // goff[q] byte i = 4 * group-in-slice read at position 4q+i by this lane.
+        // Each lane reads its row's 32 code bytes as two 16-byte halves; lanes 4-7 of every
+        // eight read the second half first (no bank conflicts between the two reads).
+        // goff[q] byte i = 4 * group at byte 4q+i of what this lane read, in its read order
+        // (position p of row o holds group (p + o) mod 32).
+        const int c0 = (lane >> 2) & 1;
         uint32_t goff[8];
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
             uint32_t v = 0;
 #pragma unroll
-            for (int i = 0; i < 4; ++i) v |= (uint32_t)(((4 * q + i + lane) & 31) * 4) << (8 * i);
+            for (int i = 0; i < 4; ++i)
+                v |= (uint32_t)((((4 * q + i + (c0 ? 16 : 0)) + lane) & 31) * 4) << (8 * i);
             goff[q] = v;
         }
 
@@ -270,35 +275,23 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                         ok = false;
                     }
                     if (ok && warp < n) {
-                        // Lanes 4-7 of each group of eight read their two 16-byte halves in the
-                        // other order, which keeps the two reads free of bank conflicts.
-                        const uint4* src = (const uint4*)(ring + (size_t)slot * kSlot + warp * 1024 + lane * 32);
-                        const int c0 = (lane >> 2) & 1;
-                        const uint4 r0 = src[c0], r1 = src[c0 ^ 1];
-                        const uint4 a = c0 ? r1 : r0, b = c0 ? r0 : r1;
+                        const unsigned char* row = ring + (size_t)slot * kSlot + warp * 1024 + lane * 32;
+                        const uint4 a = *(const uint4*)(row + c0 * 16);
+                        const uint4 b = *(const uint4*)(row + (c0 ^ 1) * 16);
                         const uint32_t wd[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
                         const uint32_t Tk = smem_u32(T) + k * 128;
-                        float acc[8];
+                        float2 acc = make_float2(0.0f, 0.0f);
 #pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-                            uint32_t off[16];
-#pragma unroll
-                            for (int qq = 0; qq < 4; ++qq) {
-                                // byte0 = goff byte i, byte1 = code byte i, bytes 2-3 = sign of goff byte (0)
-                                const uint32_t w = wd[4 * h + qq], g = goff[4 * h + qq];
-                                off[4 * qq + 0] = prmt(w, g, 0xCC04u);
-                                off[4 * qq + 1] = prmt(w, g, 0xDD15u);
-                                off[4 * qq + 2] = prmt(w, g, 0xEE26u);
-                                off[4 * qq + 3] = prmt(w, g, 0xFF37u);
-                            }
-                            float v[16];
-#pragma unroll
-                            for (int i = 0; i < 16; ++i) v[i] = lds_f32(Tk + off[i]);
-#pragma unroll
-                            for (int qq = 0; qq < 4; ++qq)
-                                acc[4 * h + qq] = (v[4 * qq] + v[4 * qq + 1]) + (v[4 * qq + 2] + v[4 * qq + 3]);
+                        for (int qq = 0; qq < 8; ++qq) {
+                            // byte0 = goff byte i, byte1 = code byte i, bytes 2-3 = sign of goff byte (0)
+                            const uint32_t w = wd[qq], g = goff[qq];
+                            const float v0 = lds_f32(Tk + prmt(w, g, 0xCC04u));
+                            const float v1 = lds_f32(Tk + prmt(w, g, 0xDD15u));
+                            const float v2 = lds_f32(Tk + prmt(w, g, 0xEE26u));
+                            const float v3 = lds_f32(Tk + prmt(w, g, 0xFF37u));
+                            acc = add2(acc, add2(make_float2(v0, v1), make_float2(v2, v3)));
                         }
-                        part += ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+                        part += acc.x + acc.y;
                     }
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&empty[slot]);
@@ -315,9 +308,6 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
             }
         }
     }
-    pdl_launch_dependents();
-    finish_items<SDT>(i1 - i0, [&](int j) { return (i0 + j) % RBc; }, counters,
-                      partials, scales, y, y_dt, out, rows_pad, S, 1);
 }
 
 // ------------------------------------------------------------------ direct kernel (any B, b <= 16)
@@ -325,9 +315,7 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
 template <int NB, int B, int BDT, int SDT>
 __global__ void __launch_bounds__(256)
 gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
-                   const uint16_t* __restrict__ x, int x_dt, const uint16_t* __restrict__ scales,
-                   float* __restrict__ partials, unsigned int* __restrict__ counters, void* y,
-                   int y_dt, int out, int m, int batch, int in, int rows_pad, int RBc, int S,
+                   const uint16_t* __restrict__ x, int x_dt, float* __restrict__ partials, int m, int batch, int in, int rows_pad, int RBc,
                    int rb_per_chunk, size_t plane_bytes) {
     constexpr int ESZ = B / 8;
     constexpr int UNIT = 32 * ESZ;
@@ -341,6 +329,7 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
     const int s = blockIdx.y, chunk = blockIdx.x;
 
     pdl_wait();
+    pdl_launch_dependents();
     for (int i = tid; i < NB * 256; i += 256) {
         const int t = i >> 8, c = i & 255;
         const int col = s * 256 + c;
@@ -406,9 +395,38 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
         for (int t = 0; t < NB; ++t)
             if (t < batch) partials[((size_t)s * batch + t) * rows_pad + o] = acc[t];
     }
+}
+
+// ------------------------------------------------------------------ split-K reduction
+
+// y[t][r] = s[r] * sum over the S slices of partials[s][t][r], in slice order (R1: the row
+// scale multiplies the codebook sum, so it factors out of the dot product). One thread per
+// (row, token); all of a thread's loads are issued before the additions.
+template <int SDT>
+__global__ void __launch_bounds__(256)
+splitk_reduce_kernel(const float* __restrict__ partials, const uint16_t* __restrict__ scales,
+                     void* y, int y_dt, int out, int rows_pad, int S, int batch) {
+    pdl_wait();                 // the product kernel's partials
     pdl_launch_dependents();
-    finish_items<SDT>(max(rb1 - rb0, 0), [&](int j) { return rb0 + j; }, counters,
-                      partials, scales, y, y_dt, out, rows_pad, S, batch);
+    const int r = blockIdx.x * blockDim.x + threadIdx.x, t = blockIdx.y;
+    if (r >= out) return;
+    const size_t stride = (size_t)batch * rows_pad;
+    const float* p = partials + (size_t)t * rows_pad + r;
+    float sum = 0.0f;
+    int sl = 0;
+    for (; sl + 16 <= S; sl += 16) {
+        float v[16];
+#pragma unroll
+        for (int q = 0; q < 16; ++q) v[q] = __ldcg(p + (size_t)(sl + q) * stride);
+#pragma unroll
+        for (int q = 0; q < 16; ++q) sum += v[q];
+    }
+    for (; sl < S; ++sl) sum += __ldcg(p + (size_t)sl * stride);
+    const float v = sum * bits_to_f32<SDT>(scales[r]);
+    const size_t yi = (size_t)t * out + r;
+    if (y_dt == AQ_F32) ((float*)y)[yi] = v;
+    else if (y_dt == AQ_F16) ((uint16_t*)y)[yi] = f32_to_bits<AQ_F16>(v);
+    else ((uint16_t*)y)[yi] = f32_to_bits<AQ_BF16>(v);
 }
 
 // ------------------------------------------------------------------ host side
@@ -481,7 +499,6 @@ struct GemvArgs {
     void* y;
     int y_dt;
     float* partials;
-    unsigned int* counters;
     unsigned int* status;
 };
 
@@ -513,8 +530,8 @@ aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
         grid = (int)(items < di.sms ? items : di.sms);
     }
     return launch_pdl(kern, dim3(grid), dim3(kLutThreads), smem, st, (const uint8_t*)a.planes,
-                      (const uint16_t*)a.books, (const uint16_t*)a.x, (const uint16_t*)a.scales,
-                      a.partials, a.counters, a.status, a.y, a.y_dt, m, d.out, d.in, d.ng,
+                      (const uint16_t*)a.books, (const uint16_t*)a.x, a.partials, a.status, m,
+                      d.in, d.ng,
                       d.rows_pad, d.RBc, d.S, items, d.plane_bytes, nslots, cps,
                       (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0);
 }
@@ -535,8 +552,7 @@ aq_status run_direct(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     chunks = (d.RBc + rbpc - 1) / rbpc;
     return launch_pdl(kern, dim3(chunks, d.S), dim3(256), smem, st, (const uint8_t*)a.planes,
                       (const uint16_t*)a.books, (const uint16_t*)a.x, a.x_dt,
-                      (const uint16_t*)a.scales, a.partials, a.counters, a.y, a.y_dt, d.out, m,
-                      a.batch, d.in, d.rows_pad, d.RBc, d.S, rbpc, d.plane_bytes);
+                      a.partials, m, a.batch, d.in, d.rows_pad, d.RBc, rbpc, d.plane_bytes);
 }
 
 template <int B, int BDT, int SDT>
@@ -550,13 +566,13 @@ aq_status dispatch_direct(const Dims& d, int m, const GemvArgs& a, cudaStream_t 
 
 }  // namespace
 
-aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* books,
-                      const void* scales, const void* x, int x_dt, int batch, void* y,
-                      int y_dt, void* ws, cudaStream_t st) {
+// The product kernel of aq_gemv: fp32 partial sums per (slice, token, row) into the workspace.
+static aq_status launch_product(const Dims& d, int m, const void* planes, const void* books,
+                                const void* scales, const void* x, int x_dt, int batch, void* y,
+                                int y_dt, void* ws, cudaStream_t st) {
     if (d.out == 0 || batch == 0) return AQ_OK;
     GemvArgs a{planes, books, scales, x, x_dt, batch, y, y_dt,
-               (float*)((char*)ws + ws_partial_offset(d)),
-               (unsigned int*)((char*)ws + kWsStatusBytes), (unsigned int*)ws};
+               (float*)((char*)ws + ws_partial_offset(d)), (unsigned int*)ws};
     const int bb = d.book_dt == AQ_BF16, xb = x_dt == AQ_BF16, sb = d.scale_dt == AQ_BF16;
     if (d.B == 8 && batch == 1 && m <= kLutMaxM) {
         switch (bb * 4 + xb * 2 + sb) {
@@ -580,6 +596,25 @@ aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* book
         case 6: return dispatch_direct<16, AQ_BF16, AQ_F16>(d, m, a, st);
         default: return dispatch_direct<16, AQ_BF16, AQ_BF16>(d, m, a, st);
     }
+}
+
+template <int SDT>
+static aq_status launch_reduce(const Dims& d, const GemvArgs& a, cudaStream_t st) {
+    return launch_pdl(splitk_reduce_kernel<SDT>, dim3((d.out + 255) / 256, a.batch), dim3(256),
+                      0, st, (const float*)a.partials, (const uint16_t*)a.scales, a.y, a.y_dt,
+                      d.out, d.rows_pad, d.S, a.batch);
+}
+
+aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* books,
+                      const void* scales, const void* x, int x_dt, int batch, void* y,
+                      int y_dt, void* ws, cudaStream_t st) {
+    if (d.out == 0 || batch == 0) return AQ_OK;
+    if (aq_status e = launch_product(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
+        e != AQ_OK)
+        return e;
+    GemvArgs a{planes, books, scales, x, x_dt, batch, y, y_dt,
+               (float*)((char*)ws + ws_partial_offset(d)), (unsigned int*)ws};
+    return d.scale_dt == AQ_BF16 ? launch_reduce<AQ_BF16>(d, a, st) : launch_reduce<AQ_F16>(d, a, st);
 }
 
 }  // namespace aq

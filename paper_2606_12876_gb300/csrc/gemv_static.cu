@@ -5,7 +5,7 @@
 // allocate after start-up (an allocation can synchronise the device or fail under memory
 // pressure), or code whose device footprint has to be fixed and known in advance. They cannot
 // provide the workspace that aq_gemv needs either. This entry point takes that scratch
-// (status word, completion counters, per-slice partial sums) from a fixed buffer that lives
+// (status word and per-slice partial sums) from a fixed buffer that lives
 // in this file as a device array, so a call allocates nothing.
 #include <mutex>
 
@@ -57,8 +57,8 @@ extern "C" aq_status aq_gemv_static_scratch(const aq_layout* layout, int m, cons
 
     void* scratch = nullptr;
     if (aq_status e = static_scratch_address(&scratch); e != AQ_OK) return e;
-    // The buffer keeps whatever the previous call left; the status word and the counters
-    // must start at zero, so clear them (the partial sums are always written before read).
+    // The buffer keeps whatever the previous call left; the status word must start at zero,
+    // so clear it (the partial sums are always written before they are read).
     if (cudaError_t e = cudaMemsetAsync(scratch, 0, aq::ws_partial_offset(d), (cudaStream_t)stream);
         e != cudaSuccess)
         return aq::cuda_fail(e, "cudaMemsetAsync");
