@@ -108,6 +108,33 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
     };
     const int npass = (m + 1) / 2;
 
+    // Producer state (warp kCons, lane 0): the next copy is book 2*p_pass + p_k of stage p_w,
+    // into ring slot p_slot (use parity p_phase); p_q copies issued so far.
+    int p_q = 0, p_slot = 0, p_pass = 0, p_k = 0;
+    uint32_t p_phase = 0;
+    Walk p_w = walk_start();
+    if (i0 >= i1) p_pass = npass;
+    auto issue_next = [&]() {
+        const int mp = min(2, m - 2 * p_pass);
+        const size_t src = ((size_t)p_w.s * rows_pad + (size_t)p_w.rb * 32) * 32;
+        mbar_arrive_expect_tx(&full[p_slot], (uint32_t)(p_w.n * 1024));
+        bulk_g2s(ring + (size_t)p_slot * kSlot,
+                 planes + (size_t)(2 * p_pass + p_k) * plane_bytes + src,
+                 (uint32_t)(p_w.n * 1024), &full[p_slot]);
+        ++p_q;
+        if (++p_slot == nslots) {
+            p_slot = 0;
+            p_phase ^= 1u;
+        }
+        if (++p_k == mp) {
+            p_k = 0;
+            walk_next(p_w);
+            if (p_w.it >= i1) {
+                ++p_pass;
+                p_w = walk_start();
+            }
+        }
+    };
     if (tid == 0) {
         for (int d = 0; d < nslots; ++d) {
             mbar_init(&full[d], 1);
@@ -116,6 +143,7 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
         mbar_fence_init();
         s_abort = 0;
     }
+    __syncthreads();            // barriers initialised before the first copy
     // Codebooks and activations are requested first (into registers); the producer starts
     // its copies only after every thread has issued these loads (the barrier below).
     // (consumer threads only: they are the ones that store the codebooks below)
@@ -129,21 +157,13 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
         }
     };
     if (static_weights) {
-        // The weights are read-only while calls run (AQ_LAYOUT_STATIC_WEIGHTS): stage the
-        // codebooks and pull the first code stages of this CTA into L2 before waiting for the
-        // preceding kernel, so that traffic overlaps its tail.
+        // The weights are read-only while calls run (AQ_LAYOUT_STATIC_WEIGHTS): request the
+        // codebooks before waiting for the preceding kernel.
         load_books();
-        if (warp == kCons && lane == 0) {
-            uint32_t budget = 96 * 1024;
-            for (int k = 0; k < m && budget > 0; ++k)
-                for (Walk w = walk_start(); w.it < i1 && budget > 0; walk_next(w)) {
-                    const uint32_t bytes = min((uint32_t)w.n * 1024u, budget);
-                    prefetch_l2(planes + (size_t)k * plane_bytes +
-                                    ((size_t)w.s * rows_pad + (size_t)w.rb * 32) * 32,
-                                bytes);
-                    budget -= bytes;
-                }
-        }
+        // The code planes are read-only too: fill the ring before waiting for the preceding
+        // kernel, so the first stages overlap its tail.
+        if (warp == kCons && lane == 0)
+            while (p_q < nslots && p_pass < npass) issue_next();
     }
     pdl_wait();                 // inputs may come from the preceding kernel in the stream
     pdl_launch_dependents();    // the split-K reduction may become resident (it waits for us)
@@ -161,33 +181,17 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
     if (warp == kCons) {
         // ---- producer (lane 0 issues; the warp stays converged for the final barriers)
         if (lane == 0) {
-            int q = 0, slot = 0;
-            uint32_t phase = 0;                 // parity of the slot's current use
-            for (int pass = 0; pass < npass; ++pass) {
-                const int mp = min(2, m - 2 * pass);
-                for (Walk w = walk_start(); w.it < i1; walk_next(w)) {
-                    const int n = w.n;
-                    const size_t src = ((size_t)w.s * rows_pad + (size_t)w.rb * 32) * 32;
-                    for (int k = 0; k < mp; ++k, ++q) {
-                        if (s_abort) break;
-                        if (q >= nslots && !mbar_wait(&empty[slot], phase ^ 1u)) {
-                            record_status(status, AQ_ERR_TIMEOUT);
-                            s_abort = 1;
-                            break;
-                        }
-                        mbar_arrive_expect_tx(&full[slot], (uint32_t)(n * 1024));
-                        bulk_g2s(ring + (size_t)slot * kSlot,
-                                 planes + (size_t)(2 * pass + k) * plane_bytes + src,
-                                 (uint32_t)(n * 1024), &full[slot]);
-                        if (++slot == nslots) {
-                            slot = 0;
-                            phase ^= 1u;
-                        }
-                    }
+            while (p_pass < npass) {
+                if (s_abort) break;
+                if (p_q >= nslots && !mbar_wait(&empty[p_slot], p_phase ^ 1u)) {
+                    record_status(status, AQ_ERR_TIMEOUT);
+                    s_abort = 1;
+                    break;
                 }
+                issue_next();
             }
             // No copy may be in flight when the CTA exits (bounded wait on the last slots).
-            for (int j = max(0, q - nslots); j < q; ++j) mbar_wait(&full[j % nslots], (j / nslots) & 1);
+            for (int j = max(0, p_q - nslots); j < p_q; ++j) mbar_wait(&full[j % nslots], (j / nslots) & 1);
         }
         __syncwarp();
     } else {
