@@ -2,27 +2,31 @@
 // (the prefix-m additive reconstruction of Sec. 3.2 / Sec. 5) decoded tile by tile into shared
 // memory and never written to HBM.
 //
-// A cluster of two CTAs (one CTA pair, one CTA per SM) computes a 512-token x 256-row tile with
-// pair MMAs (tcgen05.mma.cta_group::2, M = 256 tokens, N = 256 rows, K = 16): each CTA holds
-// 128 tokens of every A block and decodes its own 128 of the 256 weight rows, and the MMA
-// reads both halves of both operands, so every SM supplies half the operand bytes of what a
-// single-CTA MMA of the same work would read from its shared memory. Shared-memory bandwidth is
-// what the decoders' codeword gathers compete for, so this is the main point of the pair.
+// A CTA pair (two CTAs, one per SM) computes a 512-token x 256-row tile with pair MMAs
+// (tcgen05.mma.cta_group::2, M = 256 tokens, N = 256 rows, K = 16): each CTA holds 128 tokens
+// of every A block and 128 of the 256 weight rows, and the MMA reads both halves of both
+// operands, so every SM supplies half the operand bytes of what a single-CTA MMA of the same
+// work would read from its shared memory. A cluster holds two such pairs with the same rows and
+// consecutive token tiles. The CTA with the same role in the other pair (the partner) needs the
+// same 128 weight rows: each of the two decodes 64 of them and sends its slab to the other
+// with one shared-memory bulk copy per stage, which halves the codeword gathers (the decoders'
+// shared-memory traffic, what bounds the kernel at larger m).
 // Each CTA's tensor memory holds its 128 tokens x 256 rows for two token blocks (512 columns).
 // Roles (12 warps per CTA):
 //   warp 0      TMA producer: activation tiles (2-D tensor map, 128-byte swizzle, two
-//               128-token boxes per stage) and, once per 256-input slice, this CTA's code rows
-//               of the first m planes (1-D bulk copies; a CTA's rows of a slice are contiguous
-//               in every plane).
+//               128-token boxes per stage) and, once per 256-input slice, the code rows this
+//               CTA decodes, of the first m planes (1-D bulk copies).
 //   warp 1      allocates the pair's tensor memory (together with the peer's warp 1). In the
-//               leader CTA (rank 0) lane 0 issues the pair MMAs (2 token blocks x 4 K=16 steps
-//               per stage) and commits stage-release / accumulator-ready barriers to both
-//               CTAs; it waits on one barrier per stage. In the peer CTA lane 0 relays "stage
-//               ready" (its activation copies landed, its decoders wrote its weight half) to
-//               the leader with a remote mbarrier arrive.
-//   warp 2      (leader) lane 0 counts the leader's landed activation stages on the same
-//               stage barrier.
-//   warps 4-11  decoders: each thread owns one weight row and four groups of every stage; it
+//               leader CTA of a pair lane 0 issues the pair MMAs (2 token blocks x 4 K=16
+//               steps per stage) after one barrier wait per stage, and commits the
+//               activation-stage release and accumulator-ready barriers to its pair and the
+//               weight-stage release to all four CTAs. In the peer CTA lane 0 relays "stage
+//               ready" (its activations landed, its weight operand complete) to the leader
+//               with a remote mbarrier arrive.
+//   warp 2      (leader) lane 0 counts the leader's landed activation stages on the stage
+//               barrier.
+//   warp 3      lane 0 copies this CTA's decoded slab of each stage to the partner.
+//   warps 4-11  decoders: each thread owns one weight row and two groups of every stage; it
 //               sums the m codewords in fp32 (book order), rounds once to fp16 and writes the
 //               16-byte group into the B tile in the UMMA K-major 128-byte-swizzle layout.
 //               Afterwards the same warps are the epilogue: tcgen05.ld from tensor memory,
@@ -58,6 +62,8 @@ constexpr int kGemmMaxM = 4;
 constexpr int kABlock = kBM * 128;            // one 128-token x 64-input block (16 KiB)
 constexpr int kAStage = kAcc * kABlock;       // 32 KiB
 constexpr int kBStage = kRows * 128;          // 16 KiB
+constexpr int kHalfRows = kRows / 2;          // rows decoded by one CTA (shared with its partner)
+constexpr int kHalfBytes = kHalfRows * 128;    // their 64-input slab of a weight stage (8 KiB)
 constexpr int kCodeBuf = kGemmMaxM * kRows * 32;   // one slice of codes, all planes (16 KiB)
 
 // Shared-memory map (offsets from a 1024-byte aligned base; identical in both CTAs of a pair,
@@ -68,9 +74,9 @@ constexpr int kOffCodes = kOffB + kStagesB * kBStage;
 constexpr int kOffBooks = kOffCodes + 2 * kCodeBuf;
 constexpr int kOffScale = kOffBooks + kGemmMaxM * 4096;
 constexpr int kOffBar = kOffScale + kBN * 4;
-// full_a, empty_a (per A stage), full_b, empty_b, ready (per B stage), codes_full[2],
+// full_a, empty_a (per A stage), full_b, empty_b, ready, dec_done (per B stage), codes_full[2],
 // codes_empty[2], acc_full
-constexpr int kNumBars = 2 * kStagesA + 3 * kStagesB + 4 + 1;
+constexpr int kNumBars = 2 * kStagesA + 4 * kStagesB + 4 + 1;
 constexpr int kOffTmem = kOffBar + kNumBars * 8;
 constexpr int kOffAbort = kOffTmem + 16;
 // The kernel has no static shared memory, so its dynamic shared memory starts on a 1024-byte
@@ -109,6 +115,17 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
 // half a microsecond per stage, which alone exceeds a stage's MMA time.
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
     asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+// Bulk copy from this CTA's shared memory to another CTA's (cluster addresses for the
+// destination and its mbarrier), completing on that mbarrier's transaction count.
+__device__ __forceinline__ void bulk_to_peer(uint32_t dst_cluster, uint32_t src, uint32_t bytes,
+                                             uint32_t bar_cluster) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            dst_cluster),
+        "r"(src), "r"(bytes), "r"(bar_cluster)
+        : "memory");
 }
 
 // Bounded wait with cluster-scope acquire (for phases completed by another CTA's arrivals).
@@ -154,10 +171,9 @@ __device__ __forceinline__ void umma_f16_pair(uint32_t d_tmem, uint64_t a_desc, 
         : "memory");
 }
 
-// Arrive on the barrier at local offset `bar` in both CTAs of the pair once every prior pair
-// MMA of this thread has completed.
-__device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
-    const uint16_t mask = 0x3;
+// Arrive on the barrier at local offset `bar` in every CTA of `mask` (cluster ranks) once every
+// prior pair MMA of this thread has completed.
+__device__ __forceinline__ void umma_commit_pair(uint64_t* bar, uint16_t mask) {
     asm volatile(
         "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
         " [%0], %1;" ::"r"(smem_u32(bar)), "h"(mask)
@@ -276,9 +292,13 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
 }
 
 // One instantiation per book type and prefix length MB (= m): the decoders' code holds exactly
-// the lookups of that prefix.
-template <int BDT, int MB>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
+// the lookups of that prefix. SHARE: clusters of four CTAs (two pairs) that split the decode
+// of each weight operand between partners (launched with cluster size 4); otherwise clusters
+// of one pair (cluster size 2), each CTA decoding its own 128 rows. Sharing pays when the
+// gathers bound the kernel (m >= 2); at m = 1 the SMs that clusters of four leave idle cost
+// more than it saves.
+template <int BDT, int MB, bool SHARE>
+__global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ planes,
             const uint16_t* __restrict__ books, const uint16_t* __restrict__ scales, void* y,
             int y_dt, int scale_dt, unsigned int* __restrict__ status, int tokens, int out,
@@ -290,9 +310,11 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
     uint64_t* full_b = bars + 2 * kStagesA;     // this CTA's decoders wrote its weight half
     uint64_t* empty_b = full_b + kStagesB;      // the pair MMAs reading the B stage completed
     // ready (leader only): both CTAs' A and B halves of the stage are in place. Arrivals: the
-    // leader's decoder warps, the leader's activation relay and the peer's relay.
+    // leader's decoder warps (or, when sharing, its copier with the partner's bytes), the
+    // leader's activation relay and the peer's relay.
     uint64_t* ready = empty_b + kStagesB;
-    uint64_t* codes_full = ready + kStagesB;
+    uint64_t* dec_done = ready + kStagesB;      // this CTA's decoders wrote their half
+    uint64_t* codes_full = dec_done + kStagesB;
     uint64_t* codes_empty = codes_full + 2;
     uint64_t* acc_full = codes_empty + 2;
     uint32_t* tmem_slot = (uint32_t*)(smem + kOffTmem);
@@ -302,19 +324,28 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
     volatile int& s_abort = *(volatile int*)(smem + kOffAbort);
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const uint32_t rank = cluster_rank();       // 0: leader (issues the MMAs), 1: peer
-    const int n0 = (blockIdx.x >> 1) * kBN;     // first output row of the pair tile
-    const int r0 = n0 + (int)rank * kRows;      // first row decoded by this CTA
-    const int t0 = blockIdx.y * kPairTokens;    // first token of the pair tile
+    // rank = role in the pair (0: leader, issues the MMAs; 1: peer). When sharing, a cluster
+    // of four CTAs = two CTA pairs with the same 256 weight rows and different 512-token
+    // tiles; pair = which token tile. The CTA with the same rank in the other pair is the
+    // partner: both need the same 128 weight rows, and each decodes half of them.
+    constexpr int kClusterLog = SHARE ? 2 : 1;
+    constexpr int DR = SHARE ? kHalfRows : kRows;   // rows decoded by one CTA
+    const uint32_t rank4 = cluster_rank();
+    const uint32_t rank = rank4 & 1u, pair = SHARE ? rank4 >> 1 : 0u;
+    const uint32_t partner = ((pair ^ 1u) << 1) | rank;
+    const int n0 = (blockIdx.x >> kClusterLog) * kBN;   // first output row of the pair tile
+    const int r0 = n0 + (int)rank * kRows;      // first row of this CTA's weight operand
+    const int rd0 = r0 + (int)pair * DR;        // first row decoded by this CTA
+    const int t0 = (blockIdx.y * (SHARE ? 2 : 1) + (int)pair) * kPairTokens;   // first token
     const int nk = (in + kBK - 1) / kBK;        // K steps
     const int nsl = (nk + 3) / 4;               // 256-input slices
-    const int rows_valid = max(0, min(kRows, rows_pad - r0));   // packed rows present (x32)
+    const int rows_valid = max(0, min(DR, rows_pad - rd0));   // packed rows present
     // Pairs that run at the same time share their token tile; if they all walked K in the same
     // order they would request the same activation lines from L2 at the same moment. Each
     // pair therefore starts at its own 256-input slice and wraps around (only the fp32
     // accumulation order differs). Every role walks the slices in this order; `it` counts
     // stages in processing order and drives the ring.
-    const int rot = (blockIdx.x >> 1) % nsl;
+    const int rot = (blockIdx.x >> kClusterLog) % nsl;   // the same in both pairs of a cluster
 
     // Same answer in both CTAs of the pair (identical layouts), so both leave before any
     // cluster-wide step.
@@ -328,9 +359,12 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
             mbar_init(&empty_a[s], 1);            // the leader's multicast commit
         }
         for (int s = 0; s < kStagesB; ++s) {
-            mbar_init(&full_b[s], kDecWarps);     // (peer) one arrival per decoder warp
-            mbar_init(&empty_b[s], 1);            // the leader's multicast commit
-            mbar_init(&ready[s], kDecWarps + 2);  // (leader) decoders + two relays
+            // (peer) the copier with the partner's bytes, or the decoder warps
+            mbar_init(&full_b[s], SHARE ? 1 : kDecWarps);
+            mbar_init(&empty_b[s], SHARE ? 2 : 1);   // commits of the pairs writing the stage
+            // (leader) the copier or the decoder warps, plus the two relays
+            mbar_init(&ready[s], SHARE ? 3 : kDecWarps + 2);
+            mbar_init(&dec_done[s], kDecWarps);   // (SHARE) one arrival per decoder warp
         }
         for (int c = 0; c < 2; ++c) {
             mbar_init(&codes_full[c], 1);
@@ -347,7 +381,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
     }
     tc_fence_before();
-    cluster_sync();    // barriers of both CTAs initialised before any cross-CTA arrival
+    cluster_sync();    // barriers of every CTA initialised before any cross-CTA arrival
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     pdl_wait();
@@ -366,8 +400,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
                 mbar_arrive_expect_tx(&codes_full[cb], (uint32_t)(m * rows_valid * 32));
                 if (rows_valid > 0)
                     for (int k = 0; k < m; ++k)
-                        bulk_g2s(smem + kOffCodes + cb * kCodeBuf + k * (kRows * 32),
-                                 planes + (size_t)k * plane_bytes + ((size_t)sl * rows_pad + r0) * 32,
+                        bulk_g2s(smem + kOffCodes + cb * kCodeBuf + k * (DR * 32),
+                                 planes + (size_t)k * plane_bytes + ((size_t)sl * rows_pad + rd0) * 32,
                                  (uint32_t)(rows_valid * 32), &codes_full[cb]);
                 ++issued_c;
                 const int nj = min(4, nk - sl * 4);
@@ -415,13 +449,15 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
                     for (int kk = 0; kk < kBK / 16; ++kk)
                         umma_f16_pair(tmem + i * kBN, umma_desc_sw128(a0 + i * kABlock + kk * 32),
                                       umma_desc_sw128(b0 + kk * 32), idesc, (it > 0 || kk > 0) ? 1u : 0u);
-                umma_commit_pair(&empty_a[sa]);
-                umma_commit_pair(&empty_b[sb]);
+                // The activation stage belongs to this pair; when sharing, the weight stage is
+                // also written by the partners, so its release goes to all four CTAs.
+                umma_commit_pair(&empty_a[sa], (uint16_t)(0x3u << (2 * pair)));
+                umma_commit_pair(&empty_b[sb], (uint16_t)(SHARE ? 0xF : 0x3));
             }
-            umma_commit_pair(acc_full);
+            umma_commit_pair(acc_full, (uint16_t)(0x3u << (2 * pair)));
         } else if (lane == 0) {
             // ---------------- relay (peer): this CTA's half of a stage is ready
-            const uint32_t leader_ready = map_to_rank(smem_u32(ready), 0);
+            const uint32_t leader_ready = map_to_rank(smem_u32(ready), pair << 1);
             for (int it = 0; it < nk; ++it) {
                 const int sa = it % kStagesA, sb = it % kStagesB;
                 if (!wait_or_abort(&full_a[sa], (it / kStagesA) & 1, &s_abort, status)) break;
@@ -443,12 +479,35 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
                 mbar_arrive(&ready[sb]);
             }
         }
+    } else if (warp == 3) {
+        if (SHARE && lane == 0) {
+            // ---------------- copier: once this CTA's decoders have written their half of a
+            // weight stage, copy it into the partner's stage (same offset) with a bulk copy
+            // that completes on the partner's stage barrier, and count this CTA's half on its
+            // own stage barrier together with the partner's incoming bytes. The copy's
+            // source is free again once both pairs released the stage, which needs the copy
+            // to have landed.
+            uint64_t* stage_bar = rank == 0 ? ready : full_b;
+            const uint32_t peer_bar = map_to_rank(smem_u32(stage_bar), partner);
+            const uint32_t half0 = smem_u32(smem + kOffB) + pair * kHalfBytes;
+            const uint32_t peer_half0 = map_to_rank(half0, partner);
+            for (int it = 0; it < nk; ++it) {
+                const int sb = it % kStagesB;
+                if (!wait_or_abort(&dec_done[sb], (it / kStagesB) & 1, &s_abort, status)) break;
+                bulk_to_peer(peer_half0 + sb * kBStage, half0 + sb * kBStage, kHalfBytes,
+                             peer_bar + sb * 8);
+                mbar_arrive_expect_tx(&stage_bar[sb], kHalfBytes);
+            }
+        }
     } else if (warp >= kDecWarp0) {
         // ---------------- decoders, then epilogue
         const int dt = tid - kDecWarp0 * 32;        // 0..255
-        const int n = dt & (kRows - 1);             // row of this CTA's half owned by the thread
-        const int cs = dt >> 7;                     // groups 4cs..4cs+3 of every stage
-        const int row = r0 + n;
+        constexpr int GPT = SHARE ? 2 : 4;          // groups per thread and stage
+        const int n = dt & (DR - 1);                // decoded row owned by the thread
+        const int cs = dt / DR;                     // groups GPT*cs .. GPT*cs + GPT-1 of a stage
+        const int c0 = cs * GPT;
+        const int row = rd0 + n;
+        const int nn = (int)pair * DR + n;          // its row in the weight operand tile
         for (int i = dt; i < m * 256; i += kDecWarps * 32)
             books_s[i] = __ldg((const uint4*)books + i);
         for (int i = dt; i < kBN; i += kDecWarps * 32)
@@ -459,20 +518,21 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
         const int rw = r >> 2, rb = (r & 3) * 8;
         const bool row_ok = row < out;
         const uint32_t books_u = smem_u32(books_s);
-        const uint32_t b_tile = smem_u32(smem + kOffB) + (n >> 3) * 1024 + (n & 7) * 128;
+        const uint32_t b_tile = smem_u32(smem + kOffB) + (nn >> 3) * 1024 + (nn & 7) * 128;
         int it = 0;                                 // stages decoded so far (ring position)
         for (int js = 0; js < nsl; ++js) {
             const int sl = rot + js < nsl ? rot + js : rot + js - nsl;
             const int cb = js & 1;
-            // q[k][j]: the codes (one byte each) of groups 8j + 4cs .. 8j + 4cs + 3 of the
-            // slice in plane k; the front entry always belongs to the next stage.
+            // q[k][j]: the word holding the codes (one byte each) of the thread's groups
+            // 8j + c0 .. 8j + c0 + GPT-1 of the slice in plane k (from byte c0 & 3); the
+            // front entry always belongs to the next stage.
             uint32_t q[MB][4];
             const bool have = wait_or_abort(&codes_full[cb], (js >> 1) & 1, &s_abort, status);
 #pragma unroll
             for (int k = 0; k < MB; ++k) {
                 uint32_t w[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
                 if (have && n < rows_valid) {
-                    const uint32_t src = smem_u32(smem + kOffCodes + cb * kCodeBuf + k * (kRows * 32) + n * 32);
+                    const uint32_t src = smem_u32(smem + kOffCodes + cb * kCodeBuf + k * (DR * 32) + n * 32);
                     const uint4 lo = lds128_ordered(src), hi = lds128_ordered(src + 16);
                     w[0] = lo.x; w[1] = lo.y; w[2] = lo.z; w[3] = lo.w;
                     w[4] = hi.x; w[5] = hi.y; w[6] = hi.z; w[7] = hi.w;
@@ -490,9 +550,9 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
 #pragma unroll
                 for (int i = 0; i < 8; ++i) t[i] = (rw & 4) ? v[(i + 4) & 7] : v[i];
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {           // output word 2j + cs
-                    const uint32_t cur = cs ? t[2 * j + 1] : t[2 * j];
-                    const uint32_t prev = cs ? t[2 * j] : t[(2 * j + 7) & 7];
+                for (int j = 0; j < 4; ++j) {           // output word 2j + (c0 >> 2)
+                    const uint32_t cur = (c0 >> 2) ? t[2 * j + 1] : t[2 * j];
+                    const uint32_t prev = (c0 >> 2) ? t[2 * j] : t[(2 * j + 7) & 7];
                     q[k][j] = rb ? __funnelshift_l(prev, cur, rb) : cur;
                 }
             }
@@ -505,19 +565,19 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
                 const int st = it % kStagesB;
                 if (it >= kStagesB) wait_or_abort(&empty_b[st], ((it / kStagesB) - 1) & 1, &s_abort, status);
                 const uint32_t bt = b_tile + st * kBStage;
-                const int g0 = sl * 32 + j * 8 + cs * 4;     // first group of the thread's four
+                const int g0 = sl * 32 + j * 8 + c0;         // first group of the thread's GPT
 #pragma unroll
-                for (int cc = 0; cc < 4; ++cc) {
+                for (int cc = 0; cc < GPT; ++cc) {
                     uint32_t code[MB];
 #pragma unroll
-                    for (int k = 0; k < MB; ++k) code[k] = (q[k][0] >> (cc * 8)) & 0xffu;
+                    for (int k = 0; k < MB; ++k) code[k] = (q[k][0] >> (((c0 & 3) + cc) * 8)) & 0xffu;
                     uint4 o = decode_group<BDT, MB>(books_u, code);
                     if (!(row_ok && g0 + cc < ng)) o = make_uint4(0u, 0u, 0u, 0u);
-                    sts128(bt + (((cs * 4 + cc) ^ (n & 7)) << 4), o);
+                    sts128(bt + (((c0 + cc) ^ (nn & 7)) << 4), o);
                 }
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncwarp();
-                if (lane == 0) mbar_arrive(rank == 0 ? &ready[st] : &full_b[st]);
+                if (lane == 0) mbar_arrive(SHARE ? &dec_done[st] : rank == 0 ? &ready[st] : &full_b[st]);
                 ++it;
 #pragma unroll
                 for (int k = 0; k < MB; ++k) {
@@ -656,8 +716,9 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
 
     void (*kern)(const CUtensorMap, const uint8_t*, const uint16_t*, const uint16_t*, void*, int,
                  int, unsigned int*, int, int, int, int, int, size_t) =
-        m == 1 ? gemm_kernel<BDT, 1> : m == 2 ? gemm_kernel<BDT, 2> : m == 3 ? gemm_kernel<BDT, 3>
-                                                                      : gemm_kernel<BDT, 4>;
+        m == 1 ? gemm_kernel<BDT, 1, false> : m == 2 ? gemm_kernel<BDT, 2, true>
+        : m == 3 ? gemm_kernel<BDT, 3, true>  : gemm_kernel<BDT, 4, true>;
+    const int csize = m == 1 ? 2 : 4;   // CTAs per cluster: one pair, or two sharing the decode
     static std::mutex mu;
     static bool attr_done[kGemmMaxM][64] = {};
     int dev = 0;
@@ -676,16 +737,21 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
         }
     }
     cudaLaunchConfig_t cfg = {};
-    // x: CTA pairs along the rows (cluster dimension 2), y: 512-token tiles
-    cfg.gridDim = dim3(2 * ((d.out + kBN - 1) / kBN), (tokens + kPairTokens - 1) / kPairTokens);
+    // x: one cluster per 256-row tile, y: one token tile per pair of the cluster
+    const int tok_tile = (csize / 2) * kPairTokens;
+    cfg.gridDim = dim3(csize * ((d.out + kBN - 1) / kBN), (tokens + tok_tile - 1) / tok_tile);
     cfg.blockDim = dim3(kGemmThreads);
     cfg.dynamicSmemBytes = kGemmSmem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = (unsigned)csize;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     return cuda_ok(cudaLaunchKernelEx(&cfg, kern, map, (const uint8_t*)planes,
                                       (const uint16_t*)books, (const uint16_t*)scales, y, y_dt,
                                       d.scale_dt, (unsigned int*)ws, tokens, d.out, d.in, d.ng,
