@@ -119,15 +119,17 @@ aq_status aq_decode(const aq_layout* layout, int m, const void* planes, const vo
  *   x         : device, [batch][d_in] of x_dtype (AQ_F16 or AQ_BF16), row-major
  *   y         : device, [batch][d_out] of y_dtype (AQ_F16, AQ_BF16 or AQ_F32), row-major
  *   workspace : device scratch of at least aq_gemv_workspace_bytes(layout, batch) bytes:
- *               a status word and fp32 partial sums (one per 256-input slice, token and
- *               row). Zero-fill it once before its
- *               first use (aq_workspace_init); every call leaves it ready for the next one.
+ *               a status word and fp32 partial sums for every row: one per 256-input
+ *               slice and token, or, at batch 1 with 2^8-entry books, one per slice and
+ *               codebook of the largest prefix (up to 8) served that way. Zero-fill it once
+ *               before its first use (aq_workspace_init); every call leaves it ready for the
+ *               next one.
  *               Calls that may overlap on the GPU must not share a workspace.
  * Two kernels are enqueued, both with programmatic dependent launch: the product (fp32
- * partial sums per 256-input slice into the workspace) and a split-K reduction that sums
- * each row's partials, scales it and writes y. Each waits for the preceding grid before
- * reading memory. The slices of each row are summed in a fixed order, so the result does
- * not depend on scheduling.
+ * partial sums per 256-input slice, and per codebook at batch 1 with 2^8-entry books, into
+ * the workspace) and a split-K reduction that sums each row's partials, scales it and
+ * writes y. Each waits for the preceding grid before reading memory. The partials of each
+ * row are summed in a fixed order, so the result does not depend on scheduling.
  * Accuracy: |y - y_exact| <= 1e-2*(1+|y_exact|) per element and relative Frobenius error
  * <= 2e-3, with y_exact the fp64 product of the exactly widened stored values. */
 size_t aq_gemv_workspace_bytes(const aq_layout* layout, int batch);

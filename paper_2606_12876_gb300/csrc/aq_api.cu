@@ -99,7 +99,12 @@ size_t gemm_ws_bytes(const Dims& d, int tokens) {
 }
 
 size_t gemv_ws_bytes(const Dims& d, int batch) {
-    return aq::ws_partial_offset(d) + (size_t)d.S * (size_t)batch * (size_t)d.rows_pad * 4;
+    // Partial planes: S per token, or S per book of the largest prefix the table-lookup
+    // kernel serves at batch 1.
+    size_t planes = (size_t)d.S * (size_t)batch;
+    const int mt = d.M < aq::kLutMaxM ? d.M : aq::kLutMaxM;
+    if (aq::uses_lut(d, mt, batch) && (size_t)d.S * mt > planes) planes = (size_t)d.S * mt;
+    return aq::ws_partial_offset(d) + planes * (size_t)d.rows_pad * 4;
 }
 
 }  // namespace

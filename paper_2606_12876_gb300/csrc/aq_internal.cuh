@@ -40,6 +40,11 @@ constexpr size_t kWsStatusBytes = 256;
 inline size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 inline size_t ws_partial_offset(const Dims&) { return kWsStatusBytes; }
 
+// The batch-1 table-lookup GEMV (2^8-entry books, prefixes up to kLutMaxM) writes one partial
+// plane per (slice, book); every other GEMV one per (slice, token).
+constexpr int kLutMaxM = 8;
+inline bool uses_lut(const Dims& d, int m, int batch) { return d.B == 8 && batch == 1 && m <= kLutMaxM; }
+
 // Records a failed CUDA call (thread-local text for aq_last_error) and returns AQ_ERR_CUDA.
 aq_status cuda_fail(cudaError_t e, const char* what);
 // AQ_OK if e is cudaSuccess, else cuda_fail(e, what).
@@ -77,14 +82,27 @@ __device__ __forceinline__ uint16_t f32_to_bits(float v) {
 }
 
 // Eight packed 16-bit values (one uint4) -> eight floats.
+// Both halves of a packed pair of 16-bit floats, widened exactly to fp32 (low half first).
+// bf16 is the top half of an fp32, so widening is a shift. fp16 is widened by the mixed-type
+// add of sm_100 and later (fp16 operand, fp32 operand and result) with -0.0, which returns
+// the fp16 value exactly and runs on the fp32 pipe, unlike the conversion instruction.
+template <int DT>
+__device__ __forceinline__ void widen2(uint32_t w, float& lo, float& hi) {
+    if constexpr (DT == AQ_F16) {
+        asm("{.reg .b16 l, h;\n\tmov.b32 {l, h}, %2;\n\t"
+            "add.rn.f32.f16 %0, l, 0f80000000;\n\tadd.rn.f32.f16 %1, h, 0f80000000;}"
+            : "=f"(lo), "=f"(hi) : "r"(w));
+    } else {
+        lo = __uint_as_float(w << 16);
+        hi = __uint_as_float(w & 0xffff0000u);
+    }
+}
+
 template <int DT>
 __device__ __forceinline__ void unpack8(const uint4& v, float* f) {
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        f[2 * i] = bits_to_f32<DT>((uint16_t)(w[i] & 0xffffu));
-        f[2 * i + 1] = bits_to_f32<DT>((uint16_t)(w[i] >> 16));
-    }
+    for (int i = 0; i < 4; ++i) widen2<DT>(w[i], f[2 * i], f[2 * i + 1]);
 }
 
 // 16-byte streaming load of data read exactly once (codes): no L1 allocation.

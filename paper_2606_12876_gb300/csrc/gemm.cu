@@ -247,10 +247,10 @@ __device__ __forceinline__ float2 add2(float2 a, float2 b) {
 
 // One 32-bit word of a codeword (two 16-bit values, low half first) -> two floats.
 template <int BDT>
-__device__ __forceinline__ float2 widen2(uint32_t w) {
-    if constexpr (BDT == AQ_BF16) return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
-    else return make_float2(__half2float(__ushort_as_half((unsigned short)(w & 0xffffu))),
-                            __half2float(__ushort_as_half((unsigned short)(w >> 16))));
+__device__ __forceinline__ float2 widen2f(uint32_t w) {
+    float2 r;
+    widen2<BDT>(w, r.x, r.y);
+    return r;
 }
 
 __device__ __forceinline__ uint32_t f16x2(float2 v) {   // {lo, hi} -> packed fp16 pair, RN
@@ -267,15 +267,15 @@ __device__ __forceinline__ uint4 decode_group(uint32_t books, const uint32_t (&c
     if constexpr (MB == 1 && BDT == AQ_F16) {
         return c0;   // one fp16 codeword: widening to fp32 and rounding back is exact
     } else {
-        float2 a0 = widen2<BDT>(c0.x), a1 = widen2<BDT>(c0.y), a2 = widen2<BDT>(c0.z),
-               a3 = widen2<BDT>(c0.w);
+        float2 a0 = widen2f<BDT>(c0.x), a1 = widen2f<BDT>(c0.y), a2 = widen2f<BDT>(c0.z),
+               a3 = widen2f<BDT>(c0.w);
 #pragma unroll
         for (int k = 1; k < MB; ++k) {
             const uint4 ck = lds128(books + ((uint32_t)k << 12) + (code[k] << 4));
-            a0 = add2(a0, widen2<BDT>(ck.x));
-            a1 = add2(a1, widen2<BDT>(ck.y));
-            a2 = add2(a2, widen2<BDT>(ck.z));
-            a3 = add2(a3, widen2<BDT>(ck.w));
+            a0 = add2(a0, widen2f<BDT>(ck.x));
+            a1 = add2(a1, widen2f<BDT>(ck.y));
+            a2 = add2(a2, widen2f<BDT>(ck.z));
+            a3 = add2(a3, widen2f<BDT>(ck.w));
         }
         return make_uint4(f16x2(a0), f16x2(a1), f16x2(a2), f16x2(a3));
     }

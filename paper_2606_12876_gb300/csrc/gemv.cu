@@ -2,29 +2,31 @@
 // (Sec. 3.2 group sums, restricted to the first m codebooks as in Sec. 5; Y = W X of Sec. 2.2).
 //
 // Work split (split-K): the input dimension is cut into slices of 32 groups (256 inputs).
-// A work item is (slice, 32-row block). Each item reads the first m code planes of its rows
-// once and writes one fp32 partial per (row, token). A second, small kernel (splitk_reduce,
-// launched right behind with programmatic dependent launch, so its CTAs are already resident
-// when the product finishes) sums each row's partials in slice order (deterministic), scales
-// the row and stores y, with the rows spread evenly over the GPU.
+// A work item is (slice, 32-row block) for the direct kernel and (slice, codebook, 32-row
+// block) for the table-lookup kernel. Each item reads its code planes once and writes one
+// fp32 partial per (row, token). A second, small kernel (splitk_reduce, launched right behind
+// with programmatic dependent launch, so its CTAs are already resident when the product
+// finishes) sums each row's partials in a fixed order (deterministic), scales the row and
+// stores y, with the rows spread evenly over the GPU.
 //
 // Two product kernels:
-//  * gemv_lut (B = 8, one token, m <= 4). By linearity, x_g . (sum_k C_k[b_k]) =
+//  * gemv_lut (B = 8, one token, m <= 8). By linearity, x_g . (sum_k C_k[b_k]) =
 //    sum_k T_k[g][b_k] with T_k[g][j] = x_g . C_k[j]. A persistent CTA (one per SM) walks a
-//    contiguous range of work items; for each slice it builds T for the 32 groups and m books
-//    in shared memory (32 KiB per book), then every code byte costs one shared-memory lookup
+//    contiguous range of work items; for each (slice, book) it builds that book's T for the
+//    32 groups in shared memory (32 KiB), then every code byte costs one shared-memory lookup
 //    and one fp32 add. Lane L owns row 32*rb+L; because each row's 32 codes are stored
 //    rotated by the row index, at step p all 32 lanes look up 32 different groups, i.e. 32
 //    different banks, so the lookups are conflict-free and no cross-lane reduction is needed.
 //    One producer warp streams the code planes into a shared-memory ring with TMA bulk copies
 //    (the CTA's rows of a slice are contiguous in every plane), overlapping HBM reads with
-//    the table build and the lookups of the eight consumer warps.
+//    the table build and the lookups of the sixteen consumer warps.
 //  * gemv_direct (any B, 1..16 tokens). Decode each group in fp32 (sum of m codewords), then
 //    multiply by the tokens' 8 activations. Lane L owns row 32*rb+L and walks the 32 groups
 //    of the slice in a common order, so the activation loads are warp-uniform broadcasts.
 #include <map>
 #include <mutex>
 #include <tuple>
+#include <type_traits>
 
 #include "aq_internal.cuh"
 
@@ -33,67 +35,81 @@ namespace {
 
 // ------------------------------------------------------------------ LUT kernel (B = 8, b = 1)
 
-constexpr int kCons = 16;                         // consumer warps (one 32-row block each per stage)
+constexpr int kCons = 16;                         // consumer warps (two 32-row blocks each per stage)
 constexpr int kLutThreads = (kCons + 1) * 32;     // + one producer warp
-constexpr int kStageRb = 16;                      // 32-row blocks per stage: a 16 KiB plane copy
+constexpr int kStageRb = 2 * kCons;               // 32-row blocks per stage: a 32 KiB plane copy
 constexpr int kSlot = kStageRb * 1024;            // one ring slot = one plane of one stage
-constexpr int kSlots = 8;                         // largest ring depth (128 KiB)
+constexpr int kSlots = 4;                         // largest ring depth (128 KiB)
 constexpr int kXSlices = 8;                       // activation slices staged up front
-constexpr int kTBytes = 65536;                    // table of one book pair
-constexpr int kLutMaxM = 8;
+constexpr int kTBytes = 65536;                    // two single-book tables, interleaved
 
-// Shared memory: [T 64 KiB][codebooks m x 4 KiB][activations 8 x 512 B][ring][barriers]
+// Shared memory: [T 64 KiB][codebooks m x 4 KiB][activations 8 x 1 KiB fp32][ring][barriers]
 inline size_t lut_smem_bytes(int m, int slots) {
-    return (size_t)kTBytes + (size_t)m * 4096 + kXSlices * 512 + (size_t)slots * kSlot +
+    return (size_t)kTBytes + (size_t)m * 4096 + kXSlices * 1024 + (size_t)slots * kSlot +
            2 * kSlots * 8;
 }
 
-// The m books are processed in passes of at most two (pass p: books 2p, 2p+1), so the table
-// never exceeds 64 KiB: T[j][k%2][32 groups] (fp32), entry (k, j, g) at byte
-// j*256 + (k%2)*128 + g*4; j*256 + g*4 is produced from a code byte by one prmt.
+// Work is split by slice and by codebook: by linearity in the books (the successive-refinement
+// form of Sec. 5, y_m = sum over k < m of x . (s o C_k[b_k])^T), the product over slice s and
+// book k is a separate term. A unit is such a (slice s, book k) pair, numbered u = s*m + k;
+// an item is (unit, 32-row block), numbered u*RBc + rb. Each item writes one fp32 partial per
+// row into plane u of the partial sums, and the reduction adds the m*S planes of a row. So a
+// CTA builds the table of one book for every unit it touches (one or two units in general),
+// and looks it up for all of that unit's rows it owns, instead of building m tables for a
+// third as many rows.
 //
-// A CTA owns the items [i0, i1) (item = slice * RBc + 32-row block). In every pass it walks
-// them in stages of up to 16 items that never cross a slice. For each stage and each book of
-// the pass the producer warp copies the stage's rows of that book's plane into one ring slot
-// with a TMA bulk copy (16 KiB; the CTA's rows of a slice are contiguous in every plane), and
-// consumer warp w looks up item w of the stage. A row's sum over the pass's books stays in a
-// register; pass 0 stores it as the fp32 partial and later passes add to it. The codebooks
-// and the activations of the CTA's first slices are requested before any code.
-template <int BDT, int XDT, int SDT>
+// Table of a unit: T[j][h][32 groups] (fp32), entry (j, g) of the unit's book at byte
+// j*256 + h*128 + g*4, h alternating between the CTA's consecutive units, so a unit's table is
+// built while the other half still serves the previous unit; j*256 + g*4 is produced from a
+// code byte by one prmt.
+//
+// A CTA owns the items [i0, i1) and walks them in stages of up to 32 items that never cross a
+// unit. For each stage the producer warp copies the stage's rows of the unit's book plane into
+// one ring slot with a TMA bulk copy (32 KiB; the CTA's rows of a slice are contiguous in
+// every plane), and consumer warp w looks up items w and w + 16 of the stage, so each wait on
+// the ring serves two row blocks. The codebooks and the activations of the CTA's first slices
+// are requested before any code.
+template <int BDT, int XDT>
 __global__ void __launch_bounds__(kLutThreads, 1)
 gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
-                const uint16_t* __restrict__ x, float* __restrict__ partials, unsigned int* __restrict__ status, int m, int in,
-                int ng, int rows_pad, int RBc, int S, int total_items, size_t plane_bytes,
-                int nslots, int cps, int static_weights) {
+                const uint16_t* __restrict__ x, float* __restrict__ partials,
+                unsigned int* __restrict__ status, int m, int in, int ng, int rows_pad, int RBc,
+                size_t plane_bytes, int nslots, int cpu, int q, int r, int static_weights) {
     extern __shared__ __align__(128) unsigned char smem[];
     unsigned char* T = smem;
     uint4* Cb = (uint4*)(smem + kTBytes);                          // [m][256] codewords
-    unsigned char* xs = smem + kTBytes + (size_t)m * 4096;         // [kXSlices][256] activations
-    unsigned char* ring = xs + kXSlices * 512;                     // nslots x 16 KiB
+    // [kXSlices][256] activations in fp32; group g of a slice at 128-byte line g/4, its two
+    // 16-byte halves at quads (2*(g%4) + half) ^ (g/4 mod 8), so the table build's reads
+    // (eight lanes at eight different lines) hit eight different bank quads.
+    unsigned char* xs = smem + kTBytes + (size_t)m * 4096;
+    unsigned char* ring = xs + kXSlices * 1024;                    // nslots x 32 KiB
     uint64_t* full = (uint64_t*)(ring + (size_t)nslots * kSlot);
     uint64_t* empty = full + kSlots;
     __shared__ volatile int s_abort;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    // Item range of this CTA: slice-aligned (cps CTAs per slice) or balanced over the grid.
+    // Item range of this CTA: a share of one unit (cpu CTAs per unit: RBc = q*cpu + r) or a
+    // share of all items (total = q*gridDim.x + r); the first r shares are one item longer.
     // Item indices fit in 32 bits (checked by the host); the per-stage bookkeeping below is
     // incremental, without divisions (an integer division is a long instruction sequence).
     int i0, i1;
-    if (cps > 0) {
-        const int s = blockIdx.x / cps, c = blockIdx.x % cps;
-        i0 = s * RBc + c * RBc / cps;
-        i1 = s * RBc + (c + 1) * RBc / cps;
-    } else {
-        i0 = (int)((long long)blockIdx.x * total_items / gridDim.x);
-        i1 = (int)((long long)(blockIdx.x + 1) * total_items / gridDim.x);
+    {
+        int b = blockIdx.x, base = 0;
+        if (cpu > 0) {
+            const int u = b / cpu;
+            b -= u * cpu;
+            base = u * RBc;
+        }
+        i0 = base + b * q + min(b, r);
+        i1 = i0 + q + (b < r ? 1 : 0);
     }
-    const int s_first = i0 / RBc, rb_first = i0 - s_first * RBc;
-    // A walk over the CTA's items in stages: up to kStageRb items, never crossing a slice.
+    const int u_first = i0 / RBc, s_first = u_first / m;
+    // A walk over the CTA's items in stages: up to kStageRb items, never crossing a unit.
     struct Walk {
-        int it, s, rb, n;
+        int it, s, k, rb, n;
     };
     auto walk_start = [&]() {
-        Walk w{i0, s_first, rb_first, 0};
+        Walk w{i0, s_first, u_first - s_first * m, i0 - u_first * RBc, 0};
         w.n = min(min(kStageRb, RBc - w.rb), i1 - w.it);
         return w;
     };
@@ -102,38 +118,30 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
         w.rb += w.n;
         if (w.rb == RBc) {
             w.rb = 0;
-            ++w.s;
+            if (++w.k == m) {
+                w.k = 0;
+                ++w.s;
+            }
         }
         w.n = min(min(kStageRb, RBc - w.rb), i1 - w.it);
     };
-    const int npass = (m + 1) / 2;
 
-    // Producer state (warp kCons, lane 0): the next copy is book 2*p_pass + p_k of stage p_w,
-    // into ring slot p_slot (use parity p_phase); p_q copies issued so far.
-    int p_q = 0, p_slot = 0, p_pass = 0, p_k = 0;
+    // Producer state (warp kCons, lane 0): the next copy is stage p_w into ring slot p_slot
+    // (use parity p_phase); p_q copies issued so far.
+    int p_q = 0, p_slot = 0;
     uint32_t p_phase = 0;
     Walk p_w = walk_start();
-    if (i0 >= i1) p_pass = npass;
     auto issue_next = [&]() {
-        const int mp = min(2, m - 2 * p_pass);
         const size_t src = ((size_t)p_w.s * rows_pad + (size_t)p_w.rb * 32) * 32;
         mbar_arrive_expect_tx(&full[p_slot], (uint32_t)(p_w.n * 1024));
-        bulk_g2s(ring + (size_t)p_slot * kSlot,
-                 planes + (size_t)(2 * p_pass + p_k) * plane_bytes + src,
+        bulk_g2s(ring + (size_t)p_slot * kSlot, planes + (size_t)p_w.k * plane_bytes + src,
                  (uint32_t)(p_w.n * 1024), &full[p_slot]);
         ++p_q;
         if (++p_slot == nslots) {
             p_slot = 0;
             p_phase ^= 1u;
         }
-        if (++p_k == mp) {
-            p_k = 0;
-            walk_next(p_w);
-            if (p_w.it >= i1) {
-                ++p_pass;
-                p_w = walk_start();
-            }
-        }
+        walk_next(p_w);
     };
     if (tid == 0) {
         for (int d = 0; d < nslots; ++d) {
@@ -144,9 +152,8 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
         s_abort = 0;
     }
     __syncthreads();            // barriers initialised before the first copy
-    // Codebooks and activations are requested first (into registers); the producer starts
-    // its copies only after every thread has issued these loads (the barrier below).
-    // (consumer threads only: they are the ones that store the codebooks below)
+    // Codebooks and activations are requested first (into registers) by the consumer threads,
+    // which store them below.
     uint4 cb_r[4];
     auto load_books = [&]() {
 #pragma unroll
@@ -158,12 +165,11 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
     };
     if (static_weights) {
         // The weights are read-only while calls run (AQ_LAYOUT_STATIC_WEIGHTS): request the
-        // codebooks before waiting for the preceding kernel.
+        // codebooks and fill the code ring before waiting for the preceding kernel, so they
+        // overlap its tail.
         load_books();
-        // The code planes are read-only too: fill the ring before waiting for the preceding
-        // kernel, so the first stages overlap its tail.
         if (warp == kCons && lane == 0)
-            while (p_q < nslots && p_pass < npass) issue_next();
+            while (p_q < nslots && p_w.it < i1) issue_next();
     }
     pdl_wait();                 // inputs may come from the preceding kernel in the stream
     pdl_launch_dependents();    // the split-K reduction may become resident (it waits for us)
@@ -173,15 +179,11 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
         const int col = (s_first + (tid >> 6)) * 256 + (tid & 63) * 4;
         if (col < in) x_r = __ldg((const uint2*)(x + col));
     }
-    __syncthreads();
-
-    // Stage sequence shared by the producer and the consumers: pass, then the walk's stages;
-    // one ring slot per (stage, book of the pass).
 
     if (warp == kCons) {
         // ---- producer (lane 0 issues; the warp stays converged for the final barriers)
         if (lane == 0) {
-            while (p_pass < npass) {
+            while (p_w.it < i1) {
                 if (s_abort) break;
                 if (p_q >= nslots && !mbar_wait(&empty[p_slot], p_phase ^ 1u)) {
                     record_status(status, AQ_ERR_TIMEOUT);
@@ -201,7 +203,13 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
             const int i = tid + r * kCons * 32;
             if (i < m * 256) Cb[i] = cb_r[r];
         }
-        if (tid < kXSlices * 64) *(uint2*)(xs + (tid >> 6) * 512 + (tid & 63) * 8) = x_r;
+        if (tid < kXSlices * 64) {
+            const int e = tid & 63, g = e >> 1;
+            float4 f;
+            widen2<XDT>(x_r.x, f.x, f.y);
+            widen2<XDT>(x_r.y, f.z, f.w);
+            *(float4*)(xs + (tid >> 6) * 1024 + (g >> 2) * 128 + ((((g & 3) * 2) + (e & 1)) ^ ((g >> 2) & 7)) * 16) = f;
+        }
         named_barrier(1, kCons * 32);   // staged codebooks and activations visible to all consumers
 
         // Each lane reads its row's 32 code bytes as two 16-byte halves; lanes 4-7 of every
@@ -219,96 +227,133 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
             goff[q] = v;
         }
 
+        // Table build: lane L = 8*ph + gq computes groups 4gq..4gq+3 for codewords
+        // j = 16*warp + ph + 4i; one 16-byte codeword read serves four entries, stored as one
+        // 16-byte piece. xv holds the four groups' activations of the current slice.
+        const int ph = lane >> 3, gq = lane & 7;
+        float2 xv[4][4];
         int slot = 0;
         uint32_t phase = 0;                     // parity of the slot's current use
-        for (int pass = 0; pass < npass; ++pass) {
-            const int mp = min(2, m - 2 * pass);
-            int cur_s = -1;
-            for (Walk w = walk_start(); w.it < i1; walk_next(w)) {
-                const int n = w.n, s = w.s, rb = w.rb;
+        int cur_s = -1, cur_k = -1, h = 1;
+        for (Walk w = walk_start(); w.it < i1; walk_next(w)) {
+            const int n = w.n, s = w.s, rb = w.rb;
+            if (s != cur_s || w.k != cur_k) {
                 if (s != cur_s) {
-                    // Table of the pass's books for slice s. Lane L = 8*ph + gq computes groups
-                    // 4gq..4gq+3 for codewords j = 16*warp + ph + 4i: one 16-byte codeword read
-                    // serves four entries, stored as one 16-byte piece.
-                    const int ph = lane >> 3, gq = lane & 7, sl = s - s_first;
-                    float2 xv[4][4];
+                    const int sl = s - s_first;
+                    if (sl < kXSlices) {
+                        const unsigned char* xb = xs + sl * 1024 + gq * 128;
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const int g = s * 32 + gq * 4 + u;
-                        uint4 xr = make_uint4(0u, 0u, 0u, 0u);
-                        if (sl < kXSlices) xr = *(const uint4*)(xs + sl * 512 + (gq * 4 + u) * 16);
-                        else if (g < ng) xr = __ldg((const uint4*)x + g);
-                        float f[8];
-                        unpack8<XDT>(xr, f);
+                        for (int u = 0; u < 4; ++u) {
+                            const float4 lo = *(const float4*)(xb + (((2 * u) ^ gq) & 7) * 16);
+                            const float4 hi = *(const float4*)(xb + (((2 * u + 1) ^ gq) & 7) * 16);
+                            xv[u][0] = make_float2(lo.x, lo.y);
+                            xv[u][1] = make_float2(lo.z, lo.w);
+                            xv[u][2] = make_float2(hi.x, hi.y);
+                            xv[u][3] = make_float2(hi.z, hi.w);
+                        }
+                    } else {
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) xv[u][e] = make_float2(f[2 * e], f[2 * e + 1]);
-                    }
-                    named_barrier(1, kCons * 32);   // old table no longer read; Cb / xs staged
-                    for (int k = 0; k < mp; ++k) {
-                        const int kb = 2 * pass + k;
-                        unsigned char* Tk = T + k * 128 + gq * 16;
-                        uint4 cw[4];
+                        for (int u = 0; u < 4; ++u) {
+                            const int g = s * 32 + gq * 4 + u;
+                            uint4 xr = make_uint4(0u, 0u, 0u, 0u);
+                            if (g < ng) xr = __ldg((const uint4*)x + g);
+                            float f[8];
+                            unpack8<XDT>(xr, f);
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) cw[i] = Cb[kb * 256 + warp * 16 + ph + 4 * i];
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            float c[8];
-                            unpack8<BDT>(cw[i], c);
-                            float r[4];
-#pragma unroll
-                            for (int u = 0; u < 4; ++u) {
-                                float2 t = make_float2(xv[u][0].x * c[0], xv[u][0].y * c[1]);
-                                t = ffma2(xv[u][1], make_float2(c[2], c[3]), t);
-                                t = ffma2(xv[u][2], make_float2(c[4], c[5]), t);
-                                t = ffma2(xv[u][3], make_float2(c[6], c[7]), t);
-                                r[u] = t.x + t.y;
-                            }
-                            *(float4*)(Tk + (warp * 16 + ph + 4 * i) * 256) =
-                                make_float4(r[0], r[1], r[2], r[3]);
+                            for (int e = 0; e < 4; ++e) xv[u][e] = make_float2(f[2 * e], f[2 * e + 1]);
                         }
                     }
-                    named_barrier(1, kCons * 32);
                     cur_s = s;
                 }
-                float part = 0.0f;
-                for (int k = 0; k < mp; ++k) {
-                    bool ok = !s_abort;
-                    if (ok && !mbar_wait(&full[slot], phase)) {
-                        record_status(status, AQ_ERR_TIMEOUT);
-                        s_abort = 1;
-                        ok = false;
+                cur_k = w.k;
+                h ^= 1;
+                // The other half served the previous unit; this half was last read two units
+                // ago, before every consumer passed the previous unit's barrier.
+                unsigned char* Th = T + h * 128 + gq * 16;
+                uint4 cw[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) cw[i] = Cb[cur_k * 256 + warp * 16 + ph + 4 * i];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    float c[8];
+                    unpack8<BDT>(cw[i], c);
+                    float r[4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        float2 t = make_float2(xv[u][0].x * c[0], xv[u][0].y * c[1]);
+                        t = ffma2(xv[u][1], make_float2(c[2], c[3]), t);
+                        t = ffma2(xv[u][2], make_float2(c[4], c[5]), t);
+                        t = ffma2(xv[u][3], make_float2(c[6], c[7]), t);
+                        r[u] = t.x + t.y;
                     }
-                    if (ok && warp < n) {
-                        const unsigned char* row = ring + (size_t)slot * kSlot + warp * 1024 + lane * 32;
-                        const uint4 a = *(const uint4*)(row + c0 * 16);
-                        const uint4 b = *(const uint4*)(row + (c0 ^ 1) * 16);
-                        const uint32_t wd[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-                        const uint32_t Tk = smem_u32(T) + k * 128;
-                        float2 acc = make_float2(0.0f, 0.0f);
+                    *(float4*)(Th + (warp * 16 + ph + 4 * i) * 256) = make_float4(r[0], r[1], r[2], r[3]);
+                }
+                named_barrier(1, kCons * 32);
+            }
+            float part0 = 0.0f, part1 = 0.0f;
+            bool ok = !s_abort;
+            if (ok && !mbar_wait(&full[slot], phase)) {
+                record_status(status, AQ_ERR_TIMEOUT);
+                s_abort = 1;
+                ok = false;
+            }
+            if (ok && warp < n) {
+                // Each lane reads its row's 32 code bytes of item warp (and warp + 16) as two
+                // 16-byte halves. The prmt forms the table offset of a code byte: byte0 = goff
+                // byte i, byte1 = code byte i, bytes 2-3 = sign of the goff byte (0). The
+                // table half is a constant of the load, so a lookup is prmt, load and add.
+                const unsigned char* row0 = ring + (size_t)slot * kSlot + warp * 1024 + lane * 32;
+                const uint4 a0 = *(const uint4*)(row0 + c0 * 16);
+                const uint4 b0 = *(const uint4*)(row0 + (c0 ^ 1) * 16);
+                const uint32_t w0[8] = {a0.x, a0.y, a0.z, a0.w, b0.x, b0.y, b0.z, b0.w};
+                const bool two = warp + kCons < n;
+                uint32_t w1[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+                if (two) {
+                    const unsigned char* row1 = row0 + kCons * 1024;
+                    const uint4 a1 = *(const uint4*)(row1 + c0 * 16);
+                    const uint4 b1 = *(const uint4*)(row1 + (c0 ^ 1) * 16);
+                    w1[0] = a1.x; w1[1] = a1.y; w1[2] = a1.z; w1[3] = a1.w;
+                    w1[4] = b1.x; w1[5] = b1.y; w1[6] = b1.z; w1[7] = b1.w;
+                }
+                auto look = [&](auto half) {
+                    const unsigned char* Tb = T + decltype(half)::value;
+                    auto ld = [&](uint32_t wq, uint32_t g, uint32_t sel) {
+                        return *(const float*)(Tb + prmt(wq, g, sel));
+                    };
+                    if (two) {
 #pragma unroll
                         for (int qq = 0; qq < 8; ++qq) {
-                            // byte0 = goff byte i, byte1 = code byte i, bytes 2-3 = sign of goff byte (0)
-                            const uint32_t w = wd[qq], g = goff[qq];
-                            const float v0 = lds_f32(Tk + prmt(w, g, 0xCC04u));
-                            const float v1 = lds_f32(Tk + prmt(w, g, 0xDD15u));
-                            const float v2 = lds_f32(Tk + prmt(w, g, 0xEE26u));
-                            const float v3 = lds_f32(Tk + prmt(w, g, 0xFF37u));
-                            acc = add2(acc, add2(make_float2(v0, v1), make_float2(v2, v3)));
+                            const uint32_t g = goff[qq];
+                            const float v0 = ld(w0[qq], g, 0xCC04u), u0 = ld(w1[qq], g, 0xCC04u);
+                            const float v1 = ld(w0[qq], g, 0xDD15u), u1 = ld(w1[qq], g, 0xDD15u);
+                            const float v2 = ld(w0[qq], g, 0xEE26u), u2 = ld(w1[qq], g, 0xEE26u);
+                            const float v3 = ld(w0[qq], g, 0xFF37u), u3 = ld(w1[qq], g, 0xFF37u);
+                            part0 += (v0 + v1) + (v2 + v3);
+                            part1 += (u0 + u1) + (u2 + u3);
                         }
-                        part += acc.x + acc.y;
+                    } else {
+#pragma unroll
+                        for (int qq = 0; qq < 8; ++qq) {
+                            const uint32_t g = goff[qq];
+                            const float v0 = ld(w0[qq], g, 0xCC04u), v1 = ld(w0[qq], g, 0xDD15u);
+                            const float v2 = ld(w0[qq], g, 0xEE26u), v3 = ld(w0[qq], g, 0xFF37u);
+                            part0 += (v0 + v1) + (v2 + v3);
+                        }
                     }
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&empty[slot]);
-                    if (++slot == nslots) {
-                        slot = 0;
-                        phase ^= 1u;
-                    }
-                }
-                if (!s_abort && warp < n) {
-                    float* dst = partials + (size_t)s * rows_pad + (size_t)(rb + warp) * 32 + lane;
-                    if (pass > 0) part += *dst;     // this thread wrote it in the previous pass
-                    *dst = part;
-                }
+                };
+                if (h) look(std::integral_constant<int, 128>());
+                else look(std::integral_constant<int, 0>());
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[slot]);
+            if (++slot == nslots) {
+                slot = 0;
+                phase ^= 1u;
+            }
+            if (ok && warp < n) {
+                float* dst = partials + ((size_t)s * m + cur_k) * rows_pad + (size_t)(rb + warp) * 32 + lane;
+                dst[0] = part0;
+                if (warp + kCons < n) dst[kCons * 32] = part1;
             }
         }
     }
@@ -403,34 +448,54 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
 
 // ------------------------------------------------------------------ split-K reduction
 
-// y[t][r] = s[r] * sum over the S slices of partials[s][t][r], in slice order (R1: the row
-// scale multiplies the codebook sum, so it factors out of the dot product). One thread per
-// (row, token); all of a thread's loads are issued before the additions.
+// y[t][r] = s[r] * sum over the P partial planes p of partials[p*batch + t][r] (R1: the row
+// scale multiplies the codebook sum, so it factors out of the dot product). A CTA of eight
+// warps takes 32 * 8 / wpr rows of one token; the wpr warps (1, 2, 4 or 8) of a 32-row group
+// split its planes: warp j of the group adds planes j, j + wpr, ... in order (up to sixteen
+// loads in flight, coalesced over the rows), then the group's first warp adds the wpr sums in
+// order, so the summation order is fixed. With static weights the row scales are read before
+// waiting for the product kernel. The kernel is kept small: it runs once per CTA, so its
+// instructions are fetched cold.
 template <int SDT>
 __global__ void __launch_bounds__(256)
 splitk_reduce_kernel(const float* __restrict__ partials, const uint16_t* __restrict__ scales,
-                     void* y, int y_dt, int out, int rows_pad, int S, int batch) {
+                     void* y, int y_dt, int out, int rows_pad, int P, int batch, int wpr,
+                     int static_weights) {
+    __shared__ float red[8][32];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int j = w & (wpr - 1), rg = w - j;     // rg: first warp of the row group
+    const int r = blockIdx.x * (256 / wpr) + (rg / wpr) * 32 + lane, t = blockIdx.y;
+    const bool lead = j == 0 && r < out;
+    uint16_t sc = 0;
+    if (static_weights && lead) sc = scales[r];
     pdl_wait();                 // the product kernel's partials
     pdl_launch_dependents();
-    const int r = blockIdx.x * blockDim.x + threadIdx.x, t = blockIdx.y;
-    if (r >= out) return;
-    const size_t stride = (size_t)batch * rows_pad;
-    const float* p = partials + (size_t)t * rows_pad + r;
+    if (!static_weights && lead) sc = scales[r];
     float sum = 0.0f;
-    int sl = 0;
-    for (; sl + 16 <= S; sl += 16) {
-        float v[16];
+    if (r < out) {
+        const size_t step = (size_t)wpr * batch * rows_pad;   // plane p to plane p + wpr
+        const float* p = partials + ((size_t)j * batch + t) * rows_pad + r;
+#pragma unroll 1
+        for (int q = j; q < P; q += 16 * wpr, p += 16 * step) {
+            float v[16];
 #pragma unroll
-        for (int q = 0; q < 16; ++q) v[q] = __ldcg(p + (size_t)(sl + q) * stride);
+            for (int i = 0; i < 16; ++i) v[i] = q + i * wpr < P ? __ldcg(p + i * step) : 0.0f;
 #pragma unroll
-        for (int q = 0; q < 16; ++q) sum += v[q];
+            for (int i = 0; i < 16; ++i) sum += v[i];
+        }
     }
-    for (; sl < S; ++sl) sum += __ldcg(p + (size_t)sl * stride);
-    const float v = sum * bits_to_f32<SDT>(scales[r]);
-    const size_t yi = (size_t)t * out + r;
-    if (y_dt == AQ_F32) ((float*)y)[yi] = v;
-    else if (y_dt == AQ_F16) ((uint16_t*)y)[yi] = f32_to_bits<AQ_F16>(v);
-    else ((uint16_t*)y)[yi] = f32_to_bits<AQ_BF16>(v);
+    if (wpr > 1) {
+        red[w][lane] = sum;
+        __syncthreads();
+        if (lead)
+            for (int i = 1; i < wpr; ++i) sum += red[w + i][lane];
+    }
+    if (lead) {
+        const float v = sum * bits_to_f32<SDT>(sc);
+        const size_t yi = (size_t)t * out + r;
+        if (y_dt == AQ_F32) ((float*)y)[yi] = v;
+        else ((uint16_t*)y)[yi] = y_dt == AQ_F16 ? f32_to_bits<AQ_F16>(v) : f32_to_bits<AQ_BF16>(v);
+    }
 }
 
 // ------------------------------------------------------------------ host side
@@ -506,11 +571,11 @@ struct GemvArgs {
     unsigned int* status;
 };
 
-template <int BDT, int XDT, int SDT>
+template <int BDT, int XDT>
 aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     DeviceInfo di;
     if (aq_status e = device_info(&di); e != AQ_OK) return e;
-    auto kern = gemv_lut_kernel<BDT, XDT, SDT>;
+    auto kern = gemv_lut_kernel<BDT, XDT>;
     // As many 16 KiB ring slots as fit next to the table, codebooks and activations (<= 8).
     const size_t fixed = lut_smem_bytes(m, 0) + 8192;   // + static shared memory and slack
     int nslots = di.smem_optin > (int)fixed ? (int)((di.smem_optin - fixed) / kSlot) : 0;
@@ -519,24 +584,28 @@ aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     const size_t smem = lut_smem_bytes(m, nslots);
     int occ = 0;
     if (aq_status e = prepare(kern, smem, kLutThreads, m, &occ); e != AQ_OK) return e;
-    const long long items = (long long)d.S * d.RBc;
+    const long long units = (long long)d.S * m;       // (slice, book) pairs
+    const long long items = units * d.RBc;
     if (items > 0x7fffffffLL) return AQ_ERR_UNSUPPORTED;   // item indices are 32-bit
-    // One CTA per SM. If whole slices per CTA keep at least 90% of the SMs busy, every CTA
-    // gets a single slice (one table build per book); otherwise items are balanced evenly
-    // and a CTA may span two slices.
-    int cps = di.sms / d.S;
-    if (cps > d.RBc) cps = d.RBc;
-    int grid;
-    if (cps >= 1 && (long long)cps * d.S * 10 >= (long long)di.sms * 9) {
-        grid = cps * d.S;
+    // One CTA per SM. If whole shares of units keep at least 90% of the SMs busy, every CTA
+    // gets part of a single unit (one table build); otherwise items are balanced evenly and a
+    // CTA may span two units.
+    long long cpu = di.sms / units;
+    if (cpu > d.RBc) cpu = d.RBc;
+    int grid, q, r;   // a CTA's share: q items, one more for the first r shares
+    if (cpu >= 1 && cpu * units * 10 >= (long long)di.sms * 9) {
+        grid = (int)(cpu * units);
+        q = d.RBc / (int)cpu;
+        r = d.RBc % (int)cpu;
     } else {
-        cps = 0;
+        cpu = 0;
         grid = (int)(items < di.sms ? items : di.sms);
+        q = (int)(items / grid);
+        r = (int)(items % grid);
     }
     return launch_pdl(kern, dim3(grid), dim3(kLutThreads), smem, st, (const uint8_t*)a.planes,
                       (const uint16_t*)a.books, (const uint16_t*)a.x, a.partials, a.status, m,
-                      d.in, d.ng,
-                      d.rows_pad, d.RBc, d.S, items, d.plane_bytes, nslots, cps,
+                      d.in, d.ng, d.rows_pad, d.RBc, d.plane_bytes, nslots, (int)cpu, q, r,
                       (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0);
 }
 
@@ -578,16 +647,12 @@ static aq_status launch_product(const Dims& d, int m, const void* planes, const 
     GemvArgs a{planes, books, scales, x, x_dt, batch, y, y_dt,
                (float*)((char*)ws + ws_partial_offset(d)), (unsigned int*)ws};
     const int bb = d.book_dt == AQ_BF16, xb = x_dt == AQ_BF16, sb = d.scale_dt == AQ_BF16;
-    if (d.B == 8 && batch == 1 && m <= kLutMaxM) {
-        switch (bb * 4 + xb * 2 + sb) {
-            case 0: return run_lut<AQ_F16, AQ_F16, AQ_F16>(d, m, a, st);
-            case 1: return run_lut<AQ_F16, AQ_F16, AQ_BF16>(d, m, a, st);
-            case 2: return run_lut<AQ_F16, AQ_BF16, AQ_F16>(d, m, a, st);
-            case 3: return run_lut<AQ_F16, AQ_BF16, AQ_BF16>(d, m, a, st);
-            case 4: return run_lut<AQ_BF16, AQ_F16, AQ_F16>(d, m, a, st);
-            case 5: return run_lut<AQ_BF16, AQ_F16, AQ_BF16>(d, m, a, st);
-            case 6: return run_lut<AQ_BF16, AQ_BF16, AQ_F16>(d, m, a, st);
-            default: return run_lut<AQ_BF16, AQ_BF16, AQ_BF16>(d, m, a, st);
+    if (uses_lut(d, m, batch)) {
+        switch (bb * 2 + xb) {
+            case 0: return run_lut<AQ_F16, AQ_F16>(d, m, a, st);
+            case 1: return run_lut<AQ_F16, AQ_BF16>(d, m, a, st);
+            case 2: return run_lut<AQ_BF16, AQ_F16>(d, m, a, st);
+            default: return run_lut<AQ_BF16, AQ_BF16>(d, m, a, st);
         }
     }
     switch ((d.B == 16) * 4 + bb * 2 + sb) {
@@ -602,11 +667,21 @@ static aq_status launch_product(const Dims& d, int m, const void* planes, const 
     }
 }
 
+// P partial planes per token: one per (slice, book) for the LUT kernel, one per slice for the
+// direct kernel.
 template <int SDT>
-static aq_status launch_reduce(const Dims& d, const GemvArgs& a, cudaStream_t st) {
-    return launch_pdl(splitk_reduce_kernel<SDT>, dim3((d.out + 255) / 256, a.batch), dim3(256),
-                      0, st, (const float*)a.partials, (const uint16_t*)a.scales, a.y, a.y_dt,
-                      d.out, d.rows_pad, d.S, a.batch);
+static aq_status launch_reduce(const Dims& d, int P, const GemvArgs& a, cudaStream_t st) {
+    int occ = 0;
+    if (aq_status e = prepare(splitk_reduce_kernel<SDT>, 0, 256, 0, &occ); e != AQ_OK) return e;
+    // Warps per 32-row group: one while a warp's sixteen loads cover the planes (no shared
+    // memory step, a small grid), else eight (measured: 1 at P = 16, 8 at P >= 32 are the
+    // fastest choices on the layer shapes of the benchmark).
+    const int wpr = P <= 16 ? 1 : 8;
+    const int rows_per_cta = 256 / wpr;
+    return launch_pdl(splitk_reduce_kernel<SDT>, dim3((d.out + rows_per_cta - 1) / rows_per_cta, a.batch),
+                      dim3(256), 0, st, (const float*)a.partials, (const uint16_t*)a.scales, a.y,
+                      a.y_dt, d.out, d.rows_pad, P, a.batch, wpr,
+                      (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0);
 }
 
 aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* books,
@@ -618,7 +693,9 @@ aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* book
         return e;
     GemvArgs a{planes, books, scales, x, x_dt, batch, y, y_dt,
                (float*)((char*)ws + ws_partial_offset(d)), (unsigned int*)ws};
-    return d.scale_dt == AQ_BF16 ? launch_reduce<AQ_BF16>(d, a, st) : launch_reduce<AQ_F16>(d, a, st);
+    const int P = uses_lut(d, m, batch) ? d.S * m : d.S;
+    return d.scale_dt == AQ_BF16 ? launch_reduce<AQ_BF16>(d, P, a, st)
+                                 : launch_reduce<AQ_F16>(d, P, a, st);
 }
 
 }  // namespace aq
