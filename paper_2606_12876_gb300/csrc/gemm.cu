@@ -295,8 +295,8 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
 // the lookups of that prefix. SHARE: clusters of four CTAs (two pairs) that split the decode
 // of each weight operand between partners (launched with cluster size 4); otherwise clusters
 // of one pair (cluster size 2), each CTA decoding its own 128 rows. Sharing pays when the
-// gathers bound the kernel (m >= 2); at m = 1 the SMs that clusters of four leave idle cost
-// more than it saves.
+// gathers bound the kernel (m >= 2) and both pairs have tokens (more than 512); at m = 1 the
+// SMs that clusters of four leave idle cost more than it saves.
 template <int BDT, int MB, bool SHARE>
 __global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ planes,
@@ -714,18 +714,24 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
         return AQ_ERR_CUDA;
 
+    // Decode sharing between two pairs pays where the gathers bound the kernel (m >= 2) and
+    // both pairs of a cluster have tokens (more than one 512-token tile).
+    const bool share = m >= 2 && tokens > kPairTokens;
     void (*kern)(const CUtensorMap, const uint8_t*, const uint16_t*, const uint16_t*, void*, int,
                  int, unsigned int*, int, int, int, int, int, size_t) =
-        m == 1 ? gemm_kernel<BDT, 1, false> : m == 2 ? gemm_kernel<BDT, 2, true>
-        : m == 3 ? gemm_kernel<BDT, 3, true>  : gemm_kernel<BDT, 4, true>;
-    const int csize = m == 1 ? 2 : 4;   // CTAs per cluster: one pair, or two sharing the decode
+        !share ? (m == 1 ? gemm_kernel<BDT, 1, false> : m == 2 ? gemm_kernel<BDT, 2, false>
+                  : m == 3 ? gemm_kernel<BDT, 3, false> : gemm_kernel<BDT, 4, false>)
+               : (m == 2 ? gemm_kernel<BDT, 2, true> : m == 3 ? gemm_kernel<BDT, 3, true>
+                                                      : gemm_kernel<BDT, 4, true>);
+    const int csize = share ? 4 : 2;   // CTAs per cluster: two pairs sharing the decode, or one
     static std::mutex mu;
-    static bool attr_done[kGemmMaxM][64] = {};
+    static bool attr_done[2 * kGemmMaxM][64] = {};
+    const int slot = (m - 1) + (share ? kGemmMaxM : 0);
     int dev = 0;
     if (cudaError_t e = cudaGetDevice(&dev); e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
     {
         std::lock_guard<std::mutex> lock(mu);
-        if (dev >= 0 && dev < 64 && !attr_done[m - 1][dev]) {
+        if (dev >= 0 && dev < 64 && !attr_done[slot][dev]) {
             if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
                 e != cudaSuccess)
                 return cuda_fail(e, "cudaFuncSetAttribute");
@@ -733,7 +739,7 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
                                                      (int)cudaSharedmemCarveoutMaxShared);
                 e != cudaSuccess)
                 return cuda_fail(e, "cudaFuncSetAttribute");
-            attr_done[m - 1][dev] = true;
+            attr_done[slot][dev] = true;
         }
     }
     cudaLaunchConfig_t cfg = {};

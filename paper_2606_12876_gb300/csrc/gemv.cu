@@ -587,21 +587,36 @@ aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     const long long units = (long long)d.S * m;       // (slice, book) pairs
     const long long items = units * d.RBc;
     if (items > 0x7fffffffLL) return AQ_ERR_UNSUPPORTED;   // item indices are 32-bit
-    // One CTA per SM. If whole shares of units keep at least 90% of the SMs busy, every CTA
-    // gets part of a single unit (one table build); otherwise items are balanced evenly and a
-    // CTA may span two units.
+    // One CTA per SM at most. Two ways to share the items: whole shares of single units
+    // (cpu CTAs per unit, one table build each), or an even split of all items over the SMs,
+    // where a CTA may straddle units and build two or more tables. Every call waits for its
+    // slowest CTA, so the choice takes the smaller worst-CTA cost, one table build being worth
+    // kTableItems row blocks of streaming (about 0.8 us against 23 ns per 1 KiB block at the
+    // per-SM share of HBM bandwidth).
+    constexpr long long kTableItems = 35;
     long long cpu = di.sms / units;
     if (cpu > d.RBc) cpu = d.RBc;
+    long long cost_cpu = -1;
+    if (cpu >= 1) cost_cpu = kTableItems + (d.RBc + cpu - 1) / cpu;
+    const long long grid_b = items < di.sms ? items : di.sms;
+    const long long qb = items / grid_b, rb = items % grid_b;
+    long long cost_b = 0;
+    for (long long b = 0; b < grid_b; ++b) {
+        const long long i0 = b * qb + (b < rb ? b : rb), i1 = i0 + qb + (b < rb ? 1 : 0);
+        const long long tables = (i1 - 1) / d.RBc - i0 / d.RBc + 1;
+        const long long c = tables * kTableItems + (i1 - i0);
+        if (c > cost_b) cost_b = c;
+    }
     int grid, q, r;   // a CTA's share: q items, one more for the first r shares
-    if (cpu >= 1 && cpu * units * 10 >= (long long)di.sms * 9) {
+    if (cost_cpu >= 0 && cost_cpu <= cost_b) {
         grid = (int)(cpu * units);
         q = d.RBc / (int)cpu;
         r = d.RBc % (int)cpu;
     } else {
         cpu = 0;
-        grid = (int)(items < di.sms ? items : di.sms);
-        q = (int)(items / grid);
-        r = (int)(items % grid);
+        grid = (int)grid_b;
+        q = (int)qb;
+        r = (int)rb;
     }
     return launch_pdl(kern, dim3(grid), dim3(kLutThreads), smem, st, (const uint8_t*)a.planes,
                       (const uint16_t*)a.books, (const uint16_t*)a.x, a.partials, a.status, m,
