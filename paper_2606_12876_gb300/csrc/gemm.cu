@@ -6,11 +6,12 @@
 // (tcgen05.mma.cta_group::2, M = 256 tokens, N = 256 rows, K = 16): each CTA holds 128 tokens
 // of every A block and 128 of the 256 weight rows, and the MMA reads both halves of both
 // operands, so every SM supplies half the operand bytes of what a single-CTA MMA of the same
-// work would read from its shared memory. A cluster holds two such pairs with the same rows and
-// consecutive token tiles. The CTA with the same role in the other pair (the partner) needs the
-// same 128 weight rows: each of the two decodes 64 of them and sends its slab to the other
-// with one shared-memory bulk copy per stage, which halves the codeword gathers (the decoders'
-// shared-memory traffic, what bounds the kernel at larger m).
+// work would read from its shared memory. A cluster holds NP = 1, 2 or 4 such pairs with the
+// same rows and consecutive token tiles. The CTAs with the same role in the other pairs (the
+// partners) need the same 128 weight rows: each of the NP decodes 128/NP of them and sends its
+// slab to the others with one shared-memory bulk copy per partner and stage, which divides the
+// codeword gathers (the decoders' shared-memory traffic, what bounds the kernel at larger m)
+// by NP.
 // Each CTA's tensor memory holds its 128 tokens x 256 rows for two token blocks (512 columns).
 // Roles (12 warps per CTA):
 //   warp 0      TMA producer: activation tiles (2-D tensor map, 128-byte swizzle, two
@@ -20,13 +21,13 @@
 //               leader CTA of a pair lane 0 issues the pair MMAs (2 token blocks x 4 K=16
 //               steps per stage) after one barrier wait per stage, and commits the
 //               activation-stage release and accumulator-ready barriers to its pair and the
-//               weight-stage release to all four CTAs. In the peer CTA lane 0 relays "stage
+//               weight-stage release to every CTA of the cluster. In the peer CTA lane 0 relays "stage
 //               ready" (its activations landed, its weight operand complete) to the leader
 //               with a remote mbarrier arrive.
 //   warp 2      (leader) lane 0 counts the leader's landed activation stages on the stage
 //               barrier.
-//   warp 3      lane 0 copies this CTA's decoded slab of each stage to the partner.
-//   warps 4-11  decoders: each thread owns one weight row and two groups of every stage; it
+//   warp 3      lane 0 copies this CTA's decoded slab of each stage to the partners.
+//   warps 4-11  decoders: each thread owns one weight row and 4/NP groups of every stage; it
 //               sums the m codewords in fp32 (book order), rounds once to fp16 and writes the
 //               16-byte group into the B tile in the UMMA K-major 128-byte-swizzle layout.
 //               Afterwards the same warps are the epilogue: tcgen05.ld from tensor memory,
@@ -62,8 +63,6 @@ constexpr int kGemmMaxM = 4;
 constexpr int kABlock = kBM * 128;            // one 128-token x 64-input block (16 KiB)
 constexpr int kAStage = kAcc * kABlock;       // 32 KiB
 constexpr int kBStage = kRows * 128;          // 16 KiB
-constexpr int kHalfRows = kRows / 2;          // rows decoded by one CTA (shared with its partner)
-constexpr int kHalfBytes = kHalfRows * 128;    // their 64-input slab of a weight stage (8 KiB)
 constexpr int kCodeBuf = kGemmMaxM * kRows * 32;   // one slice of codes, all planes (16 KiB)
 
 // Shared-memory map (offsets from a 1024-byte aligned base; identical in both CTAs of a pair,
@@ -292,12 +291,12 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
 }
 
 // One instantiation per book type and prefix length MB (= m): the decoders' code holds exactly
-// the lookups of that prefix. SHARE: clusters of four CTAs (two pairs) that split the decode
-// of each weight operand between partners (launched with cluster size 4); otherwise clusters
-// of one pair (cluster size 2), each CTA decoding its own 128 rows. Sharing pays when the
-// gathers bound the kernel (m >= 2) and both pairs have tokens (more than 512); at m = 1 the
-// SMs that clusters of four leave idle cost more than it saves.
-template <int BDT, int MB, bool SHARE>
+// the lookups of that prefix. NP: pairs per cluster (launched with cluster size 2*NP) that
+// split the decode of each weight operand between partners; with NP = 1 each CTA decodes its
+// own 128 rows. Sharing pays when the gathers bound the kernel (m >= 2) and every pair has
+// tokens; larger clusters leave more SMs idle (36 clusters of four, or fewer of eight, fit on
+// the 152 SMs), which at m = 1 costs more than the decode they save.
+template <int BDT, int MB, int NP>
 __global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ planes,
             const uint16_t* __restrict__ books, const uint16_t* __restrict__ scales, void* y,
@@ -324,19 +323,21 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
     volatile int& s_abort = *(volatile int*)(smem + kOffAbort);
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    // rank = role in the pair (0: leader, issues the MMAs; 1: peer). When sharing, a cluster
-    // of four CTAs = two CTA pairs with the same 256 weight rows and different 512-token
-    // tiles; pair = which token tile. The CTA with the same rank in the other pair is the
-    // partner: both need the same 128 weight rows, and each decodes half of them.
-    constexpr int kClusterLog = SHARE ? 2 : 1;
-    constexpr int DR = SHARE ? kHalfRows : kRows;   // rows decoded by one CTA
+    // rank = role in the pair (0: leader, issues the MMAs; 1: peer). A cluster = NP CTA pairs
+    // with the same 256 weight rows and different 512-token tiles; pair = which token tile.
+    // The CTAs with the same rank in the other pairs are the partners: all need the same 128
+    // weight rows, and each decodes 128/NP of them.
+    static_assert(NP == 1 || NP == 2 || NP == 4, "pairs per cluster");
+    constexpr bool SHARE = NP > 1;
+    constexpr int kClusterLog = NP == 1 ? 1 : NP == 2 ? 2 : 3;
+    constexpr int DR = kRows / NP;              // rows decoded by one CTA
+    constexpr int kSlab = DR * 128;             // their 64-input slab of a weight stage
     const uint32_t rank4 = cluster_rank();
     const uint32_t rank = rank4 & 1u, pair = SHARE ? rank4 >> 1 : 0u;
-    const uint32_t partner = ((pair ^ 1u) << 1) | rank;
     const int n0 = (blockIdx.x >> kClusterLog) * kBN;   // first output row of the pair tile
     const int r0 = n0 + (int)rank * kRows;      // first row of this CTA's weight operand
     const int rd0 = r0 + (int)pair * DR;        // first row decoded by this CTA
-    const int t0 = (blockIdx.y * (SHARE ? 2 : 1) + (int)pair) * kPairTokens;   // first token
+    const int t0 = (blockIdx.y * NP + (int)pair) * kPairTokens;   // first token
     const int nk = (in + kBK - 1) / kBK;        // K steps
     const int nsl = (nk + 3) / 4;               // 256-input slices
     const int rows_valid = max(0, min(DR, rows_pad - rd0));   // packed rows present
@@ -361,7 +362,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
         for (int s = 0; s < kStagesB; ++s) {
             // (peer) the copier with the partner's bytes, or the decoder warps
             mbar_init(&full_b[s], SHARE ? 1 : kDecWarps);
-            mbar_init(&empty_b[s], SHARE ? 2 : 1);   // commits of the pairs writing the stage
+            mbar_init(&empty_b[s], NP);           // commits of the pairs writing the stage
             // (leader) the copier or the decoder warps, plus the two relays
             mbar_init(&ready[s], SHARE ? 3 : kDecWarps + 2);
             mbar_init(&dec_done[s], kDecWarps);   // (SHARE) one arrival per decoder warp
@@ -450,9 +451,9 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
                         umma_f16_pair(tmem + i * kBN, umma_desc_sw128(a0 + i * kABlock + kk * 32),
                                       umma_desc_sw128(b0 + kk * 32), idesc, (it > 0 || kk > 0) ? 1u : 0u);
                 // The activation stage belongs to this pair; when sharing, the weight stage is
-                // also written by the partners, so its release goes to all four CTAs.
+                // also written by the partners, so its release goes to every CTA of the cluster.
                 umma_commit_pair(&empty_a[sa], (uint16_t)(0x3u << (2 * pair)));
-                umma_commit_pair(&empty_b[sb], (uint16_t)(SHARE ? 0xF : 0x3));
+                umma_commit_pair(&empty_b[sb], (uint16_t)((1u << (2 * NP)) - 1u));
             }
             umma_commit_pair(acc_full, (uint16_t)(0x3u << (2 * pair)));
         } else if (lane == 0) {
@@ -481,28 +482,30 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
         }
     } else if (warp == 3) {
         if (SHARE && lane == 0) {
-            // ---------------- copier: once this CTA's decoders have written their half of a
-            // weight stage, copy it into the partner's stage (same offset) with a bulk copy
-            // that completes on the partner's stage barrier, and count this CTA's half on its
-            // own stage barrier together with the partner's incoming bytes. The copy's
-            // source is free again once both pairs released the stage, which needs the copy
+            // ---------------- copier: once this CTA's decoders have written their slab of a
+            // weight stage, copy it into each partner's stage (same offset) with a bulk copy
+            // that completes on that partner's stage barrier, and count this CTA's slab on its
+            // own stage barrier together with the partners' incoming bytes. The copies'
+            // source is free again once every pair released the stage, which needs the copies
             // to have landed.
             uint64_t* stage_bar = rank == 0 ? ready : full_b;
-            const uint32_t peer_bar = map_to_rank(smem_u32(stage_bar), partner);
-            const uint32_t half0 = smem_u32(smem + kOffB) + pair * kHalfBytes;
-            const uint32_t peer_half0 = map_to_rank(half0, partner);
+            const uint32_t slab0 = smem_u32(smem + kOffB) + pair * kSlab;
             for (int it = 0; it < nk; ++it) {
                 const int sb = it % kStagesB;
                 if (!wait_or_abort(&dec_done[sb], (it / kStagesB) & 1, &s_abort, status)) break;
-                bulk_to_peer(peer_half0 + sb * kBStage, half0 + sb * kBStage, kHalfBytes,
-                             peer_bar + sb * 8);
-                mbar_arrive_expect_tx(&stage_bar[sb], kHalfBytes);
+#pragma unroll
+                for (int pp = 1; pp < NP; ++pp) {
+                    const uint32_t partner = ((((int)pair + pp) % NP) << 1) | rank;
+                    bulk_to_peer(map_to_rank(slab0, partner) + sb * kBStage, slab0 + sb * kBStage,
+                                 kSlab, map_to_rank(smem_u32(stage_bar), partner) + sb * 8);
+                }
+                mbar_arrive_expect_tx(&stage_bar[sb], (NP - 1) * kSlab);
             }
         }
     } else if (warp >= kDecWarp0) {
         // ---------------- decoders, then epilogue
         const int dt = tid - kDecWarp0 * 32;        // 0..255
-        constexpr int GPT = SHARE ? 2 : 4;          // groups per thread and stage
+        constexpr int GPT = DR * 8 / 256;           // groups per thread and stage
         const int n = dt & (DR - 1);                // decoded row owned by the thread
         const int cs = dt / DR;                     // groups GPT*cs .. GPT*cs + GPT-1 of a stage
         const int c0 = cs * GPT;
@@ -697,6 +700,13 @@ aq_status get_encode_fn(EncodeTiledFn* fn) {
     return AQ_OK;
 }
 
+// Four pairs per cluster (clusters of eight) measured slower than two at every m: only 16
+// clusters of eight fit at once (128 of the 152 SMs), which costs more than the halved
+// gathers save.
+int gemm_pairs_per_cluster(int m, int tokens) {
+    return m >= 2 && tokens > kPairTokens ? 2 : 1;
+}
+
 template <int BDT>
 aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
                    const void* scales, const void* x, int tokens, void* y, int y_dt, void* ws,
@@ -714,19 +724,20 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
         return AQ_ERR_CUDA;
 
-    // Decode sharing between two pairs pays where the gathers bound the kernel (m >= 2) and
-    // both pairs of a cluster have tokens (more than one 512-token tile).
-    const bool share = m >= 2 && tokens > kPairTokens;
-    void (*kern)(const CUtensorMap, const uint8_t*, const uint16_t*, const uint16_t*, void*, int,
-                 int, unsigned int*, int, int, int, int, int, size_t) =
-        !share ? (m == 1 ? gemm_kernel<BDT, 1, false> : m == 2 ? gemm_kernel<BDT, 2, false>
-                  : m == 3 ? gemm_kernel<BDT, 3, false> : gemm_kernel<BDT, 4, false>)
-               : (m == 2 ? gemm_kernel<BDT, 2, true> : m == 3 ? gemm_kernel<BDT, 3, true>
-                                                      : gemm_kernel<BDT, 4, true>);
-    const int csize = share ? 4 : 2;   // CTAs per cluster: two pairs sharing the decode, or one
+    // Pairs per cluster sharing the decode: sharing pays where the gathers bound the kernel
+    // (m >= 2) and every pair of a cluster has tokens (one 512-token tile per pair).
+    const int np = gemm_pairs_per_cluster(m, tokens);
+    using Kern = void (*)(const CUtensorMap, const uint8_t*, const uint16_t*, const uint16_t*,
+                          void*, int, int, unsigned int*, int, int, int, int, int, size_t);
+    const Kern k1[4] = {gemm_kernel<BDT, 1, 1>, gemm_kernel<BDT, 2, 1>, gemm_kernel<BDT, 3, 1>,
+                        gemm_kernel<BDT, 4, 1>};
+    const Kern k2[4] = {nullptr, gemm_kernel<BDT, 2, 2>, gemm_kernel<BDT, 3, 2>,
+                        gemm_kernel<BDT, 4, 2>};
+    const Kern kern = (np == 2 ? k2 : k1)[m - 1];
+    const int csize = 2 * np;         // CTAs per cluster
     static std::mutex mu;
     static bool attr_done[2 * kGemmMaxM][64] = {};
-    const int slot = (m - 1) + (share ? kGemmMaxM : 0);
+    const int slot = (m - 1) + (np == 2 ? kGemmMaxM : 0);
     int dev = 0;
     if (cudaError_t e = cudaGetDevice(&dev); e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
     {
@@ -744,7 +755,7 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
     }
     cudaLaunchConfig_t cfg = {};
     // x: one cluster per 256-row tile, y: one token tile per pair of the cluster
-    const int tok_tile = (csize / 2) * kPairTokens;
+    const int tok_tile = np * kPairTokens;
     cfg.gridDim = dim3(csize * ((d.out + kBN - 1) / kBN), (tokens + tok_tile - 1) / tok_tile);
     cfg.blockDim = dim3(kGemmThreads);
     cfg.dynamicSmemBytes = kGemmSmem;
