@@ -98,6 +98,22 @@ __device__ __forceinline__ void widen2(uint32_t w, float& lo, float& hi) {
     }
 }
 
+// lo += low half of w, hi += high half of w (16-bit floats of type DT), each with one
+// mixed-type add (16-bit operand, fp32 sum and result, sm_100 and later): the same result as
+// widening exactly and adding in fp32.
+template <int DT>
+__device__ __forceinline__ void add_widen2(uint32_t w, float& lo, float& hi) {
+    if constexpr (DT == AQ_F16) {
+        asm("{.reg .b16 l, h;\n\tmov.b32 {l, h}, %2;\n\t"
+            "add.rn.f32.f16 %0, l, %0;\n\tadd.rn.f32.f16 %1, h, %1;}"
+            : "+f"(lo), "+f"(hi) : "r"(w));
+    } else {
+        asm("{.reg .b16 l, h;\n\tmov.b32 {l, h}, %2;\n\t"
+            "add.rn.f32.bf16 %0, l, %0;\n\tadd.rn.f32.bf16 %1, h, %1;}"
+            : "+f"(lo), "+f"(hi) : "r"(w));
+    }
+}
+
 template <int DT>
 __device__ __forceinline__ void unpack8(const uint4& v, float* f) {
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
@@ -190,6 +206,23 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
         if (mbar_try_wait(bar, parity)) return true;
     } while (global_ns() - t0 < kWaitLimitNs);
     return false;
+}
+
+// The 32 code bytes of row o of a slice as stored (position p holds group (p + o) mod 32),
+// returned in group order: byte q of word j of u is the code of group 4j + q. A rotation by
+// o bytes: whole words by o / 4 in three conditional steps (no dynamically indexed register
+// array), then the byte part with funnel shifts.
+__device__ __forceinline__ void unrotate_codes(const uint32_t (&w)[8], int o, uint32_t (&u)[8]) {
+    const int r = o & 31, rw = r >> 2, rb = (r & 3) * 8;
+    uint32_t t[8], v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) t[i] = (rw & 1) ? w[(i + 7) & 7] : w[i];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = (rw & 2) ? t[(i + 6) & 7] : t[i];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) t[i] = (rw & 4) ? v[(i + 4) & 7] : v[i];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) u[j] = rb ? __funnelshift_l(t[(j + 7) & 7], t[j], rb) : t[j];
 }
 
 // Record a device-side failure in the workspace status word (first error wins).

@@ -446,6 +446,152 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
     }
 }
 
+// ------------------------------------------------------------------ tensor-core kernel (B = 8, 2..16 tokens, m <= 4)
+
+// Partials for 2..16 tokens with the multiply on the tensor cores (mma.sync m16n8k8, tf32
+// operands, fp32 accumulation). Each warp takes one 32-row block of the CTA's slice: the
+// block's code rows (first MB planes) are staged in shared memory in group order, and for
+// every group the lanes gather the codeword elements of their A-fragment positions (rows g,
+// g+8, g+16, g+24 of the block, elements c and c+4 of the group), sum them over the MB books
+// in fp32 in book order, round the sum once to tf32 and multiply with the activations (B
+// fragments: 8 or 16 tokens, exact in tf32). The codebooks are staged with the elements of
+// every codeword interleaved (0,4,1,5,2,6,3,7), so a lane's two elements are one 32-bit word;
+// each element is added to its fp32 sum by one mixed-type add (16-bit operand, fp32 sum).
+// (Eight bank-disjoint copies of each book, which make the gathers conflict-free, measured
+// slower: at m = 3, 4 their 32 KiB per book leave one CTA per SM.)
+constexpr int kMmaMaxM = 4;       // prefixes compiled for this kernel
+constexpr int kMmaXStride = 260;   // floats per staged token row (4 of padding: conflict-free)
+constexpr int kMmaCodeRow = 36;    // bytes per staged code row (4 of padding: conflict-free)
+
+inline size_t mma_smem_bytes(int nt, int mb) {
+    return (size_t)8 * nt * kMmaXStride * 4 + (size_t)mb * 4096 + (size_t)8 * mb * 32 * kMmaCodeRow;
+}
+
+__device__ __forceinline__ uint32_t to_tf32(float v) {
+    uint32_t r;
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(v));
+    return r;
+}
+
+__device__ __forceinline__ void mma_tf32(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+        "{%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
+template <int NT, int BDT, int MB>
+__global__ void __launch_bounds__(256)
+gemv_mma_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
+                const uint16_t* __restrict__ x, int x_dt, float* __restrict__ partials, int batch,
+                int in, int rows_pad, int RBc, int rb_per_chunk, size_t plane_bytes) {
+    constexpr int NBT = 8 * NT;                 // tokens held (missing ones are zero)
+    extern __shared__ __align__(16) unsigned char smem[];
+    float* xs = (float*)smem;                                            // [NBT][260]
+    uint32_t* books_s = (uint32_t*)(smem + NBT * kMmaXStride * 4);      // [MB][256][4]
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    unsigned char* codes_w =
+        smem + NBT * kMmaXStride * 4 + MB * 4096 + warp * (MB * 32 * kMmaCodeRow);
+    const int s = blockIdx.y, chunk = blockIdx.x;
+
+    pdl_wait();
+    pdl_launch_dependents();
+    for (int i = tid; i < NBT * 256; i += 256) {
+        const int t = i >> 8, c = i & 255, col = s * 256 + c;
+        float v = 0.0f;
+        if (t < batch && col < in) v = bits_to_f32_rt(x[(size_t)t * in + col], x_dt);
+        xs[t * kMmaXStride + c] = v;
+    }
+    for (int i = tid; i < MB * 256; i += 256) {
+        const uint4 w = __ldg((const uint4*)books + i);   // halves 0..7 of codeword i
+        *(uint4*)(books_s + i * 4) = make_uint4(prmt(w.x, w.z, 0x5410u), prmt(w.x, w.z, 0x7632u),
+                                                prmt(w.y, w.w, 0x5410u), prmt(w.y, w.w, 0x7632u));
+    }
+    __syncthreads();
+
+    const int g = lane >> 2, c = lane & 3;
+    const int rb0 = chunk * rb_per_chunk;
+    const int rb1 = min(rb0 + rb_per_chunk, RBc);
+    for (int rb = rb0 + warp; rb < rb1; rb += 8) {
+        // the block's code rows, in group order (lane = row)
+#pragma unroll
+        for (int k = 0; k < MB; ++k) {
+            const uint4* src = (const uint4*)(planes + k * plane_bytes +
+                                              ((size_t)s * rows_pad + (size_t)rb * 32 + lane) * 32);
+            const uint4 lo = ld_stream_v4(src), hi = ld_stream_v4(src + 1);
+            const uint32_t w[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+            uint32_t u[8];
+            unrotate_codes(w, lane, u);
+            uint32_t* dst = (uint32_t*)(codes_w + (k * 32 + lane) * kMmaCodeRow);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) dst[j] = u[j];
+        }
+        __syncwarp();
+        float acc[2][NT][4];
+#pragma unroll
+        for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) acc[mt][nt][e] = 0.0f;
+#pragma unroll 1
+        for (int q = 0; q < 8; ++q) {           // groups 4q .. 4q+3
+            uint32_t cw[4][MB];                 // codes of rows g + 8rr, one byte per group
+#pragma unroll
+            for (int rr = 0; rr < 4; ++rr)
+#pragma unroll
+                for (int k = 0; k < MB; ++k)
+                    cw[rr][k] = *(const uint32_t*)(codes_w + (k * 32 + g + 8 * rr) * kMmaCodeRow + 4 * q);
+#pragma unroll
+            for (int gg = 0; gg < 4; ++gg) {
+                const int G = 4 * q + gg;
+                uint32_t bf[NT][2];
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt) {
+                    const float* xr = xs + (8 * nt + g) * kMmaXStride + 8 * G + c;
+                    bf[nt][0] = __float_as_uint(xr[0]);
+                    bf[nt][1] = __float_as_uint(xr[4]);
+                }
+                uint32_t af[4][2];
+#pragma unroll
+                for (int rr = 0; rr < 4; ++rr) {
+                    float lo = -0.0f, hi = -0.0f;   // -0 + v = v exactly, so the first add widens
+#pragma unroll
+                    for (int k = 0; k < MB; ++k) {
+                        const uint32_t code = (cw[rr][k] >> (8 * gg)) & 0xffu;
+                        add_widen2<BDT>(books_s[(k * 256 + code) * 4 + c], lo, hi);
+                    }
+                    af[rr][0] = to_tf32(lo);
+                    af[rr][1] = to_tf32(hi);
+                }
+#pragma unroll
+                for (int mt = 0; mt < 2; ++mt) {
+                    const uint32_t a[4] = {af[2 * mt][0], af[2 * mt + 1][0], af[2 * mt][1], af[2 * mt + 1][1]};
+#pragma unroll
+                    for (int nt = 0; nt < NT; ++nt) mma_tf32(acc[mt][nt], a, bf[nt]);
+                }
+            }
+        }
+        __syncwarp();                           // the code buffer is refilled next
+#pragma unroll
+        for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+                const int r0 = rb * 32 + mt * 16 + g, t0 = 8 * nt + 2 * c;
+                float* p0 = partials + ((size_t)s * batch + t0) * rows_pad + r0;
+                if (t0 < batch) {
+                    p0[0] = acc[mt][nt][0];
+                    p0[8] = acc[mt][nt][2];
+                }
+                if (t0 + 1 < batch) {
+                    p0[rows_pad] = acc[mt][nt][1];
+                    p0[rows_pad + 8] = acc[mt][nt][3];
+                }
+            }
+    }
+}
+
 // ------------------------------------------------------------------ split-K reduction
 
 // y[t][r] = s[r] * sum over the P partial planes p of partials[p*batch + t][r] (R1: the row
@@ -643,6 +789,42 @@ aq_status run_direct(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
                       a.partials, m, a.batch, d.in, d.rows_pad, d.RBc, rbpc, d.plane_bytes);
 }
 
+template <int NT, int BDT, int MB>
+aq_status run_mma(const Dims& d, const GemvArgs& a, cudaStream_t st) {
+    DeviceInfo di;
+    if (aq_status e = device_info(&di); e != AQ_OK) return e;
+    const size_t smem = mma_smem_bytes(NT, MB);
+    auto kern = gemv_mma_kernel<NT, BDT, MB>;
+    int occ = 0;
+    if (aq_status e = prepare(kern, smem, 256, 0, &occ); e != AQ_OK) return e;
+    const int target = di.sms * occ;
+    int chunks = (target + d.S - 1) / d.S;
+    chunks = chunks < 1 ? 1 : (chunks > d.RBc ? d.RBc : chunks);
+    const int rbpc = (d.RBc + chunks - 1) / chunks;
+    chunks = (d.RBc + rbpc - 1) / rbpc;
+    return launch_pdl(kern, dim3(chunks, d.S), dim3(256), smem, st, (const uint8_t*)a.planes,
+                      (const uint16_t*)a.books, (const uint16_t*)a.x, a.x_dt, a.partials, a.batch,
+                      d.in, d.rows_pad, d.RBc, rbpc, d.plane_bytes);
+}
+
+template <int BDT>
+aq_status dispatch_mma(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
+    if (a.batch <= 8) {
+        switch (m) {
+            case 1: return run_mma<1, BDT, 1>(d, a, st);
+            case 2: return run_mma<1, BDT, 2>(d, a, st);
+            case 3: return run_mma<1, BDT, 3>(d, a, st);
+            default: return run_mma<1, BDT, 4>(d, a, st);
+        }
+    }
+    switch (m) {
+        case 1: return run_mma<2, BDT, 1>(d, a, st);
+        case 2: return run_mma<2, BDT, 2>(d, a, st);
+        case 3: return run_mma<2, BDT, 3>(d, a, st);
+        default: return run_mma<2, BDT, 4>(d, a, st);
+    }
+}
+
 template <int B, int BDT, int SDT>
 aq_status dispatch_direct(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     if (a.batch <= 1) return run_direct<1, B, BDT, SDT>(d, m, a, st);
@@ -670,6 +852,8 @@ static aq_status launch_product(const Dims& d, int m, const void* planes, const 
             default: return run_lut<AQ_BF16, AQ_BF16>(d, m, a, st);
         }
     }
+    if (d.B == 8 && batch >= 2 && m <= kMmaMaxM)
+        return bb ? dispatch_mma<AQ_BF16>(d, m, a, st) : dispatch_mma<AQ_F16>(d, m, a, st);
     switch ((d.B == 16) * 4 + bb * 2 + sb) {
         case 0: return dispatch_direct<8, AQ_F16, AQ_F16>(d, m, a, st);
         case 1: return dispatch_direct<8, AQ_F16, AQ_BF16>(d, m, a, st);
