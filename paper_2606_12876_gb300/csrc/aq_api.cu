@@ -99,11 +99,11 @@ size_t gemm_ws_bytes(const Dims& d, int tokens) {
 }
 
 size_t gemv_ws_bytes(const Dims& d, int batch) {
-    // Partial planes: S per token, or S per book of the largest prefix the table-lookup
-    // kernel serves at batch 1.
+    // Partial planes: S per token, or S per book and token for the largest prefix the
+    // table-lookup kernel serves at this batch.
     size_t planes = (size_t)d.S * (size_t)batch;
-    const int mt = d.M < aq::kLutMaxM ? d.M : aq::kLutMaxM;
-    if (aq::uses_lut(d, mt, batch) && (size_t)d.S * mt > planes) planes = (size_t)d.S * mt;
+    const int lm = aq::lut_max_m(batch), mt = d.M < lm ? d.M : lm;
+    if (mt > 0 && aq::uses_lut(d, mt, batch)) planes = (size_t)d.S * (size_t)batch * (size_t)mt;
     return aq::ws_partial_offset(d) + planes * (size_t)d.rows_pad * 4;
 }
 

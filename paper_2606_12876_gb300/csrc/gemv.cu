@@ -33,19 +33,21 @@
 namespace aq {
 namespace {
 
-// ------------------------------------------------------------------ LUT kernel (B = 8, b = 1)
+// ------------------------------------------------------------------ LUT kernel (B = 8, b <= 4)
 
 constexpr int kCons = 16;                         // consumer warps (two 32-row blocks each per stage)
 constexpr int kLutThreads = (kCons + 1) * 32;     // + one producer warp
 constexpr int kStageRb = 2 * kCons;               // 32-row blocks per stage: a 32 KiB plane copy
 constexpr int kSlot = kStageRb * 1024;            // one ring slot = one plane of one stage
 constexpr int kSlots = 4;                         // largest ring depth (128 KiB)
-constexpr int kXSlices = 8;                       // activation slices staged up front
-constexpr int kTBytes = 65536;                    // two single-book tables, interleaved
+constexpr int kXStage = 8;                        // (token, slice) activation rows staged up front
 
-// Shared memory: [T 64 KiB][codebooks m x 4 KiB][activations 8 x 1 KiB fp32][ring][barriers]
-inline size_t lut_smem_bytes(int m, int slots) {
-    return (size_t)kTBytes + (size_t)m * 4096 + kXSlices * 1024 + (size_t)slots * kSlot +
+// Tables: 64 KiB per two tokens (NT = 1 uses the two halves for consecutive units).
+constexpr int lut_table_bytes(int nt) { return nt == 4 ? 131072 : 65536; }
+
+// Shared memory: [T][codebooks m x 4 KiB][activations 8 x 1 KiB fp32][ring][barriers]
+inline size_t lut_smem_bytes(int nt, int m, int slots) {
+    return (size_t)lut_table_bytes(nt) + (size_t)m * 4096 + kXStage * 1024 + (size_t)slots * kSlot +
            2 * kSlots * 8;
 }
 
@@ -63,26 +65,34 @@ inline size_t lut_smem_bytes(int m, int slots) {
 // built while the other half still serves the previous unit; j*256 + g*4 is produced from a
 // code byte by one prmt.
 //
+// NT = 2 or 4 tokens (batch 2..4): one table per token, token t in the 64 KiB table t/2 at
+// half t%2, so the same prmt offset serves every token and the token is a constant of the
+// load: a code byte costs one prmt plus one load and one add per token. The tables are
+// rebuilt in place (a barrier first) and the partial planes are per (unit, token).
+//
 // A CTA owns the items [i0, i1) and walks them in stages of up to 32 items that never cross a
 // unit. For each stage the producer warp copies the stage's rows of the unit's book plane into
 // one ring slot with a TMA bulk copy (32 KiB; the CTA's rows of a slice are contiguous in
 // every plane), and consumer warp w looks up items w and w + 16 of the stage, so each wait on
 // the ring serves two row blocks. The codebooks and the activations of the CTA's first slices
 // are requested before any code.
-template <int BDT, int XDT>
+template <int BDT, int XDT, int NT>
 __global__ void __launch_bounds__(kLutThreads, 1)
 gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
                 const uint16_t* __restrict__ x, float* __restrict__ partials,
                 unsigned int* __restrict__ status, int m, int in, int ng, int rows_pad, int RBc,
-                size_t plane_bytes, int nslots, int cpu, int q, int r, int static_weights) {
+                size_t plane_bytes, int nslots, int cpu, int q, int r, int static_weights,
+                int batch) {
+    constexpr int kTB = lut_table_bytes(NT);
+    constexpr int kXSlices = kXStage / NT;      // activation slices staged per token
     extern __shared__ __align__(128) unsigned char smem[];
     unsigned char* T = smem;
-    uint4* Cb = (uint4*)(smem + kTBytes);                          // [m][256] codewords
-    // [kXSlices][256] activations in fp32; group g of a slice at 128-byte line g/4, its two
-    // 16-byte halves at quads (2*(g%4) + half) ^ (g/4 mod 8), so the table build's reads
+    uint4* Cb = (uint4*)(smem + kTB);                              // [m][256] codewords
+    // [NT][kXSlices][256] activations in fp32; group g of a slice at 128-byte line g/4, its
+    // two 16-byte halves at quads (2*(g%4) + half) ^ (g/4 mod 8), so the table build's reads
     // (eight lanes at eight different lines) hit eight different bank quads.
-    unsigned char* xs = smem + kTBytes + (size_t)m * 4096;
-    unsigned char* ring = xs + kXSlices * 1024;                    // nslots x 32 KiB
+    unsigned char* xs = smem + kTB + (size_t)m * 4096;
+    unsigned char* ring = xs + kXStage * 1024;                     // nslots x 32 KiB
     uint64_t* full = (uint64_t*)(ring + (size_t)nslots * kSlot);
     uint64_t* empty = full + kSlots;
     __shared__ volatile int s_abort;
@@ -175,9 +185,9 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
     pdl_launch_dependents();    // the split-K reduction may become resident (it waits for us)
     if (!static_weights) load_books();
     uint2 x_r = make_uint2(0u, 0u);
-    if (tid < kXSlices * 64) {
-        const int col = (s_first + (tid >> 6)) * 256 + (tid & 63) * 4;
-        if (col < in) x_r = __ldg((const uint2*)(x + col));
+    if (tid < kXStage * 64) {                   // row tid/64 = token * kXSlices + slice
+        const int xt = (tid >> 6) / kXSlices, col = (s_first + (tid >> 6) % kXSlices) * 256 + (tid & 63) * 4;
+        if (xt < batch && col < in) x_r = __ldg((const uint2*)(x + (size_t)xt * in + col));
     }
 
     if (warp == kCons) {
@@ -203,7 +213,7 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
             const int i = tid + r * kCons * 32;
             if (i < m * 256) Cb[i] = cb_r[r];
         }
-        if (tid < kXSlices * 64) {
+        if (tid < kXStage * 64) {
             const int e = tid & 63, g = e >> 1;
             float4 f;
             widen2<XDT>(x_r.x, f.x, f.y);
@@ -238,10 +248,11 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
         for (Walk w = walk_start(); w.it < i1; walk_next(w)) {
             const int n = w.n, s = w.s, rb = w.rb;
             if (s != cur_s || w.k != cur_k) {
-                if (s != cur_s) {
+                // Activations of the four groups 4gq..4gq+3 of slice s for token t.
+                auto load_xv = [&](int t) {
                     const int sl = s - s_first;
                     if (sl < kXSlices) {
-                        const unsigned char* xb = xs + sl * 1024 + gq * 128;
+                        const unsigned char* xb = xs + (t * kXSlices + sl) * 1024 + gq * 128;
 #pragma unroll
                         for (int u = 0; u < 4; ++u) {
                             const float4 lo = *(const float4*)(xb + (((2 * u) ^ gq) & 7) * 16);
@@ -256,41 +267,57 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                         for (int u = 0; u < 4; ++u) {
                             const int g = s * 32 + gq * 4 + u;
                             uint4 xr = make_uint4(0u, 0u, 0u, 0u);
-                            if (g < ng) xr = __ldg((const uint4*)x + g);
+                            if (t < batch && g < ng) xr = __ldg((const uint4*)(x + (size_t)t * in) + g);
                             float f[8];
                             unpack8<XDT>(xr, f);
 #pragma unroll
                             for (int e = 0; e < 4; ++e) xv[u][e] = make_float2(f[2 * e], f[2 * e + 1]);
                         }
                     }
-                    cur_s = s;
-                }
-                cur_k = w.k;
-                h ^= 1;
-                // The other half served the previous unit; this half was last read two units
-                // ago, before every consumer passed the previous unit's barrier.
-                unsigned char* Th = T + h * 128 + gq * 16;
-                uint4 cw[4];
+                };
+                // Entries j = 16*warp + ph + 4i, groups 4gq..4gq+3 of the unit's book, for the
+                // activations in xv, stored as 16-byte pieces at Th.
+                auto build = [&](unsigned char* Th) {
+                    uint4 cw[4];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) cw[i] = Cb[cur_k * 256 + warp * 16 + ph + 4 * i];
+                    for (int i = 0; i < 4; ++i) cw[i] = Cb[w.k * 256 + warp * 16 + ph + 4 * i];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    float c[8];
-                    unpack8<BDT>(cw[i], c);
-                    float r[4];
+                    for (int i = 0; i < 4; ++i) {
+                        float c[8];
+                        unpack8<BDT>(cw[i], c);
+                        float r[4];
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        float2 t = make_float2(xv[u][0].x * c[0], xv[u][0].y * c[1]);
-                        t = ffma2(xv[u][1], make_float2(c[2], c[3]), t);
-                        t = ffma2(xv[u][2], make_float2(c[4], c[5]), t);
-                        t = ffma2(xv[u][3], make_float2(c[6], c[7]), t);
-                        r[u] = t.x + t.y;
+                        for (int u = 0; u < 4; ++u) {
+                            float2 t = make_float2(xv[u][0].x * c[0], xv[u][0].y * c[1]);
+                            t = ffma2(xv[u][1], make_float2(c[2], c[3]), t);
+                            t = ffma2(xv[u][2], make_float2(c[4], c[5]), t);
+                            t = ffma2(xv[u][3], make_float2(c[6], c[7]), t);
+                            r[u] = t.x + t.y;
+                        }
+                        *(float4*)(Th + (warp * 16 + ph + 4 * i) * 256) = make_float4(r[0], r[1], r[2], r[3]);
                     }
-                    *(float4*)(Th + (warp * 16 + ph + 4 * i) * 256) = make_float4(r[0], r[1], r[2], r[3]);
+                };
+                if constexpr (NT == 1) {
+                    if (s != cur_s) load_xv(0);
+                    h ^= 1;
+                    // The other half served the previous unit; this half was last read two
+                    // units ago, before every consumer passed the previous unit's barrier.
+                    build(T + h * 128 + gq * 16);
+                } else {
+                    if (cur_k >= 0) named_barrier(1, kCons * 32);   // previous unit looked up
+#pragma unroll 1
+                    for (int t = 0; t < NT; ++t) {
+                        load_xv(t);
+                        build(T + (t >> 1) * 65536 + (t & 1) * 128 + gq * 16);
+                    }
                 }
+                cur_s = s;
+                cur_k = w.k;
                 named_barrier(1, kCons * 32);
             }
-            float part0 = 0.0f, part1 = 0.0f;
+            float part0[NT], part1[NT];
+#pragma unroll
+            for (int t = 0; t < NT; ++t) part0[t] = part1[t] = 0.0f;
             bool ok = !s_abort;
             if (ok && !mbar_wait(&full[slot], phase)) {
                 record_status(status, AQ_ERR_TIMEOUT);
@@ -301,7 +328,8 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                 // Each lane reads its row's 32 code bytes of item warp (and warp + 16) as two
                 // 16-byte halves. The prmt forms the table offset of a code byte: byte0 = goff
                 // byte i, byte1 = code byte i, bytes 2-3 = sign of the goff byte (0). The
-                // table half is a constant of the load, so a lookup is prmt, load and add.
+                // table half (and for NT > 1 the token) is a constant of the load, so a lookup
+                // is prmt, then a load and an add per token.
                 const unsigned char* row0 = ring + (size_t)slot * kSlot + warp * 1024 + lane * 32;
                 const uint4 a0 = *(const uint4*)(row0 + c0 * 16);
                 const uint4 b0 = *(const uint4*)(row0 + (c0 ^ 1) * 16);
@@ -317,31 +345,41 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                 }
                 auto look = [&](auto half) {
                     const unsigned char* Tb = T + decltype(half)::value;
-                    auto ld = [&](uint32_t wq, uint32_t g, uint32_t sel) {
-                        return *(const float*)(Tb + prmt(wq, g, sel));
+                    // token t of the table entry at offset o (token 0 when NT = 1)
+                    auto ld = [&](uint32_t o, int t) {
+                        return *(const float*)(Tb + (t >> 1) * 65536 + (t & 1) * 128 + o);
                     };
                     if (two) {
 #pragma unroll
                         for (int qq = 0; qq < 8; ++qq) {
                             const uint32_t g = goff[qq];
-                            const float v0 = ld(w0[qq], g, 0xCC04u), u0 = ld(w1[qq], g, 0xCC04u);
-                            const float v1 = ld(w0[qq], g, 0xDD15u), u1 = ld(w1[qq], g, 0xDD15u);
-                            const float v2 = ld(w0[qq], g, 0xEE26u), u2 = ld(w1[qq], g, 0xEE26u);
-                            const float v3 = ld(w0[qq], g, 0xFF37u), u3 = ld(w1[qq], g, 0xFF37u);
-                            part0 += (v0 + v1) + (v2 + v3);
-                            part1 += (u0 + u1) + (u2 + u3);
+                            const uint32_t o0 = prmt(w0[qq], g, 0xCC04u), p0 = prmt(w1[qq], g, 0xCC04u);
+                            const uint32_t o1 = prmt(w0[qq], g, 0xDD15u), p1 = prmt(w1[qq], g, 0xDD15u);
+                            const uint32_t o2 = prmt(w0[qq], g, 0xEE26u), p2 = prmt(w1[qq], g, 0xEE26u);
+                            const uint32_t o3 = prmt(w0[qq], g, 0xFF37u), p3 = prmt(w1[qq], g, 0xFF37u);
+#pragma unroll
+                            for (int t = 0; t < NT; ++t) {
+                                const float v0 = ld(o0, t), u0 = ld(p0, t), v1 = ld(o1, t), u1 = ld(p1, t);
+                                const float v2 = ld(o2, t), u2 = ld(p2, t), v3 = ld(o3, t), u3 = ld(p3, t);
+                                part0[t] += (v0 + v1) + (v2 + v3);
+                                part1[t] += (u0 + u1) + (u2 + u3);
+                            }
                         }
                     } else {
 #pragma unroll
                         for (int qq = 0; qq < 8; ++qq) {
                             const uint32_t g = goff[qq];
-                            const float v0 = ld(w0[qq], g, 0xCC04u), v1 = ld(w0[qq], g, 0xDD15u);
-                            const float v2 = ld(w0[qq], g, 0xEE26u), v3 = ld(w0[qq], g, 0xFF37u);
-                            part0 += (v0 + v1) + (v2 + v3);
+                            const uint32_t o0 = prmt(w0[qq], g, 0xCC04u), o1 = prmt(w0[qq], g, 0xDD15u);
+                            const uint32_t o2 = prmt(w0[qq], g, 0xEE26u), o3 = prmt(w0[qq], g, 0xFF37u);
+#pragma unroll
+                            for (int t = 0; t < NT; ++t) {
+                                const float v0 = ld(o0, t), v1 = ld(o1, t), v2 = ld(o2, t), v3 = ld(o3, t);
+                                part0[t] += (v0 + v1) + (v2 + v3);
+                            }
                         }
                     }
                 };
-                if (h) look(std::integral_constant<int, 128>());
+                if (NT == 1 && h) look(std::integral_constant<int, 128>());
                 else look(std::integral_constant<int, 0>());
             }
             __syncwarp();
@@ -351,9 +389,13 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                 phase ^= 1u;
             }
             if (ok && warp < n) {
-                float* dst = partials + ((size_t)s * m + cur_k) * rows_pad + (size_t)(rb + warp) * 32 + lane;
-                dst[0] = part0;
-                if (warp + kCons < n) dst[kCons * 32] = part1;
+#pragma unroll
+                for (int t = 0; t < NT; ++t) {
+                    if (t >= batch) break;
+                    float* dst = partials + (((size_t)s * m + cur_k) * batch + t) * rows_pad + (size_t)(rb + warp) * 32 + lane;
+                    dst[0] = part0[t];
+                    if (warp + kCons < n) dst[kCons * 32] = part1[t];
+                }
             }
         }
     }
@@ -717,17 +759,17 @@ struct GemvArgs {
     unsigned int* status;
 };
 
-template <int BDT, int XDT>
+template <int BDT, int XDT, int NT>
 aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     DeviceInfo di;
     if (aq_status e = device_info(&di); e != AQ_OK) return e;
-    auto kern = gemv_lut_kernel<BDT, XDT>;
-    // As many 16 KiB ring slots as fit next to the table, codebooks and activations (<= 8).
-    const size_t fixed = lut_smem_bytes(m, 0) + 8192;   // + static shared memory and slack
+    auto kern = gemv_lut_kernel<BDT, XDT, NT>;
+    // As many 32 KiB ring slots as fit next to the tables, codebooks and activations (<= 4).
+    const size_t fixed = lut_smem_bytes(NT, m, 0) + 8192;   // + static shared memory and slack
     int nslots = di.smem_optin > (int)fixed ? (int)((di.smem_optin - fixed) / kSlot) : 0;
     if (nslots > kSlots) nslots = kSlots;
     if (nslots < 2) return AQ_ERR_UNSUPPORTED;
-    const size_t smem = lut_smem_bytes(m, nslots);
+    const size_t smem = lut_smem_bytes(NT, m, nslots);
     int occ = 0;
     if (aq_status e = prepare(kern, smem, kLutThreads, m, &occ); e != AQ_OK) return e;
     const long long units = (long long)d.S * m;       // (slice, book) pairs
@@ -767,7 +809,7 @@ aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     return launch_pdl(kern, dim3(grid), dim3(kLutThreads), smem, st, (const uint8_t*)a.planes,
                       (const uint16_t*)a.books, (const uint16_t*)a.x, a.partials, a.status, m,
                       d.in, d.ng, d.rows_pad, d.RBc, d.plane_bytes, nslots, (int)cpu, q, r,
-                      (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0);
+                      (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0, a.batch);
 }
 
 template <int NB, int B, int BDT, int SDT>
@@ -845,11 +887,27 @@ static aq_status launch_product(const Dims& d, int m, const void* planes, const 
                (float*)((char*)ws + ws_partial_offset(d)), (unsigned int*)ws};
     const int bb = d.book_dt == AQ_BF16, xb = x_dt == AQ_BF16, sb = d.scale_dt == AQ_BF16;
     if (uses_lut(d, m, batch)) {
+        if (batch == 1) {
+            switch (bb * 2 + xb) {
+                case 0: return run_lut<AQ_F16, AQ_F16, 1>(d, m, a, st);
+                case 1: return run_lut<AQ_F16, AQ_BF16, 1>(d, m, a, st);
+                case 2: return run_lut<AQ_BF16, AQ_F16, 1>(d, m, a, st);
+                default: return run_lut<AQ_BF16, AQ_BF16, 1>(d, m, a, st);
+            }
+        }
+        if (batch == 2) {
+            switch (bb * 2 + xb) {
+                case 0: return run_lut<AQ_F16, AQ_F16, 2>(d, m, a, st);
+                case 1: return run_lut<AQ_F16, AQ_BF16, 2>(d, m, a, st);
+                case 2: return run_lut<AQ_BF16, AQ_F16, 2>(d, m, a, st);
+                default: return run_lut<AQ_BF16, AQ_BF16, 2>(d, m, a, st);
+            }
+        }
         switch (bb * 2 + xb) {
-            case 0: return run_lut<AQ_F16, AQ_F16>(d, m, a, st);
-            case 1: return run_lut<AQ_F16, AQ_BF16>(d, m, a, st);
-            case 2: return run_lut<AQ_BF16, AQ_F16>(d, m, a, st);
-            default: return run_lut<AQ_BF16, AQ_BF16>(d, m, a, st);
+            case 0: return run_lut<AQ_F16, AQ_F16, 4>(d, m, a, st);
+            case 1: return run_lut<AQ_F16, AQ_BF16, 4>(d, m, a, st);
+            case 2: return run_lut<AQ_BF16, AQ_F16, 4>(d, m, a, st);
+            default: return run_lut<AQ_BF16, AQ_BF16, 4>(d, m, a, st);
         }
     }
     if (d.B == 8 && batch >= 2 && m <= kMmaMaxM)
