@@ -120,13 +120,13 @@ aq_status aq_decode(const aq_layout* layout, int m, const void* planes, const vo
  *   y         : device, [batch][d_out] of y_dtype (AQ_F16, AQ_BF16 or AQ_F32), row-major
  *   workspace : device scratch of at least aq_gemv_workspace_bytes(layout, batch) bytes:
  *               a status word and fp32 partial sums for every row: one per 256-input
- *               slice and token, or, at batch 1 with 2^8-entry books, one per slice and
- *               codebook of the largest prefix (up to 8) served that way. Zero-fill it once
- *               before its first use (aq_workspace_init); every call leaves it ready for the
- *               next one.
+ *               slice and token, or, with 2^8-entry books at batch 1 (batch 2..4), one per
+ *               slice, token and codebook of the largest prefix up to 8 (up to 4) served
+ *               that way. Zero-fill it once before its first use (aq_workspace_init); every
+ *               call leaves it ready for the next one.
  *               Calls that may overlap on the GPU must not share a workspace.
  * Two kernels are enqueued, both with programmatic dependent launch: the product (fp32
- * partial sums per 256-input slice, and per codebook at batch 1 with 2^8-entry books, into
+ * partial sums per 256-input slice, and per codebook at batch 1..4 with 2^8-entry books, into
  * the workspace) and a split-K reduction that sums each row's partials, scales it and
  * writes y. Each waits for the preceding grid before reading memory. The partials of each
  * row are summed in a fixed order, so the result does not depend on scheduling.
