@@ -346,6 +346,7 @@ def own_arm(args):
         x_host = torch.from_numpy(x_bits.view(np.int16)).view(torch.float16).pin_memory()
         y_host = torch.empty(len(ms), out, dtype=torch.float16).pin_memory()
         x_dev = torch.empty_like(x_host, device=dev)
+        y_dev = torch.empty(len(ms), out, dtype=torch.float16, device=dev)   # one row per m
         e_s, e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         n_e2e = max(20, args.steps // 2)
         with torch.cuda.stream(stream):
@@ -356,9 +357,9 @@ def own_arm(args):
                 x_dev.copy_(x_host, non_blocking=True)
                 planes = copies[i % ncopies]
                 for j, m in enumerate(ms):
-                    aq.aq_gemv(L, m, planes, lin.books, lin.scales, x_dev, aq.AQ_F16, 1, ys[m],
-                               aq.AQ_F16, ws)
-                    y_host[j].copy_(ys[m][0], non_blocking=True)
+                    aq.aq_gemv(L, m, planes, lin.books, lin.scales, x_dev, aq.AQ_F16, 1,
+                               y_dev[j:j + 1], aq.AQ_F16, ws)
+                y_host.copy_(y_dev, non_blocking=True)    # the step's four results
             e_e.record()
         torch.cuda.synchronize(dev)
         e2e_ms = e_s.elapsed_time(e_e) / n_e2e

@@ -95,8 +95,15 @@ def _ptr(t):
     return t.data_ptr()
 
 
+# The current stream as a raw handle, without building a Stream object per call (torch's
+# accessor when present).
+_raw_stream = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+
+
 def _stream(stream):
     if stream is None:
+        if _raw_stream is not None:
+            return _raw_stream(torch.cuda.current_device())
         return torch.cuda.current_stream().cuda_stream
     if isinstance(stream, int):
         return stream

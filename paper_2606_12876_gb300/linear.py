@@ -10,7 +10,7 @@ import torch
 from . import (AQ_BF16, AQ_F16, AQ_F32, AQ_LAYOUT_STATIC_WEIGHTS, DTYPES, TORCH_DTYPES, Layout,
                aq_decode, aq_gemm,
                aq_gemv, aq_pack, gemm_workspace_bytes, gemv_workspace_bytes, packed_bytes,
-               workspace)
+               workspace, _stream)
 
 
 def _u16_to_device(a, device):
@@ -59,12 +59,21 @@ class AQLinear:
         return self.planes[: packed_bytes(self.layout, m)]
 
     def _workspace(self, kind, n):
-        nbytes = (gemv_workspace_bytes if kind == "gemv" else gemm_workspace_bytes)(self.layout, n)
-        key = (kind, torch.cuda.current_stream(self.device).cuda_stream)
+        # One workspace per (kind, stream), grown on demand; GEMV calls (batch <= 16) also
+        # remember the size per batch, so a repeated call makes no size query.
+        stream = _stream(None)
+        key = (kind, stream)
         ws = self._ws.get(key)
+        if kind == "gemv":
+            known = self._ws.get((kind, stream, n))
+            if known is not None and ws is not None and ws.numel() >= known:
+                return ws
+        nbytes = (gemv_workspace_bytes if kind == "gemv" else gemm_workspace_bytes)(self.layout, n)
         if ws is None or ws.numel() < nbytes:
             ws = workspace(nbytes, self.device)
             self._ws[key] = ws
+        if kind == "gemv":
+            self._ws[(kind, stream, n)] = nbytes
         return ws
 
     def decode(self, m, out=None):
