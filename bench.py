@@ -79,6 +79,19 @@ def dist_env():
     return world, rank, local
 
 
+def whole_job(ms_total, world, bytes_step, steps, device=None):
+    """The slowest rank's timed-region length (ms) and the whole-job throughput (GB/s): every
+    rank runs its own replica of the step on its own data (weak scaling), so the job moves
+    world * bytes_step bytes per step. With world > 1 the process group must be initialised."""
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        t = torch.tensor([ms_total], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_total = float(t.item())
+    return ms_total, world * bytes_step * steps / (ms_total / 1e3) / 1e9
+
+
 class ClockSampler:
     """nvidia-smi clock / throttle samples during the timed region."""
 
@@ -315,12 +328,8 @@ def own_arm(args):
     ms_total = time_graph(g_timed)
     barrier()
     clk = clocks.stop()
-    if world > 1:
-        t = torch.tensor([ms_total], device=dev, dtype=torch.float64)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms_total = float(t.item())
+    ms_total, value = whole_job(ms_total, world, bytes_step, args.steps, device=dev)
     ms_step = ms_total / args.steps
-    value = world * bytes_step * args.steps / (ms_total / 1e3) / 1e9
 
     # Per prefix: a graph of `steps` launches of that prefix alone (rotating weight copies),
     # CUDA events around the graph only, so back-to-back launches keep their overlap.
