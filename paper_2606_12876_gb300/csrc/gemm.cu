@@ -233,25 +233,6 @@ __device__ __forceinline__ void sts128(uint32_t a, uint4 v) {
                  : "memory");
 }
 
-// Two fp32 additions in one instruction (each lane rounded to nearest, as a scalar add).
-__device__ __forceinline__ float2 add2(float2 a, float2 b) {
-    unsigned long long ar, br, dr;
-    asm("mov.b64 %0, {%1, %2};" : "=l"(ar) : "f"(a.x), "f"(a.y));
-    asm("mov.b64 %0, {%1, %2};" : "=l"(br) : "f"(b.x), "f"(b.y));
-    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(dr) : "l"(ar), "l"(br));
-    float2 d;
-    asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(dr));
-    return d;
-}
-
-// One 32-bit word of a codeword (two 16-bit values, low half first) -> two floats.
-template <int BDT>
-__device__ __forceinline__ float2 widen2f(uint32_t w) {
-    float2 r;
-    widen2<BDT>(w, r.x, r.y);
-    return r;
-}
-
 __device__ __forceinline__ uint32_t f16x2(float2 v) {   // {lo, hi} -> packed fp16 pair, RN
     uint32_t h;
     asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(h) : "f"(v.y), "f"(v.x));
@@ -266,17 +247,25 @@ __device__ __forceinline__ uint4 decode_group(uint32_t books, const uint32_t (&c
     if constexpr (MB == 1 && BDT == AQ_F16) {
         return c0;   // one fp16 codeword: widening to fp32 and rounding back is exact
     } else {
-        float2 a0 = widen2f<BDT>(c0.x), a1 = widen2f<BDT>(c0.y), a2 = widen2f<BDT>(c0.z),
-               a3 = widen2f<BDT>(c0.w);
+        // one mixed-type add per element (16-bit operand into the fp32 sum); -0 + v = v
+        // exactly, so the first book is widened by the same instruction
+        float a[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) a[e] = -0.0f;
+        add_widen2<BDT>(c0.x, a[0], a[1]);
+        add_widen2<BDT>(c0.y, a[2], a[3]);
+        add_widen2<BDT>(c0.z, a[4], a[5]);
+        add_widen2<BDT>(c0.w, a[6], a[7]);
 #pragma unroll
         for (int k = 1; k < MB; ++k) {
             const uint4 ck = lds128(books + ((uint32_t)k << 12) + (code[k] << 4));
-            a0 = add2(a0, widen2f<BDT>(ck.x));
-            a1 = add2(a1, widen2f<BDT>(ck.y));
-            a2 = add2(a2, widen2f<BDT>(ck.z));
-            a3 = add2(a3, widen2f<BDT>(ck.w));
+            add_widen2<BDT>(ck.x, a[0], a[1]);
+            add_widen2<BDT>(ck.y, a[2], a[3]);
+            add_widen2<BDT>(ck.z, a[4], a[5]);
+            add_widen2<BDT>(ck.w, a[6], a[7]);
         }
-        return make_uint4(f16x2(a0), f16x2(a1), f16x2(a2), f16x2(a3));
+        return make_uint4(f16x2(make_float2(a[0], a[1])), f16x2(make_float2(a[2], a[3])),
+                          f16x2(make_float2(a[4], a[5])), f16x2(make_float2(a[6], a[7])));
     }
 }
 
