@@ -2,27 +2,32 @@
 // (Sec. 3.2 group sums, restricted to the first m codebooks as in Sec. 5; Y = W X of Sec. 2.2).
 //
 // Work split (split-K): the input dimension is cut into slices of 32 groups (256 inputs).
-// A work item is (slice, 32-row block) for the direct kernel and (slice, codebook, 32-row
-// block) for the table-lookup kernel. Each item reads its code planes once and writes one
-// fp32 partial per (row, token). A second, small kernel (splitk_reduce, launched right behind
-// with programmatic dependent launch, so its CTAs are already resident when the product
-// finishes) sums each row's partials in a fixed order (deterministic), scales the row and
-// stores y, with the rows spread evenly over the GPU.
+// A work item is (slice, 32-row block) for the direct and tensor-core kernels and (slice,
+// codebook, 32-row block) for the table-lookup kernel. Each item reads its code planes once
+// and writes one fp32 partial per (row, token). A second, small kernel (splitk_reduce,
+// launched right behind with programmatic dependent launch, so its CTAs are already resident
+// when the product finishes) sums each row's partials in a fixed order (deterministic),
+// scales the row and stores y, with the rows spread evenly over the GPU.
 //
-// Two product kernels:
-//  * gemv_lut (B = 8, one token, m <= 8). By linearity, x_g . (sum_k C_k[b_k]) =
-//    sum_k T_k[g][b_k] with T_k[g][j] = x_g . C_k[j]. A persistent CTA (one per SM) walks a
-//    contiguous range of work items; for each (slice, book) it builds that book's T for the
-//    32 groups in shared memory (32 KiB), then every code byte costs one shared-memory lookup
-//    and one fp32 add. Lane L owns row 32*rb+L; because each row's 32 codes are stored
-//    rotated by the row index, at step p all 32 lanes look up 32 different groups, i.e. 32
-//    different banks, so the lookups are conflict-free and no cross-lane reduction is needed.
-//    One producer warp streams the code planes into a shared-memory ring with TMA bulk copies
-//    (the CTA's rows of a slice are contiguous in every plane), overlapping HBM reads with
-//    the table build and the lookups of the sixteen consumer warps.
-//  * gemv_direct (any B, 1..16 tokens). Decode each group in fp32 (sum of m codewords), then
-//    multiply by the tokens' 8 activations. Lane L owns row 32*rb+L and walks the 32 groups
-//    of the slice in a common order, so the activation loads are warp-uniform broadcasts.
+// Three product kernels, chosen by batch, code width and prefix:
+//  * gemv_lut (B = 8; 1 token with m <= 8, or 2..4 tokens with m <= 4). By linearity,
+//    x_g . (sum_k C_k[b_k]) = sum_k T_k[g][b_k] with T_k[g][j] = x_g . C_k[j]. A persistent
+//    CTA (one per SM) walks a contiguous range of work items; for each (slice, book) it builds
+//    that book's T for the 32 groups in shared memory (32 KiB per token), then every code
+//    byte costs one shared-memory lookup and one fp32 add per token. Lane L owns row
+//    32*rb+L; because each row's 32 codes are stored rotated by the row index, at step p all
+//    32 lanes look up 32 different groups, i.e. 32 different banks, so the lookups are
+//    conflict-free and no cross-lane reduction is needed. One producer warp streams the code
+//    planes into a shared-memory ring with TMA bulk copies (the CTA's rows of a slice are
+//    contiguous in every plane), overlapping HBM reads with the table build and the lookups
+//    of the sixteen consumer warps.
+//  * gemv_mma (B = 8, 5..16 tokens, m <= 4). The decoded group (fp32 sum of the m
+//    codewords, rounded once to tf32) is an A fragment of a tensor-core multiply with 8 or
+//    16 tokens of activations (mma.sync m16n8k8).
+//  * gemv_direct (any other case: 16-bit codes, larger m). Decode each group in fp32 (sum of
+//    m codewords), then multiply by the tokens' 8 activations. Lane L owns row 32*rb+L and
+//    walks the 32 groups of the slice in a common order, so the activation loads are
+//    warp-uniform broadcasts.
 #include <map>
 #include <mutex>
 #include <tuple>
