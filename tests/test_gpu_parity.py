@@ -183,10 +183,11 @@ def test_gemv_static_weights_flag_gives_same_result():
     layer = _layer(2000, 4096, 4, 8, "f16", seed=12)
     lin = AQLinear.from_layer(layer)
     assert lin.layout.flags == aq.AQ_LAYOUT_STATIC_WEIGHTS
-    x = x_to_device(workloads.make_x(1, 4096, "f16", seed=5), "f16")
-    for m in (1, 3, 4):
-        a = lin.gemv(x, m).clone()
-        lin.layout.flags = 0
-        b = lin.gemv(x, m).clone()
-        lin.layout.flags = aq.AQ_LAYOUT_STATIC_WEIGHTS
-        assert torch.equal(a, b), m
+    for batch in (1, 3, 8):     # table lookups for 1 and 3 tokens, tensor cores for 8
+        x = x_to_device(workloads.make_x(batch, 4096, "f16", seed=5), "f16")
+        for m in (1, 3, 4):
+            a = lin.gemv(x, m).clone()
+            lin.layout.flags = 0
+            b = lin.gemv(x, m).clone()
+            lin.layout.flags = aq.AQ_LAYOUT_STATIC_WEIGHTS
+            assert torch.equal(a, b), (batch, m)
