@@ -137,6 +137,26 @@ aq_status aq_gemv(const aq_layout* layout, int m, const void* planes, const void
                   const void* scales, const void* x, int x_dtype, int batch, void* y,
                   int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
 
+/* ---------------------------------------------------------------- GEMV refinement (prefix m-1 -> m)
+ * y = y_prev + x * (s o C_{m-1}[b_{m-1}])^T: the increment that raises a product computed with
+ * the first m-1 codebooks to the product with the first m (the successive reconstruction of
+ * Sec. 4, y^(k) = y^(k-1) + increment, applied to the codebook prefixes of Sec. 5; by the
+ * linearity of the product in the books, y_prev = the prefix-(m-1) product gives the prefix-m
+ * product). Only plane m-1 of the codes and codebook m-1 are read, so raising the precision
+ * of a result at run time costs one plane of HBM traffic.
+ *   m       : 1 <= m <= num_books; the book whose increment is added is m-1
+ *   planes  : device, at least the first m planes (only plane m-1 is read)
+ *   y_prev  : device, [batch][d_out] of y_dtype, 16-byte aligned, or NULL (read as zero: y is
+ *             then the increment alone). It may be y itself (in-place refinement).
+ *   all other arguments, the workspace size and the error behaviour are those of aq_gemv.
+ * Each element is y_prev + (the increment in fp32), rounded once to y_dtype; with
+ * y_dtype = AQ_F32 a chain of refinements from m = 1 (y_prev = NULL) to m stays within the
+ * aq_gemv accuracy bounds of the prefix-m product. */
+aq_status aq_gemv_refine(const aq_layout* layout, int m, const void* planes, const void* books,
+                         const void* scales, const void* x, int x_dtype, int batch,
+                         const void* y_prev, void* y, int y_dtype, void* workspace,
+                         size_t workspace_bytes, void* stream);
+
 /* ---------------------------------------------------------------- GEMV without a workspace
  * (This entry point has no counterpart in the paper.) The GEMV of aq_gemv for callers that
  * cannot allocate device memory when they run a layer, and so cannot pass a workspace: for

@@ -23,7 +23,8 @@ TORCH_DTYPES = {AQ_F16: torch.float16, AQ_BF16: torch.bfloat16, AQ_F32: torch.fl
 # Every entry point that include/aq.h declares.
 EXPORTS = ["aq_abi_version", "aq_status_string", "aq_last_error", "aq_plane_bytes", "aq_packed_bytes", "aq_pack",
            "aq_decode", "aq_gemv_workspace_bytes", "aq_gemv", "aq_gemm_workspace_bytes",
-           "aq_gemm", "aq_workspace_init", "aq_workspace_status", "aq_gemv_static_scratch"]
+           "aq_gemm", "aq_workspace_init", "aq_workspace_status", "aq_gemv_static_scratch",
+           "aq_gemv_refine"]
 
 
 class AQError(RuntimeError):
@@ -75,6 +76,7 @@ def lib():
             "aq_workspace_init": (i32, [vp, sz, vp]),
             "aq_workspace_status": (i32, [vp, vp]),
             "aq_gemv_static_scratch": (i32, [lp, i32, vp, vp, vp, vp, i32, i32, vp, i32, vp]),
+            "aq_gemv_refine": (i32, [lp, i32, vp, vp, vp, vp, i32, i32, vp, vp, i32, vp, sz, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -152,6 +154,17 @@ def aq_gemv(layout, m, planes, books, scales, x, x_dtype, batch, y, y_dtype, wor
     _check(lib().aq_gemv(ctypes.byref(layout), m, _ptr(planes), _ptr(books), _ptr(scales),
                          _ptr(x), x_dtype, batch, _ptr(y), y_dtype, _ptr(workspace),
                          workspace_bytes, _stream(stream)), "aq_gemv")
+
+
+def aq_gemv_refine(layout, m, planes, books, scales, x, x_dtype, batch, y_prev, y, y_dtype,
+                   workspace, workspace_bytes=None, stream=None):
+    """y = y_prev + x (s o C_{m-1}[b_{m-1}])^T (y_prev None: zero); reads plane m-1 only."""
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    _check(lib().aq_gemv_refine(ctypes.byref(layout), m, _ptr(planes), _ptr(books), _ptr(scales),
+                                _ptr(x), x_dtype, batch, _ptr(y_prev), _ptr(y), y_dtype,
+                                _ptr(workspace), workspace_bytes, _stream(stream)),
+           "aq_gemv_refine")
 
 
 def aq_gemm(layout, m, planes, books, scales, x, x_dtype, tokens, y, y_dtype, workspace,

@@ -183,6 +183,31 @@ aq_status aq_gemv(const aq_layout* layout, int m, const void* planes, const void
                            as_stream(stream));
 }
 
+aq_status aq_gemv_refine(const aq_layout* layout, int m, const void* planes, const void* books,
+                         const void* scales, const void* x, int x_dtype, int batch,
+                         const void* y_prev, void* y, int y_dtype, void* workspace,
+                         size_t workspace_bytes, void* stream) {
+    Dims d;
+    aq_status st = aq::make_dims(layout, &d);
+    if (st != AQ_OK) return st;
+    if ((st = check_m(d, m)) != AQ_OK) return st;
+    if (batch < 0 || batch > 16) return AQ_ERR_INVALID_ARG;
+    if (x_dtype != AQ_F16 && x_dtype != AQ_BF16) return AQ_ERR_INVALID_ARG;
+    if (y_dtype != AQ_F16 && y_dtype != AQ_BF16 && y_dtype != AQ_F32) return AQ_ERR_INVALID_ARG;
+    if (batch == 0 || d.out == 0) return AQ_OK;
+    if ((st = check_ptrs({planes, books, scales, x, y})) != AQ_OK) return st;
+    if (y_prev && !aligned16(y_prev)) return AQ_ERR_ALIGNMENT;
+    if (!workspace || workspace_bytes < gemv_ws_bytes(d, batch)) return AQ_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;
+    // The increment of book m-1 is a one-book product: plane m-1 and book m-1 are the whole
+    // code planes and codebooks of a one-book layout (the partial planes it needs fit in the
+    // workspace of the full layout).
+    const char* plane1 = (const char*)planes + (size_t)(m - 1) * d.plane_bytes;
+    const char* book1 = (const char*)books + (size_t)(m - 1) * ((size_t)1 << d.B) * d.G * 2;
+    return aq::launch_gemv(d, 1, plane1, book1, scales, x, x_dtype, batch, y, y_dtype, workspace,
+                           as_stream(stream), y_prev);
+}
+
 size_t aq_gemm_workspace_bytes(const aq_layout* layout, int tokens) {
     Dims d;
     if (aq::make_dims(layout, &d) != AQ_OK || tokens < 0) return 0;

@@ -58,9 +58,10 @@ inline aq_status cuda_ok(cudaError_t e, const char* what) {
 aq_status launch_pack(const Dims& d, const void* codes, void* planes, cudaStream_t st);
 aq_status launch_decode(const Dims& d, int m, const void* planes, const void* books,
                         const void* scales, void* w, cudaStream_t st);
+// y_prev (optional): added to the product (y = y_prev + product), read in y's type.
 aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* books,
                       const void* scales, const void* x, int x_dt, int batch, void* y,
-                      int y_dt, void* ws, cudaStream_t st);
+                      int y_dt, void* ws, cudaStream_t st, const void* y_prev = nullptr);
 aq_status launch_gemm(const Dims& d, int m, const void* planes, const void* books,
                       const void* scales, const void* x, int x_dt, int tokens, void* y, int y_dt,
                       void* ws, cudaStream_t st);

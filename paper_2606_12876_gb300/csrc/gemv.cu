@@ -647,13 +647,14 @@ gemv_mma_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
 // split its planes: warp j of the group adds planes j, j + wpr, ... in order (up to sixteen
 // loads in flight, coalesced over the rows), then the group's first warp adds the wpr sums in
 // order, so the summation order is fixed. With static weights the row scales are read before
-// waiting for the product kernel. The kernel is kept small: it runs once per CTA, so its
-// instructions are fetched cold.
+// waiting for the product kernel. With y_prev (a refinement, Sec. 4 successive
+// reconstruction) the scaled sum is added to y_prev[t][r], read in y's type (y_prev may be y).
+// The kernel is kept small: it runs once per CTA, so its instructions are fetched cold.
 template <int SDT>
 __global__ void __launch_bounds__(256)
 splitk_reduce_kernel(const float* __restrict__ partials, const uint16_t* __restrict__ scales,
                      void* y, int y_dt, int out, int rows_pad, int P, int batch, int wpr,
-                     int static_weights) {
+                     int static_weights, const void* y_prev) {
     __shared__ float red[8][32];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     const int j = w & (wpr - 1), rg = w - j;     // rg: first warp of the row group
@@ -684,8 +685,11 @@ splitk_reduce_kernel(const float* __restrict__ partials, const uint16_t* __restr
             for (int i = 1; i < wpr; ++i) sum += red[w + i][lane];
     }
     if (lead) {
-        const float v = sum * bits_to_f32<SDT>(sc);
+        float v = sum * bits_to_f32<SDT>(sc);
         const size_t yi = (size_t)t * out + r;
+        if (y_prev)
+            v = (y_dt == AQ_F32 ? ((const float*)y_prev)[yi]
+                                : bits_to_f32_rt(((const uint16_t*)y_prev)[yi], y_dt)) + v;
         if (y_dt == AQ_F32) ((float*)y)[yi] = v;
         else ((uint16_t*)y)[yi] = y_dt == AQ_F16 ? f32_to_bits<AQ_F16>(v) : f32_to_bits<AQ_BF16>(v);
     }
@@ -932,7 +936,8 @@ static aq_status launch_product(const Dims& d, int m, const void* planes, const 
 // P partial planes per token: one per (slice, book) for the LUT kernel, one per slice for the
 // direct kernel.
 template <int SDT>
-static aq_status launch_reduce(const Dims& d, int P, const GemvArgs& a, cudaStream_t st) {
+static aq_status launch_reduce(const Dims& d, int P, const GemvArgs& a, const void* y_prev,
+                               cudaStream_t st) {
     int occ = 0;
     if (aq_status e = prepare(splitk_reduce_kernel<SDT>, 0, 256, 0, &occ); e != AQ_OK) return e;
     // Warps per 32-row group: one while a warp's sixteen loads cover the planes (no shared
@@ -943,12 +948,12 @@ static aq_status launch_reduce(const Dims& d, int P, const GemvArgs& a, cudaStre
     return launch_pdl(splitk_reduce_kernel<SDT>, dim3((d.out + rows_per_cta - 1) / rows_per_cta, a.batch),
                       dim3(256), 0, st, (const float*)a.partials, (const uint16_t*)a.scales, a.y,
                       a.y_dt, d.out, d.rows_pad, P, a.batch, wpr,
-                      (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0);
+                      (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0, y_prev);
 }
 
 aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* books,
                       const void* scales, const void* x, int x_dt, int batch, void* y,
-                      int y_dt, void* ws, cudaStream_t st) {
+                      int y_dt, void* ws, cudaStream_t st, const void* y_prev) {
     if (d.out == 0 || batch == 0) return AQ_OK;
     if (aq_status e = launch_product(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
         e != AQ_OK)
@@ -956,8 +961,8 @@ aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* book
     GemvArgs a{planes, books, scales, x, x_dt, batch, y, y_dt,
                (float*)((char*)ws + ws_partial_offset(d)), (unsigned int*)ws};
     const int P = uses_lut(d, m, batch) ? d.S * m : d.S;
-    return d.scale_dt == AQ_BF16 ? launch_reduce<AQ_BF16>(d, P, a, st)
-                                 : launch_reduce<AQ_F16>(d, P, a, st);
+    return d.scale_dt == AQ_BF16 ? launch_reduce<AQ_BF16>(d, P, a, y_prev, st)
+                                 : launch_reduce<AQ_F16>(d, P, a, y_prev, st);
 }
 
 }  // namespace aq

@@ -9,7 +9,8 @@ import torch
 
 from . import (AQ_BF16, AQ_F16, AQ_F32, AQ_LAYOUT_STATIC_WEIGHTS, DTYPES, TORCH_DTYPES, Layout,
                aq_decode, aq_gemm,
-               aq_gemv, aq_pack, gemm_workspace_bytes, gemv_workspace_bytes, packed_bytes,
+               aq_gemv, aq_gemv_refine, aq_pack, gemm_workspace_bytes, gemv_workspace_bytes,
+               packed_bytes,
                workspace, _stream)
 
 
@@ -93,6 +94,20 @@ class AQLinear:
             y = torch.empty(batch, self.out, dtype=TORCH_DTYPES[yd], device=self.device)
         ws = self._workspace("gemv", batch)
         aq_gemv(self.layout, m, self.planes, self.books, self.scales, x, xd, batch, y, yd, ws)
+        return y
+
+    def refine(self, x, m, y_prev, y=None):
+        """y = y_prev + x (s o C_{m-1}[b_{m-1}])^T: raises a prefix-(m-1) result to prefix m,
+        reading plane m-1 only (y_prev None: the increment alone). y has y_prev's dtype
+        (fp32 by default when y_prev is None); y may be y_prev (in place)."""
+        xd = _dtype_code(x.dtype)
+        batch = x.shape[0]
+        yd = _dtype_code(y_prev.dtype) if y_prev is not None else AQ_F32
+        if y is None:
+            y = torch.empty(batch, self.out, dtype=TORCH_DTYPES[yd], device=self.device)
+        ws = self._workspace("gemv", batch)
+        aq_gemv_refine(self.layout, m, self.planes, self.books, self.scales, x, xd, batch, y_prev,
+                       y, yd, ws)
         return y
 
     def gemm(self, x, m, y=None, y_dtype=None):
