@@ -341,12 +341,28 @@ def own_arm(args):
         del g
 
 
+    # Refinement step (aq_gemv_refine): the increment from prefix m-1 to m, reading plane m-1
+    # only, fp32 output added to the previous fp32 result; same graph timing.
+    ys32 = {m: torch.zeros(1, out, dtype=torch.float32, device=dev) for m in (0,) + ms}
+    refine_us = {}
+    for m in ms:
+        prev = ys32[m - 1] if m > 1 else None
+        g = capture(lambda i, m=m, prev=prev: aq.aq_gemv_refine(
+            L, m, copies[i % ncopies], lin.books, lin.scales, x, aq.AQ_F16, 1, prev, ys32[m],
+            aq.AQ_F32, ws), args.steps)
+        g.replay()
+        refine_us[m] = time_graph(g) * 1e3 / args.steps
+        del g
+    refine_bytes = layer_bytes(out, inp, 1, ysize=4) + 4 * out   # one plane; y_prev read too
+
     per_m = []
     for m in ms:
         us = per_m_us[m]
         gbs = bytes_m[m] / (us * 1e-6) / 1e9
         per_m.append({"m": m, "bits_per_weight": m, "us": round(us, 3), "GB_s": round(gbs, 1),
-                      "frac_hbm": round(gbs / hbm_peak, 4), "bytes": bytes_m[m]})
+                      "frac_hbm": round(gbs / hbm_peak, 4), "bytes": bytes_m[m],
+                      "refine_from_m_minus_1_us": round(refine_us[m], 3),
+                      "refine_GB_s": round(refine_bytes / (refine_us[m] * 1e-6) / 1e9, 1)})
     dom = max(per_m, key=lambda r: r["us"])
 
     # end to end through the public API: pinned host x -> device, 4 GEMVs, y -> pinned host
