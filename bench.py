@@ -39,6 +39,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-gemm", action="store_true")
+    ap.add_argument("--no-loading", action="store_true",
+                    help="skip the prefix-store loading measurement")
     ap.add_argument("--gemm-tokens", type=int, default=4096,
                     help="tokens of the prefill GEMM case (smaller values: profiling runs)")
     ap.add_argument("--skip-gemv", action="store_true",
@@ -236,6 +238,61 @@ def measure_gemm(dev, stream, peaks, reps=5, tokens=4096):
             "peak_TFLOP_s": peak, "peak_source": "measured" if "bf16_tflops" in peaks else "fallback"}
 
 
+def measure_loading(lin, dev, stream, ms, reps=7):
+    """Dynamic loading through a prefix store (aq_store_*): the layer's packed form in pinned
+    host memory, device memory for the resident prefix only. Raising the prefix from m-1 to m
+    maps memory for plane m-1 and copies that plane and codebook m-1 from the host; lowering
+    back synchronises the device and unmaps it. Host wall time (median over reps) around the
+    call and a synchronisation of the stream; the plain host->device copy of the same bytes
+    (CUDA events) is timed beside it."""
+    import time
+
+    import torch
+    from paper_2606_12876_gb300.linear import AQLinear
+
+    host = lin.to_host()
+    pb = host["planes"].numel() // lin.M
+    raise_us, lower_us = {}, {}
+    with torch.cuda.stream(stream):
+        dyn = AQLinear.from_host(host, 0, device=dev)
+        for m in ms:
+            up, down = [], []
+            for _ in range(reps):
+                dyn.set_prefix(m - 1)
+                torch.cuda.synchronize(dev)
+                t0 = time.perf_counter()
+                dyn.set_prefix(m)
+                stream.synchronize()
+                up.append(time.perf_counter() - t0)
+                t0 = time.perf_counter()
+                dyn.set_prefix(m - 1)
+                down.append(time.perf_counter() - t0)
+            raise_us[m] = sorted(up)[reps // 2] * 1e6
+            lower_us[m] = sorted(down)[reps // 2] * 1e6
+        dyn.set_prefix(max(ms))
+        x = torch.randn(1, lin.inp, device=dev, dtype=torch.float16)
+        same = bool(torch.equal(dyn.gemv(x, max(ms)), lin.gemv(x, max(ms))))
+        resident = dyn.device_bytes()
+        dyn.close()
+        dst = torch.empty(pb, dtype=torch.uint8, device=dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        copy = []
+        for _ in range(reps):
+            e0.record()
+            dst.copy_(host["planes"][:pb], non_blocking=True)
+            e1.record()
+            e1.synchronize()
+            copy.append(e0.elapsed_time(e1) * 1e3)
+    copy_us = sorted(copy)[reps // 2]
+    return {"store": "aq_store_* (virtual address range for all M planes, memory mapped per prefix)",
+            "source": "pinned host memory", "plane_bytes": pb,
+            "raise_to_m_us": {m: round(raise_us[m], 1) for m in ms},
+            "lower_from_m_us": {m: round(lower_us[m], 1) for m in ms},
+            "h2d_copy_one_plane_us": round(copy_us, 1),
+            "h2d_GB_s": round(pb / (copy_us * 1e-6) / 1e9, 1),
+            "device_bytes_at_m4": resident, "matches_full_layer": same}
+
+
 def own_arm(args):
     import numpy as np
     import torch
@@ -394,6 +451,7 @@ def own_arm(args):
                "api": "paper_2606_12876_gb300.aq_gemv (ctypes -> libaq.so), eager"}
 
     gemm = None if args.no_gemm else measure_gemm(dev, stream, peaks, tokens=args.gemm_tokens)
+    loading = measure_loading(lin, dev, stream, ms) if rank == 0 and not args.no_loading else None
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -416,6 +474,7 @@ def own_arm(args):
                            ncopies, ncopies, pbytes / 1e6, l2 / 1e6)},
             "per_m": per_m,
             "gemm": gemm,
+            "dynamic_loading": loading,
             "roofline": {
                 "bound": "hbm", "kernel": "gemv_lut_kernel m=%d" % dom["m"],
                 "achieved": dom["GB_s"], "peak": hbm_peak, "unit": "GB/s",

@@ -12,8 +12,9 @@
  *     y[t, o]         = sum_i x[t, i] * W_m[o, i]                     (Sec. 2.2, Y = W X)
  *
  * Conventions that hold for every entry point:
- *   - All data pointers are DEVICE pointers, 16-byte aligned, owned by the caller. The
- *     library allocates and frees nothing and keeps no pointer after a call returns.
+ *   - All data pointers are DEVICE pointers, 16-byte aligned, owned by the caller. Apart
+ *     from the aq_store_* entry points (dynamic loading, below), the library allocates and
+ *     frees nothing and keeps no pointer after a call returns.
  *   - stream is a cudaStream_t passed as void* (NULL = the legacy default stream). All work
  *     is enqueued asynchronously on it; no call synchronises unless its comment says so.
  *   - Argument errors are detected on the host before anything is launched; the call then
@@ -196,6 +197,65 @@ size_t aq_gemm_workspace_bytes(const aq_layout* layout, int tokens);
 aq_status aq_gemm(const aq_layout* layout, int m, const void* planes, const void* books,
                   const void* scales, const void* x, int x_dtype, int tokens, void* y,
                   int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
+
+/* ---------------------------------------------------------------- dynamic loading
+ * Device storage for one layer that holds only a prefix of its codebooks. One stored model
+ * serves every bit width, and each deployment keeps as many codebooks on the device as its
+ * memory or latency budget allows, loading more (or dropping some) at run time (Sec. 1 and
+ * Sec. 5). Since the planes are codebook-major, a prefix is one contiguous byte range.
+ * A store reserves device address space for the whole layer once and backs with physical
+ * memory only the scales, the codebooks and the planes of the resident prefix (in whole
+ * allocation granules, the device's minimum for virtual-memory mappings, 2 MiB on current
+ * GPUs). Raising the prefix maps memory behind the resident planes and copies the new planes
+ * in; lowering it releases the memory of the dropped planes. The device addresses never
+ * move: pointers taken from a store stay valid for its life and may be passed to every
+ * compute entry point with any m up to the resident prefix. A call with a larger m would read
+ * unmapped addresses: the caller must not make one. These entry points allocate and free
+ * device memory; a store is used by one host thread at a time. */
+typedef struct aq_store aq_store;   /* opaque */
+
+/* Create an empty store (prefix 0) for layout on the current device: reserves the address
+ * range and maps memory for the scales and all M codebooks (2^B*16 bytes per codebook), none
+ * for planes. Synchronous.
+ *   store : receives the handle (NULL on failure).
+ * Errors: AQ_ERR_INVALID_ARG / AQ_ERR_UNSUPPORTED (null store or a bad layout, as aq_pack),
+ * AQ_ERR_CUDA (a runtime or driver call failed, e.g. out of memory; see aq_last_error). */
+aq_status aq_store_create(const aq_layout* layout, aq_store** store);
+
+/* Make planes 0..m-1 and codebooks 0..m-1 resident, 0 <= m <= M; m0 = the current prefix.
+ * Raising (m > m0) maps memory for planes m0..m-1, then enqueues on stream the copies of
+ * planes m0..m-1 and codebooks m0..m-1, and of the scales when m0 = 0, from:
+ *   src_planes : the packed planes of all M codebooks, aq_packed_bytes(layout, M) bytes laid
+ *                out as aq_pack writes them (only planes m0..m-1 are read)
+ *   src_books  : [M][2^B][8] of book_dtype (only codebooks m0..m-1 are read)
+ *   src_scales : [d_out] of scale_dtype (read only when m0 = 0)
+ * Each may be host memory (pinned, for a copy that runs asynchronously) or device memory, and
+ * must stay valid until the copies have run. Work that reads the new prefix must be ordered
+ * after them: enqueue it on stream, or make its stream wait for an event recorded there.
+ * Lowering (m < m0) synchronises the device, so that no kernel can still be reading the
+ * dropped planes, then unmaps the memory that only planes m..m0-1 use (the granule that plane
+ * m-1 shares with plane m stays). The src pointers are not used and may be NULL. m = m0 does
+ * nothing.
+ * Errors: AQ_ERR_INVALID_ARG (null store, m outside 0..M, a NULL src pointer that a raise
+ * needs), AQ_ERR_CUDA (mapping or copy failed; the prefix then stays m0). */
+aq_status aq_store_set_prefix(aq_store* store, int m, const void* src_planes,
+                              const void* src_books, const void* src_scales, void* stream);
+
+/* The resident prefix (0 for a NULL store). */
+int aq_store_prefix(const aq_store* store);
+/* Device addresses of the store's planes ([M planes], plane k at k*aq_plane_bytes), codebooks
+ * ([M][2^B][8]) and scales ([d_out]); fixed for the store's life, 16-byte aligned, readable
+ * for the resident prefix only. NULL for a NULL store. */
+void* aq_store_planes(const aq_store* store);
+void* aq_store_books(const aq_store* store);
+void* aq_store_scales(const aq_store* store);
+/* Bytes of device memory the store holds mapped (0 for a NULL store). */
+size_t aq_store_device_bytes(const aq_store* store);
+
+/* Synchronise the device, release the store's memory and address range, free the handle.
+ * NULL: nothing (AQ_OK). Errors: AQ_ERR_CUDA if the synchronisation reported an error (the
+ * store is released all the same). */
+aq_status aq_store_destroy(aq_store* store);
 
 /* ---------------------------------------------------------------- workspace helpers
  * aq_workspace_init: enqueue a zero-fill of bytes at workspace (cudaMemsetAsync).

@@ -24,7 +24,9 @@ TORCH_DTYPES = {AQ_F16: torch.float16, AQ_BF16: torch.bfloat16, AQ_F32: torch.fl
 EXPORTS = ["aq_abi_version", "aq_status_string", "aq_last_error", "aq_plane_bytes", "aq_packed_bytes", "aq_pack",
            "aq_decode", "aq_gemv_workspace_bytes", "aq_gemv", "aq_gemm_workspace_bytes",
            "aq_gemm", "aq_workspace_init", "aq_workspace_status", "aq_gemv_static_scratch",
-           "aq_gemv_refine"]
+           "aq_gemv_refine", "aq_store_create", "aq_store_set_prefix", "aq_store_prefix",
+           "aq_store_planes", "aq_store_books", "aq_store_scales", "aq_store_device_bytes",
+           "aq_store_destroy"]
 
 
 class AQError(RuntimeError):
@@ -77,6 +79,14 @@ def lib():
             "aq_workspace_status": (i32, [vp, vp]),
             "aq_gemv_static_scratch": (i32, [lp, i32, vp, vp, vp, vp, i32, i32, vp, i32, vp]),
             "aq_gemv_refine": (i32, [lp, i32, vp, vp, vp, vp, i32, i32, vp, vp, i32, vp, sz, vp]),
+            "aq_store_create": (i32, [lp, ctypes.POINTER(vp)]),
+            "aq_store_set_prefix": (i32, [vp, i32, vp, vp, vp, vp]),
+            "aq_store_prefix": (i32, [vp]),
+            "aq_store_planes": (vp, [vp]),
+            "aq_store_books": (vp, [vp]),
+            "aq_store_scales": (vp, [vp]),
+            "aq_store_device_bytes": (sz, [vp]),
+            "aq_store_destroy": (i32, [vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -182,6 +192,44 @@ def aq_gemv_static_scratch(layout, m, planes, books, scales, x, x_dtype, batch, 
     _check(lib().aq_gemv_static_scratch(ctypes.byref(layout), m, _ptr(planes), _ptr(books),
                                         _ptr(scales), _ptr(x), x_dtype, batch, _ptr(y), y_dtype,
                                         _stream(stream)), "aq_gemv_static_scratch")
+
+
+def aq_store_create(layout):
+    """An empty prefix store for layout on the current device (an opaque handle, an int)."""
+    h = ctypes.c_void_p()
+    _check(lib().aq_store_create(ctypes.byref(layout), ctypes.byref(h)), "aq_store_create")
+    return h.value
+
+
+def aq_store_set_prefix(store, m, src_planes, src_books, src_scales, stream=None):
+    """Make planes/codebooks 0..m-1 resident (copies enqueued on the stream when raising; the
+    device is synchronised when lowering). Sources: tensors or addresses, host or device."""
+    _check(lib().aq_store_set_prefix(store, m, _ptr(src_planes), _ptr(src_books),
+                                     _ptr(src_scales), _stream(stream)), "aq_store_set_prefix")
+
+
+def aq_store_prefix(store):
+    return lib().aq_store_prefix(store)
+
+
+def aq_store_planes(store):
+    return lib().aq_store_planes(store)
+
+
+def aq_store_books(store):
+    return lib().aq_store_books(store)
+
+
+def aq_store_scales(store):
+    return lib().aq_store_scales(store)
+
+
+def aq_store_device_bytes(store):
+    return lib().aq_store_device_bytes(store)
+
+
+def aq_store_destroy(store):
+    _check(lib().aq_store_destroy(store), "aq_store_destroy")
 
 
 def aq_workspace_init(workspace, nbytes=None, stream=None):

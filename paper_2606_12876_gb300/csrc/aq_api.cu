@@ -49,6 +49,12 @@ aq_status cuda_fail(cudaError_t e, const char* what) {
     return AQ_ERR_CUDA;
 }
 
+aq_status driver_fail(int result, const char* name, const char* what) {
+    snprintf(g_last_error, sizeof(g_last_error), "%s: CUresult %d (%s)", what, result,
+             name ? name : "unknown");
+    return AQ_ERR_CUDA;
+}
+
 aq_status device_info(DeviceInfo* info) {
     static std::mutex mu;
     static DeviceInfo cache[64];

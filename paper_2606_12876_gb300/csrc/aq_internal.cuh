@@ -53,6 +53,9 @@ aq_status cuda_fail(cudaError_t e, const char* what);
 inline aq_status cuda_ok(cudaError_t e, const char* what) {
     return e == cudaSuccess ? AQ_OK : cuda_fail(e, what);
 }
+// Records a failed CUDA driver call (its CUresult code and, when known, name) for
+// aq_last_error and returns AQ_ERR_CUDA.
+aq_status driver_fail(int result, const char* name, const char* what);
 
 // ---- launchers (each returns AQ_OK or AQ_ERR_CUDA; arguments are already validated) ----
 aq_status launch_pack(const Dims& d, const void* codes, void* planes, cudaStream_t st);

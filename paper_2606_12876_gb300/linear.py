@@ -1,17 +1,26 @@
 """AQLinear: one additive-codebook linear layer resident on the GPU, served at any prefix m.
 
 The layer is stored once (AQLMFormat(C, b, s) of Alg. 1: M codebooks, codes, per-row scales)
-and evaluated with the first m codebooks chosen per call (Sec. 5). Device memory comes from
-torch; all work is done by libaq through the binding in this package.
+and evaluated with the first m codebooks chosen per call (Sec. 5). A layer either holds all M
+codebooks in torch device memory, or (from_host) holds only a resident prefix in a libaq store
+that loads further codebooks from host memory at run time. All work is done by libaq through
+the binding in this package.
 """
+import weakref
+
 import numpy as np
 import torch
 
 from . import (AQ_BF16, AQ_F16, AQ_F32, AQ_LAYOUT_STATIC_WEIGHTS, DTYPES, TORCH_DTYPES, Layout,
                aq_decode, aq_gemm,
-               aq_gemv, aq_gemv_refine, aq_pack, gemm_workspace_bytes, gemv_workspace_bytes,
-               packed_bytes,
+               aq_gemv, aq_gemv_refine, aq_pack, aq_store_books, aq_store_create,
+               aq_store_device_bytes, aq_store_planes, aq_store_scales, aq_store_set_prefix,
+               gemm_workspace_bytes, gemv_workspace_bytes, lib, packed_bytes,
                workspace, _stream)
+
+
+def _destroy_store(store):
+    lib().aq_store_destroy(store)
 
 
 def _u16_to_device(a, device):
@@ -48,12 +57,78 @@ class AQLinear:
         self.layout.flags = AQ_LAYOUT_STATIC_WEIGHTS
         self.codes = codes_t if keep_codes else None
         self._ws = {}
+        self.store, self.resident = None, M
 
     @classmethod
     def from_layer(cls, layer, device="cuda", keep_codes=False):
         """From a workloads.make_layer() dict."""
         return cls(layer["books"], layer["codes"], layer["scales"], layer["book_dtype"],
                    layer["scale_dtype"], device, keep_codes)
+
+    def to_host(self, pin=True):
+        """The packed layer in host memory, the form a deployment keeps outside the GPU: a dict
+        of the layout, the planes of all M codebooks (uint8), the codebooks and the scales
+        (int16 bit patterns), and the dtype names; page-locked when pin is true, so that
+        loading from it runs as asynchronous copies."""
+        if self.store is not None:
+            raise TypeError("to_host needs a layer that holds all its codebooks")
+        t = lambda a: a.cpu().pin_memory() if pin else a.cpu()
+        layout = Layout(*[getattr(self.layout, f) for f, _ in Layout._fields_])
+        return dict(layout=layout, planes=t(self.planes), books=t(self.books),
+                    scales=t(self.scales), book_dtype=self.book_dtype,
+                    scale_dtype=self.scale_dtype)
+
+    @classmethod
+    def from_host(cls, host, m, device="cuda"):
+        """A layer whose device memory holds only the first m codebooks (a libaq store); more
+        are loaded from `host` (a to_host() dict, kept referenced) by set_prefix. Calls accept
+        prefixes up to the resident one."""
+        self = cls.__new__(cls)
+        L = host["layout"]
+        self.layout = Layout(*[getattr(L, f) for f, _ in Layout._fields_])
+        self.layout.flags = AQ_LAYOUT_STATIC_WEIGHTS
+        self.out, self.inp, self.M, self.B = (L.out_features, L.in_features, L.num_books,
+                                              L.code_bits)
+        self.device = torch.device(device)
+        self.book_dtype, self.scale_dtype = host["book_dtype"], host["scale_dtype"]
+        with torch.cuda.device(self.device):
+            self.store = aq_store_create(self.layout)
+        self._finalizer = weakref.finalize(self, _destroy_store, self.store)
+        self._host = host
+        self.planes = aq_store_planes(self.store)
+        self.books = aq_store_books(self.store)
+        self.scales = aq_store_scales(self.store)
+        self.codes, self._ws, self.resident = None, {}, 0
+        self.set_prefix(m)
+        return self
+
+    def set_prefix(self, m):
+        """Raise or lower the resident prefix of a from_host layer to m (0..M). Raising copies
+        planes and codebooks on the current stream, so later work on that stream sees them;
+        lowering synchronises the device and frees the dropped planes' memory."""
+        if self.store is None:
+            raise TypeError("set_prefix needs a layer made by from_host")
+        h = self._host
+        with torch.cuda.device(self.device):
+            aq_store_set_prefix(self.store, m, h["planes"], h["books"], h["scales"])
+        self.resident = m
+
+    def device_bytes(self):
+        """Device memory held for the layer's weights (scales, codebooks, resident planes)."""
+        if self.store is not None:
+            return aq_store_device_bytes(self.store)
+        return sum(t.numel() * t.element_size() for t in (self.planes, self.books, self.scales))
+
+    def close(self):
+        """Release a from_host layer's device memory now (synchronises the device)."""
+        if self.store is not None:
+            self._finalizer()
+            self.store, self.planes, self.books, self.scales, self.resident = None, None, None, None, 0
+
+    def _check_m(self, m):
+        # A prefix beyond the resident one would read device memory that is not mapped.
+        if not 1 <= m <= self.resident:
+            raise ValueError("prefix m=%d outside 1..%d (resident codebooks)" % (m, self.resident))
 
     def planes_prefix(self, m):
         """The first m planes: the only code bytes a prefix-m call reads."""
@@ -82,6 +157,7 @@ class AQLinear:
         if out is None:
             out = torch.empty(self.out, self.inp, dtype=TORCH_DTYPES[DTYPES[self.book_dtype]],
                               device=self.device)
+        self._check_m(m)
         aq_decode(self.layout, m, self.planes, self.books, self.scales, out)
         return out
 
@@ -92,6 +168,7 @@ class AQLinear:
         batch = x.shape[0]
         if y is None:
             y = torch.empty(batch, self.out, dtype=TORCH_DTYPES[yd], device=self.device)
+        self._check_m(m)
         ws = self._workspace("gemv", batch)
         aq_gemv(self.layout, m, self.planes, self.books, self.scales, x, xd, batch, y, yd, ws)
         return y
@@ -105,6 +182,7 @@ class AQLinear:
         yd = _dtype_code(y_prev.dtype) if y_prev is not None else AQ_F32
         if y is None:
             y = torch.empty(batch, self.out, dtype=TORCH_DTYPES[yd], device=self.device)
+        self._check_m(m)
         ws = self._workspace("gemv", batch)
         aq_gemv_refine(self.layout, m, self.planes, self.books, self.scales, x, xd, batch, y_prev,
                        y, yd, ws)
@@ -117,6 +195,7 @@ class AQLinear:
         tokens = x.shape[0]
         if y is None:
             y = torch.empty(tokens, self.out, dtype=TORCH_DTYPES[yd], device=self.device)
+        self._check_m(m)
         ws = self._workspace("gemm", tokens)
         aq_gemm(self.layout, m, self.planes, self.books, self.scales, x, xd, tokens, y, yd, ws)
         return y

@@ -25,7 +25,7 @@ def built():
 
 def header_functions():
     text = open(HEADER).read()
-    return sorted(set(re.findall(r"^\s*(?:aq_status|size_t|int|const char\*)\s+(aq_\w+)\s*\(",
+    return sorted(set(re.findall(r"^\s*(?:aq_status|size_t|int|const char\*|void\*)\s+(aq_\w+)\s*\(",
                                  text, flags=re.M)))
 
 
@@ -125,3 +125,20 @@ def test_decode_and_pack_argument_errors():
     assert lib.aq_pack(ctypes.byref(L), None, FAKE, None) == aq.AQ_ERR_INVALID_ARG
     assert lib.aq_pack(None, FAKE, FAKE, None) == aq.AQ_ERR_INVALID_ARG
     assert lib.aq_workspace_init(None, 16, None) == aq.AQ_ERR_INVALID_ARG
+
+
+def test_store_argument_errors_on_the_host():
+    """Checks a prefix store makes before any CUDA call (no device needed)."""
+    lib = aq.lib()
+    h = ctypes.c_void_p()
+    assert lib.aq_store_create(None, ctypes.byref(h)) == aq.AQ_ERR_INVALID_ARG
+    assert h.value is None
+    assert lib.aq_store_create(ctypes.byref(_lay()), None) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_store_create(ctypes.byref(_lay(G=4)), ctypes.byref(h)) == aq.AQ_ERR_UNSUPPORTED
+    assert lib.aq_store_create(ctypes.byref(_lay(M=0)), ctypes.byref(h)) == aq.AQ_ERR_INVALID_ARG
+    assert h.value is None
+    assert lib.aq_store_set_prefix(None, 1, FAKE, FAKE, FAKE, None) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_store_prefix(None) == 0 and lib.aq_store_device_bytes(None) == 0
+    assert lib.aq_store_planes(None) is None and lib.aq_store_books(None) is None
+    assert lib.aq_store_scales(None) is None
+    assert lib.aq_store_destroy(None) == aq.AQ_OK
