@@ -40,10 +40,25 @@ def _run_mutant(tmpdir, name, old, new):
     lib = os.path.join(tmpdir, name + ".so")
     subprocess.run(["g++", "-O1", "-std=c++17", "-ffp-contract=off", "-fopenmp", "-shared",
                     "-fPIC", mut_src, "-o", lib], check=True)
-    env = dict(os.environ, ORACLE_LIB=lib, OMP_NUM_THREADS="1")
+    return (name,) + _run_pins(lib)
+
+
+def _run_pins(lib):
+    """Run every pin in a fresh interpreter against the oracle build `lib`: (exit code, output).
+    Exit code 1 with a pin's name in the output means a pin failed."""
+    env = dict(os.environ, ORACLE_LIB=lib, OMP_NUM_THREADS="1",
+               PYTHONPATH=os.pathsep.join([ROOT, os.path.join(ROOT, "tests")]))
     r = subprocess.run([sys.executable, os.path.join(ROOT, "tests", "oracle_pins.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
-    return name, r.returncode, r.stdout[-2000:] + r.stderr[-2000:]
+    return r.returncode, r.stdout[-2000:] + r.stderr[-2000:]
+
+
+def test_unmutated_oracle_passes_the_pin_script():
+    """Control: the script the mutants run passes on the real oracle, so a mutant's failure is
+    a pin failing, not the script failing to start."""
+    import oracle
+    rc, out = _run_pins(oracle.build.build())
+    assert rc == 0 and "all pins passed" in out, out
 
 
 def test_every_planted_mistake_is_caught(tmp_path):
@@ -52,3 +67,6 @@ def test_every_planted_mistake_is_caught(tmp_path):
         results = [f.result() for f in futs]
     survivors = [(n, out) for n, rc, out in results if rc == 0]
     assert not survivors, "mutants not caught by any pin: %s" % survivors
+    # a caught mutant is one whose pins ran and at least one failed (not a crash on start-up)
+    broken = [(n, out) for n, rc, out in results if "pin_" not in out]
+    assert not broken, "mutant runs that did not reach the pins: %s" % broken
