@@ -32,6 +32,8 @@ def lib():
         L.oracle_decode.argtypes = [i32] * 6 + [vp, u16p, i32, u16p, i32, u16p]
         L.oracle_product_exact.restype = i32
         L.oracle_product_exact.argtypes = [i32] * 6 + [vp, u16p, i32, u16p, i32, u16p, i32, i32, vp]
+        L.oracle_reconstruct_exact.restype = i32
+        L.oracle_reconstruct_exact.argtypes = [i32] * 6 + [vp, u16p, i32, u16p, i32, vp]
         L.oracle_product_dense.restype = i32
         L.oracle_product_dense.argtypes = [i32, i32, u16p, i32, u16p, i32, i32, vp]
         L.oracle_pack.restype = i32
@@ -109,6 +111,66 @@ def product_exact(layer, x, x_dtype, m, rows=None):
     if rc:
         raise ValueError("oracle_product_exact rejected the shape")
     return y
+
+
+def reconstruct_exact(layer, m):
+    """W^(m) of Sec. 5 in fp64, unrounded: [out][in], s[o]*sum_{k<m} C_k[b_{o,g,k}][e]."""
+    out, inp, G, M, B = layer["out"], layer["in"], layer["G"], layer["M"], layer["B"]
+    codes = layer["codes"]
+    _codes_ok(codes, B)
+    w = np.empty((out, inp), dtype=np.float64)
+    rc = lib().oracle_reconstruct_exact(out, inp, G, M, B, m, _p(codes), _p(layer["books"]),
+                                        _DT[layer["book_dtype"]], _p(layer["scales"]),
+                                        _DT[layer["scale_dtype"]], _p(w))
+    if rc:
+        raise ValueError("oracle_reconstruct_exact rejected the shape")
+    return w
+
+
+def wmse(layer, W, H, ks=None):
+    """Per-prefix distortion of Sec. 5 with the weighted MSE of Sec. 2.2 (Eq. wmse-task, its
+    trace form): D^(k) = (1/d_out) * tr[(W - W^(k)) H (W - W^(k))^T] for k in ks (default
+    1..M), W^(k) the exact prefix-k reconstruction. W: [out][in] float64 (the original weight),
+    H: [in][in] float64 (the proxy X X^T / n; any square matrix is evaluated as given).
+    Returns a float64 array, entry i for prefix ks[i].
+
+    The trace is taken as the sum of the diagonal of (W - W^(k)) H (W - W^(k))^T, whose entry
+    o is sum_i ((W - W^(k)) H)[o, i] * (W - W^(k))[o, i]; the out x out product itself is not
+    formed. The matrix product is numpy's (fp64)."""
+    out = layer["out"]
+    ks = range(1, layer["M"] + 1) if ks is None else ks
+    W = np.asarray(W, dtype=np.float64)
+    H = np.asarray(H, dtype=np.float64)
+    res = []
+    for k in ks:
+        E = W - reconstruct_exact(layer, k)
+        res.append(float(np.sum((E @ H) * E)) / out)
+    return np.array(res)
+
+
+def wmse_abs(layer, W, H, ks=None):
+    """(1/d_out) * sum_o |e_o| |H| |e_o|^T for each prefix (e_o = row o of W - W^(k)): the
+    magnitude that first-order rounding-error bounds of D^(k) scale with."""
+    out = layer["out"]
+    ks = range(1, layer["M"] + 1) if ks is None else ks
+    A = np.abs(np.asarray(H, dtype=np.float64))
+    res = []
+    for k in ks:
+        E = np.abs(np.asarray(W, dtype=np.float64) - reconstruct_exact(layer, k))
+        res.append(float(np.sum((E @ A) * E)) / out)
+    return np.array(res)
+
+
+def dbyd_loss(D, lam):
+    """Sec. 5 Drop-by-Drop objective: L = sum_k lambda_k D^(k) (lam[k-1] weights prefix k)."""
+    D = np.asarray(D, dtype=np.float64)
+    lam = np.asarray(lam, dtype=np.float64)
+    if lam.shape != D.shape:
+        raise ValueError("one weight per prefix")
+    total = 0.0
+    for k in range(D.shape[0]):
+        total += lam[k] * D[k]
+    return total
 
 
 def product_dense(w_bits, w_dtype, x, x_dtype):

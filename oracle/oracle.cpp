@@ -16,6 +16,8 @@
 //     the input activations. Here activations are row vectors, y[t,o] = sum_i x[t,i] W[o,i].
 //   * App. C ("Estimating Model Size", Eq. avg_bits): storage cost of codebooks, codes and
 //     per-output-unit scales.
+//   * Sec. 5 partial reconstruction W^(k) in fp64, the input of the per-prefix distortion
+//     D^(k) (Sec. 2.2 Eq. wmse-task; evaluated in oracle/__init__.py).
 //
 // Readings where the paper is silent (each is listed in the design notes of the repository):
 //   R1 the per-output-row scale s[o] multiplies the codebook sum: W[o, group] = s[o]*sum_k C_k[b].
@@ -199,6 +201,31 @@ int oracle_product_exact(int out, int in, int G, int M, int B, int m, const void
             }
         }
         delete[] wrow;
+    }
+    return 0;
+}
+
+// Exact partial reconstruction W^(m) of Sec. 5 in fp64 (no rounding): the stored values
+// widened exactly, w_out[o][g*G+e] = s[o] * sum_{k<m} C_k[b_{o,g,k}][e], summed in book order.
+// This is the reconstruction inside the distortion D^(k) of Sec. 5.
+int oracle_reconstruct_exact(int out, int in, int G, int M, int B, int m, const void* codes,
+                             const uint16_t* books, int book_dtype, const uint16_t* scales,
+                             int scale_dtype, double* w_out) {
+    if (check_shape(out, in, G, M, B, m)) return 1;
+    const long ng = in / G;
+    const long book_stride = (1L << B) * G;
+#pragma omp parallel for schedule(static)
+    for (long o = 0; o < out; ++o) {
+        const double s = bits_to_double(scales[o], scale_dtype);
+        for (long g = 0; g < ng; ++g)
+            for (int e = 0; e < G; ++e) {
+                double acc = 0.0;
+                for (int k = 0; k < m; ++k) {
+                    const uint32_t j = code_at(codes, B, (o * ng + g) * M + k);
+                    acc += bits_to_double(books[k * book_stride + (long)j * G + e], book_dtype);
+                }
+                w_out[o * in + g * G + e] = s * acc;
+            }
     }
     return 0;
 }

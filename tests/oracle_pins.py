@@ -290,6 +290,124 @@ def pin_dense_product_of_decode():
         assert np.all(np.abs(a - b) <= bound + 1e-12), m
 
 
+# ---------------------------------------------------------------- distortion (Sec. 2.2, Sec. 5)
+
+def _wmse_case(out=24, inp=64, M=3, seed=7, dt="bf16"):
+    """A layer, an 'original' weight W near its full reconstruction, and an activation matrix."""
+    layer = workloads.make_layer(out, inp, G=8, M=M, B=8, book_dtype=dt, book_std=0.3,
+                                 scale_dtype=dt, seed=seed)
+    rng = _rng(seed + 1)
+    W = _onehot_reconstruction(layer, M) + 0.05 * rng.standard_normal((out, inp))
+    X = rng.standard_normal((inp, 2 * inp))
+    return layer, W, X
+
+
+def pin_reconstruct_exact_matches_onehot():
+    """The exact W^(k) equals the one-hot brute force of Sec. 3.2 / Sec. 5 for every prefix."""
+    for layer in _tiny_layers():
+        for m in range(1, layer["M"] + 1):
+            assert np.array_equal(oracle.reconstruct_exact(layer, m),
+                                  _onehot_reconstruction(layer, m)), (layer["out"], m)
+
+
+def pin_wmse_identity_is_frobenius():
+    """X = I (H = I) reduces the weighted MSE to the plain MSE: D^(k) = ||W - W^(k)||_F^2 / d_out."""
+    layer, W, _ = _wmse_case()
+    D = oracle.wmse(layer, W, np.eye(layer["in"]))
+    for k in range(1, layer["M"] + 1):
+        E = W - _onehot_reconstruction(layer, k)
+        want = sum(float(v) * float(v) for v in E.ravel()) / layer["out"]
+        assert abs(D[k - 1] - want) <= 1e-12 * want, (k, D[k - 1], want)
+
+
+def pin_wmse_trace_form_equals_activation_form():
+    """The two sides of Eq. wmse-task: tr[E (X X^T / n) E^T] / d_out = ||E X||_F^2 / (d_out n)."""
+    layer, W, X = _wmse_case()
+    n = X.shape[1]
+    D = oracle.wmse(layer, W, X @ X.T / n)
+    for k in range(1, layer["M"] + 1):
+        EX = (W - _onehot_reconstruction(layer, k)) @ X
+        want = float(np.sum(EX * EX)) / (layer["out"] * n)
+        assert abs(D[k - 1] - want) <= 1e-10 * want, (k, D[k - 1], want)
+
+
+def pin_wmse_bruteforce_tiny():
+    """Triple sum over rows and input pairs, in plain Python, on a 3 x 16 layer."""
+    layer, W, X = _wmse_case(out=3, inp=16, M=2, seed=11, dt="f16")
+    H = X @ X.T / X.shape[1]
+    D = oracle.wmse(layer, W, H)
+    for k in (1, 2):
+        E = W - _onehot_reconstruction(layer, k)
+        tot = 0.0
+        for o in range(3):
+            for i in range(16):
+                for j in range(16):
+                    tot += E[o, i] * H[i, j] * E[o, j]
+        assert abs(D[k - 1] - tot / 3) <= 1e-10 * abs(tot / 3), (k, D[k - 1], tot / 3)
+
+
+def pin_wmse_vanishes_at_the_exact_weight():
+    """W = W^(M): the full prefix has zero distortion; a shorter prefix leaves the dropped
+    codebooks' contribution, which is positive for a positive definite H."""
+    layer, _, X = _wmse_case(seed=13)
+    M = layer["M"]
+    W = _onehot_reconstruction(layer, M)
+    D = oracle.wmse(layer, W, X @ X.T / X.shape[1])
+    assert D[M - 1] == 0.0
+    assert all(d > 0 for d in D[:-1]), D
+
+
+def pin_wmse_invariances():
+    """Only the symmetric part of H matters; D is linear in H; permuting rows (codes, scales
+    and W together) changes nothing; the row sum splits over row blocks."""
+    layer, W, X = _wmse_case(out=20, seed=17)
+    rng = _rng(18)
+    H = X @ X.T / X.shape[1]
+    A = rng.standard_normal(H.shape)
+    D = oracle.wmse(layer, W, H)
+    assert np.allclose(oracle.wmse(layer, W, H + A - A.T), D, rtol=1e-12, atol=0)
+    assert np.allclose(oracle.wmse(layer, W, 2.5 * H), 2.5 * D, rtol=1e-12, atol=0)
+    perm = rng.permutation(layer["out"])
+    pl = dict(layer, codes=np.ascontiguousarray(layer["codes"][perm]),
+              scales=np.ascontiguousarray(layer["scales"][perm]))
+    assert np.allclose(oracle.wmse(pl, W[perm], H), D, rtol=1e-12, atol=0)
+    top = dict(layer, out=8, codes=np.ascontiguousarray(layer["codes"][:8]),
+               scales=np.ascontiguousarray(layer["scales"][:8]))
+    bot = dict(layer, out=12, codes=np.ascontiguousarray(layer["codes"][8:]),
+               scales=np.ascontiguousarray(layer["scales"][8:]))
+    split = (8 * oracle.wmse(top, W[:8], H) + 12 * oracle.wmse(bot, W[8:], H)) / 20
+    assert np.allclose(split, D, rtol=1e-12, atol=0)
+
+
+def _paper_loss_weights():
+    out = {}
+    with open(os.path.join(GOLDEN, "dbyd_loss_weights.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                name, *vals = line.split()
+                out[name] = [float(Fraction(v)) for v in vals]
+    return out
+
+
+def pin_dbyd_loss_paper_weightings():
+    """Sec. 5 / App. G.2 weightings: L = sum_k lambda_k D^(k) with lambda_k weighting prefix k.
+    A unit distortion at prefix j alone gives lambda_j; Uni averages; 35W averages prefixes 3
+    and 5; 345W averages prefixes 3, 4 and 5."""
+    w = _paper_loss_weights()
+    assert set(w) == {"Uni", "35W", "3W", "345W"}
+    for name, lam in w.items():
+        assert len(lam) == 5 and abs(sum(lam) - 1.0) < 1e-15, name
+        for j in range(5):
+            D = np.zeros(5)
+            D[j] = 1.0
+            assert oracle.dbyd_loss(D, lam) == lam[j], (name, j)
+    D = np.array([16.0, 8.0, 4.0, 2.0, 1.0])
+    assert abs(oracle.dbyd_loss(D, w["Uni"]) - 31.0 / 5) < 1e-14
+    assert oracle.dbyd_loss(D, w["35W"]) == (4.0 + 1.0) / 2
+    assert oracle.dbyd_loss(D, w["3W"]) == 4.0
+    assert abs(oracle.dbyd_loss(D, w["345W"]) - 7.0 / 3) < 1e-15
+
+
 # ---------------------------------------------------------------- packed planes
 
 def pin_pack_positions():

@@ -1,6 +1,8 @@
 """Plant plausible mistakes in a copy of the oracle (on the CPU) and check that the pins catch
 each one: a dropped scale, a wrong prefix bound, a transposed codebook, a reversed book order,
-a sign error, wrong rounding, a wrong packing rotation, a wrong storage formula. A mutant that
+a sign error, wrong rounding, a wrong packing rotation, a wrong storage formula, and in the
+distortion and loss a dropped normalisation, an off-by-one prefix, a sign error, a wrong
+proxy Hessian power and shifted loss weights. A mutant that
 passes every pin would mean the pins could not tell that mistake from the truth."""
 import concurrent.futures as cf
 import os
@@ -28,6 +30,20 @@ MUTANTS = [
      "sum += bits_to_double(x[t * in + (in - 1 - i)], x_dtype) * wrow[i];"),
     ("pack_rotation_wrong", "((p + o) % 32)", "((p + 32 - o % 32) % 32)"),
     ("avg_bits_without_M", "(double)M * (double)d_out", "(double)d_out"),
+    ("reconstruct_drops_scale", "w_out[o * in + g * G + e] = s * acc;",
+     "w_out[o * in + g * G + e] = acc;"),
+]
+
+# Mistakes planted in the Python part of the oracle (oracle/__init__.py): the distortion and
+# loss of Sec. 2.2 / Sec. 5.
+PY_MUTANTS = [
+    ("wmse_drops_normalisation", "np.sum((E @ H) * E)) / out", "np.sum((E @ H) * E))"),
+    ("wmse_prefix_off_by_one", "E = W - reconstruct_exact(layer, k)\n        res.append(float(np.sum((E @ H)",
+     "E = W - reconstruct_exact(layer, max(1, k - 1))\n        res.append(float(np.sum((E @ H)"),
+    ("wmse_sign_error", "E = W - reconstruct_exact(layer, k)\n        res.append(float(np.sum((E @ H)",
+     "E = W + reconstruct_exact(layer, k)\n        res.append(float(np.sum((E @ H)"),
+    ("wmse_squares_H", "np.sum((E @ H) * E)", "np.sum((E @ H @ H) * E)"),
+    ("dbyd_shifted_weights", "total += lam[k] * D[k]", "total += lam[k] * D[k - 1]"),
 ]
 
 
@@ -43,11 +59,27 @@ def _run_mutant(tmpdir, name, old, new):
     return (name,) + _run_pins(lib)
 
 
-def _run_pins(lib):
+def _run_py_mutant(tmpdir, name, old, new):
+    """A copy of the oracle package with one replacement in __init__.py, first on the path."""
+    import shutil
+    src_dir = os.path.join(ROOT, "oracle")
+    pkg = os.path.join(tmpdir, name, "oracle")
+    os.makedirs(pkg)
+    for f in ("build.py", "oracle.cpp"):
+        shutil.copy(os.path.join(src_dir, f), pkg)
+    text = open(os.path.join(src_dir, "__init__.py")).read()
+    assert old in text, "mutation site for %s not found in oracle/__init__.py" % name
+    with open(os.path.join(pkg, "__init__.py"), "w") as f:
+        f.write(text.replace(old, new))
+    import oracle
+    return (name,) + _run_pins(oracle.build.build(), first=os.path.join(tmpdir, name))
+
+
+def _run_pins(lib, first=None):
     """Run every pin in a fresh interpreter against the oracle build `lib`: (exit code, output).
     Exit code 1 with a pin's name in the output means a pin failed."""
-    env = dict(os.environ, ORACLE_LIB=lib, OMP_NUM_THREADS="1",
-               PYTHONPATH=os.pathsep.join([ROOT, os.path.join(ROOT, "tests")]))
+    path = ([first] if first else []) + [ROOT, os.path.join(ROOT, "tests")]
+    env = dict(os.environ, ORACLE_LIB=lib, OMP_NUM_THREADS="1", PYTHONPATH=os.pathsep.join(path))
     r = subprocess.run([sys.executable, os.path.join(ROOT, "tests", "oracle_pins.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
     return r.returncode, r.stdout[-2000:] + r.stderr[-2000:]
@@ -64,6 +96,7 @@ def test_unmutated_oracle_passes_the_pin_script():
 def test_every_planted_mistake_is_caught(tmp_path):
     with cf.ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 2)) as ex:
         futs = [ex.submit(_run_mutant, str(tmp_path), *m) for m in MUTANTS]
+        futs += [ex.submit(_run_py_mutant, str(tmp_path), *m) for m in PY_MUTANTS]
         results = [f.result() for f in futs]
     survivors = [(n, out) for n, rc, out in results if rc == 0]
     assert not survivors, "mutants not caught by any pin: %s" % survivors
