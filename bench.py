@@ -39,6 +39,10 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-gemm", action="store_true")
+    ap.add_argument("--no-wmse", action="store_true",
+                    help="skip the per-prefix distortion measurement")
+    ap.add_argument("--wmse-only", action="store_true",
+                    help="only the per-prefix distortion measurement (for profiling)")
     ap.add_argument("--no-loading", action="store_true",
                     help="skip the prefix-store loading measurement")
     ap.add_argument("--gemm-tokens", type=int, default=4096,
@@ -293,6 +297,46 @@ def measure_loading(lin, dev, stream, ms, reps=7):
             "device_bytes_at_m4": resident, "matches_full_layer": same}
 
 
+def measure_wmse(lin, dev, stream, peaks, reps=10):
+    """aq_wmse on the benchmark layer: D^(k) for all four prefixes in one call (Sec. 2.2
+    Eq. wmse-task, Sec. 5). W = the full reconstruction plus N(0, 0.01^2) noise in the book
+    type; H = X X^T / n for Gaussian X with n = 2 * d_in (fp32). CUDA events around `reps`
+    back-to-back calls (each: folding of H, the tensor-core pass, the reduction)."""
+    import torch
+    out, inp, M = lin.out, lin.inp, lin.M
+    g = torch.Generator(device=dev).manual_seed(7)
+    W = (lin.decode(M).float() + 0.01 * torch.randn(out, inp, device=dev, generator=g)).half()
+    X = torch.randn(inp, 2 * inp, device=dev, generator=g)
+    H = (X @ X.t()) / X.shape[1]
+    del X
+    lam = [0.25] * M
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            d = lin.wmse(W, H, lam)
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            d = lin.wmse(W, H, lam)
+        e1.record()
+    torch.cuda.synchronize(dev)
+    ms = e0.elapsed_time(e1) / reps
+    # tensor-core work actually issued: per pair tile (256 t x 128 rows) K = min(256 (tb+1), in)
+    tb_n, ob_n = -(-inp // 256), -(-out // 128)
+    ksum = sum(-(-min(256 * (tb + 1), inp) // 64) * 64 for tb in range(tb_n))
+    mma_flops = 2.0 * 256 * 128 * ksum * ob_n * M
+    def_flops = 2.0 * M * out * inp * inp          # E_k H for every prefix, as defined
+    peak = peaks.get("bf16_tflops", 1900.0)
+    tf = mma_flops / (ms * 1e-3) / 1e12
+    return {"workload": "attn_4096", "out": out, "in": inp, "M": M,
+            "compute": "bf16 tcgen05 pair MMA (E_k x folded H), fp32 accumulation, all prefixes per pass",
+            "ms": round(ms, 4), "mma_TFLOP_s": round(tf, 1), "frac_bf16_peak": round(tf / peak, 4),
+            "definition_TFLOP_s": round(def_flops / (ms * 1e-3) / 1e12, 1),
+            "mma_flops": mma_flops, "D": [round(float(v), 6) for v in d[:M].tolist()],
+            "loss_uniform": round(float(d[M]), 6),
+            "peak_source": "measured" if "bf16_tflops" in peaks else "fallback"}
+
+
 def own_arm(args):
     import numpy as np
     import torch
@@ -335,6 +379,9 @@ def own_arm(args):
     peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
 
     stream = torch.cuda.Stream(device=dev)
+    if args.wmse_only:
+        print(json.dumps({"wmse_only": measure_wmse(lin, dev, stream, peaks)}), flush=True)
+        return
     if args.skip_gemv:
         g = measure_gemm(dev, stream, peaks, tokens=args.gemm_tokens)
         print(json.dumps({"gemm_only": g}), flush=True)
@@ -452,6 +499,7 @@ def own_arm(args):
 
     gemm = None if args.no_gemm else measure_gemm(dev, stream, peaks, tokens=args.gemm_tokens)
     loading = measure_loading(lin, dev, stream, ms) if rank == 0 and not args.no_loading else None
+    wmse = None if args.no_wmse else measure_wmse(lin, dev, stream, peaks)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -475,6 +523,7 @@ def own_arm(args):
             "per_m": per_m,
             "gemm": gemm,
             "dynamic_loading": loading,
+            "wmse": wmse,
             "roofline": {
                 "bound": "hbm", "kernel": "gemv_lut_kernel m=%d" % dom["m"],
                 "achieved": dom["GB_s"], "peak": hbm_peak, "unit": "GB/s",

@@ -198,6 +198,34 @@ aq_status aq_gemm(const aq_layout* layout, int m, const void* planes, const void
                   const void* scales, const void* x, int x_dtype, int tokens, void* y,
                   int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
 
+/* ---------------------------------------------------------------- distortion of every prefix
+ * The weighted MSE of Sec. 2.2 (Eq. wmse-task, trace form) for every prefix, as Drop-by-Drop
+ * measures its partial reconstructions (Sec. 5), and the Drop-by-Drop objective:
+ *     D[k-1] = (1/d_out) * tr[(W - W^(k)) H (W - W^(k))^T],   k = 1..M,
+ *     W^(k)[o, g*8+e] = s[o] * sum_{j<k} C_j[b_j[o,g]][e]   (unrounded; fp32 on the GPU),
+ *     L = sum_k lambda[k-1] * D[k-1]                        (when lambda is given).
+ * H is the proxy Hessian X X^T / n of the layer's calibration inputs; only its symmetric part
+ * enters the trace, so any square H is accepted and evaluated as (H + H^T)/2.
+ *   w       : device, [d_out][d_in] of book_dtype (the original weight)
+ *   h       : device, [d_in][d_in] of h_dtype (AQ_F32 or AQ_BF16), row-major
+ *   lambda  : HOST, M doubles (the weight of prefix k at index k-1), or NULL
+ *   d       : device, M doubles, 8-byte aligned (M + 1 when lambda is given: d[M] = L);
+ *             written, not accumulated; d_out = 0 gives zeros
+ *   workspace : device, aq_wmse_workspace_bytes(layout) bytes, 16-byte aligned: a status word,
+ *             a bf16 copy of the folded H (d_in^2 * 2 bytes) and per-CTA partial sums. Zero-
+ *             fill it once before first use (aq_workspace_init); device-side waits that time
+ *             out are reported through it (aq_workspace_status).
+ * Computation: E_k = W - W^(k) (fp32, then rounded once to bf16) times H folded to its
+ * block-lower-triangular symmetric form (bf16) on the tcgen05 tensor cores with fp32
+ * accumulation, for up to four prefixes per pass; per-tile sums are added in fp64 in a fixed
+ * order. Accuracy: |D - D_exact| <= 1.25e-2 * D_abs with D_abs = (1/d_out) sum_o |e_o||H||e_o|^T
+ * (three bf16 roundings, first order), typically far smaller.
+ * Supported: code_bits = 8. Errors: as aq_gemv (AQ_ERR_UNSUPPORTED for 16-bit codes). */
+size_t aq_wmse_workspace_bytes(const aq_layout* layout);
+aq_status aq_wmse(const aq_layout* layout, const void* w, const void* planes, const void* books,
+                  const void* scales, const void* h, int h_dtype, const double* lambda, double* d,
+                  void* workspace, size_t workspace_bytes, void* stream);
+
 /* ---------------------------------------------------------------- dynamic loading
  * Device storage for one layer that holds only a prefix of its codebooks. One stored model
  * serves every bit width, and each deployment keeps as many codebooks on the device as its

@@ -26,7 +26,7 @@ EXPORTS = ["aq_abi_version", "aq_status_string", "aq_last_error", "aq_plane_byte
            "aq_gemm", "aq_workspace_init", "aq_workspace_status", "aq_gemv_static_scratch",
            "aq_gemv_refine", "aq_store_create", "aq_store_set_prefix", "aq_store_prefix",
            "aq_store_planes", "aq_store_books", "aq_store_scales", "aq_store_device_bytes",
-           "aq_store_destroy"]
+           "aq_store_destroy", "aq_wmse_workspace_bytes", "aq_wmse"]
 
 
 class AQError(RuntimeError):
@@ -87,6 +87,9 @@ def lib():
             "aq_store_scales": (vp, [vp]),
             "aq_store_device_bytes": (sz, [vp]),
             "aq_store_destroy": (i32, [vp]),
+            "aq_wmse_workspace_bytes": (sz, [lp]),
+            "aq_wmse": (i32, [lp, vp, vp, vp, vp, vp, i32, ctypes.POINTER(ctypes.c_double), vp,
+                              vp, sz, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -230,6 +233,24 @@ def aq_store_device_bytes(store):
 
 def aq_store_destroy(store):
     _check(lib().aq_store_destroy(store), "aq_store_destroy")
+
+
+def wmse_workspace_bytes(layout):
+    return lib().aq_wmse_workspace_bytes(ctypes.byref(layout))
+
+
+def aq_wmse(layout, w, planes, books, scales, h, h_dtype, lam, d, workspace,
+            workspace_bytes=None, stream=None):
+    """d[k-1] = tr[(W - W^(k)) H (W - W^(k))^T] / d_out for k = 1..M; with lam (M host
+    floats) also d[M] = sum_k lam[k-1] d[k-1]."""
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    lam_arr = None
+    if lam is not None:
+        lam_arr = (ctypes.c_double * len(lam))(*[float(v) for v in lam])
+    _check(lib().aq_wmse(ctypes.byref(layout), _ptr(w), _ptr(planes), _ptr(books), _ptr(scales),
+                         _ptr(h), h_dtype, lam_arr, _ptr(d), _ptr(workspace), workspace_bytes,
+                         _stream(stream)), "aq_wmse")
 
 
 def aq_workspace_init(workspace, nbytes=None, stream=None):

@@ -214,6 +214,31 @@ aq_status aq_gemv_refine(const aq_layout* layout, int m, const void* planes, con
                            as_stream(stream), y_prev);
 }
 
+size_t aq_wmse_workspace_bytes(const aq_layout* layout) {
+    Dims d;
+    if (aq::make_dims(layout, &d) != AQ_OK) return 0;
+    return aq::wmse_ws_bytes(d);
+}
+
+aq_status aq_wmse(const aq_layout* layout, const void* w, const void* planes, const void* books,
+                  const void* scales, const void* h, int h_dtype, const double* lambda, double* d_out,
+                  void* workspace, size_t workspace_bytes, void* stream) {
+    Dims d;
+    aq_status st = aq::make_dims(layout, &d);
+    if (st != AQ_OK) return st;
+    if (d.B != 8) return AQ_ERR_UNSUPPORTED;
+    if (h_dtype != AQ_F32 && h_dtype != AQ_BF16) return AQ_ERR_INVALID_ARG;
+    if (!d_out) return AQ_ERR_INVALID_ARG;
+    if (((uintptr_t)d_out & 7u) != 0) return AQ_ERR_ALIGNMENT;
+    if (d.out > 0) {
+        if ((st = check_ptrs({w, planes, books, scales, h})) != AQ_OK) return st;
+        if (!workspace || workspace_bytes < aq::wmse_ws_bytes(d)) return AQ_ERR_WORKSPACE;
+        if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;
+    }
+    return aq::launch_wmse(d, w, planes, books, scales, h, h_dtype, lambda, d_out, workspace,
+                           as_stream(stream));
+}
+
 size_t aq_gemm_workspace_bytes(const aq_layout* layout, int tokens) {
     Dims d;
     if (aq::make_dims(layout, &d) != AQ_OK || tokens < 0) return 0;

@@ -44,6 +44,7 @@
 #include <mutex>
 
 #include "aq_internal.cuh"
+#include "tc_ptx.cuh"
 
 namespace aq {
 namespace {
@@ -83,127 +84,6 @@ constexpr int kOffAbort = kOffTmem + 16;
 constexpr int kGemmSmem = kOffAbort + 16;
 static_assert(kGemmSmem <= 227 * 1024, "shared memory map exceeds the per-CTA limit");
 
-// ---- tcgen05 / TMA / cluster helpers (PTX) --------------------------------------------------
-
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int c0, int c1,
-                                            uint64_t* bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
-        "l"((uint64_t)map), "r"(c0), "r"(c1), "r"(smem_u32(bar))
-        : "memory");
-}
-
-__device__ __forceinline__ uint32_t cluster_rank() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-
-// Address, in the cluster shared window, of the variable at local address `addr` in CTA `rank`.
-__device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
-    uint32_t r;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
-    return r;
-}
-
-// Arrive on an mbarrier of another CTA of the cluster. The data it announces lives in the
-// arriving CTA's own shared memory (written there by its TMA copies and its decoders, which
-// this thread has already waited for), so the arrive orders those writes at CTA scope, the
-// usual form of a cross-CTA pipeline signal; a cluster-scope release costs this thread about
-// half a microsecond per stage, which alone exceeds a stage's MMA time.
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
-    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
-}
-
-// Bulk copy from this CTA's shared memory to another CTA's (cluster addresses for the
-// destination and its mbarrier), completing on that mbarrier's transaction count.
-__device__ __forceinline__ void bulk_to_peer(uint32_t dst_cluster, uint32_t src, uint32_t bytes,
-                                             uint32_t bar_cluster) {
-    asm volatile(
-        "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-            dst_cluster),
-        "r"(src), "r"(bytes), "r"(bar_cluster)
-        : "memory");
-}
-
-// Bounded wait with cluster-scope acquire (for phases completed by another CTA's arrivals).
-__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity) {
-    auto try_once = [&]() {
-        uint32_t ok;
-        asm volatile(
-            "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n"
-            " selp.u32 %0, 1, 0, p;\n}\n"
-            : "=r"(ok)
-            : "r"(smem_u32(bar)), "r"(parity), "r"(kSuspendHintNs)
-            : "memory");
-        return ok != 0;
-    };
-    if (try_once()) return true;
-    const uint64_t t0 = global_ns();
-    do {
-        if (try_once()) return true;
-    } while (global_ns() - t0 < kWaitLimitNs);
-    return false;
-}
-
-// All threads of both CTAs (release / acquire at cluster scope); callable from divergent code.
-__device__ __forceinline__ void cluster_sync() {
-    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
-}
-
-// UMMA shared-memory descriptor: K-major operand, 128-byte swizzle, 8-row atoms 1024 bytes
-// apart (SBO), version 1, leading offset unused (16 bytes).
-__device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr) {
-    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)64 << 32) |
-           ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
-}
-
-// Pair MMA: D[256 x N] (+)= A[256 x 16] * B[N x 16]^T, A and D split by rows across the pair,
-// B split by rows (N) across the pair; issued by one thread of the leader CTA.
-__device__ __forceinline__ void umma_f16_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                              uint32_t idesc, uint32_t accumulate) {
-    asm volatile(
-        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
-        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-
-// Arrive on the barrier at local offset `bar` in every CTA of `mask` (cluster ranks) once every
-// prior pair MMA of this thread has completed.
-__device__ __forceinline__ void umma_commit_pair(uint64_t* bar, uint16_t mask) {
-    asm volatile(
-        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-        " [%0], %1;" ::"r"(smem_u32(bar)), "h"(mask)
-        : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_before() {
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-
-// 32 consecutive fp32 columns of this warp's 32 tensor-memory lanes (one lane per thread).
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
-    uint32_t r[32];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-        "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
-          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
-          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
-          "=r"(r[31])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
-
 __device__ __forceinline__ uint32_t pack2(float lo, float hi, int dt) {
     if (dt == AQ_BF16) {
         __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
@@ -211,26 +91,6 @@ __device__ __forceinline__ uint32_t pack2(float lo, float hi, int dt) {
     }
     __half2 h = __floats2half2_rn(lo, hi);
     return *(uint32_t*)&h;
-}
-
-// Shared-memory accesses through 32-bit shared-window addresses. lds128 is for data that no
-// thread writes while it may be read (codebooks): the compiler may reorder it freely.
-// lds128_ordered stays after the barrier wait that precedes it.
-__device__ __forceinline__ uint4 lds128(uint32_t a) {
-    uint4 v;
-    asm("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
-    return v;
-}
-__device__ __forceinline__ uint4 lds128_ordered(uint32_t a) {
-    uint4 v;
-    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a) : "memory");
-    return v;
-}
-__device__ __forceinline__ void sts128(uint32_t a, uint4 v) {
-    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z),
-                 "r"(v.w)
-                 : "memory");
 }
 
 __device__ __forceinline__ uint32_t f16x2(float2 v) {   // {lo, hi} -> packed fp16 pair, RN
@@ -267,16 +127,6 @@ __device__ __forceinline__ uint4 decode_group(uint32_t books, const uint32_t (&c
         return make_uint4(f16x2(make_float2(a[0], a[1])), f16x2(make_float2(a[2], a[3])),
                           f16x2(make_float2(a[4], a[5])), f16x2(make_float2(a[6], a[7])));
     }
-}
-
-// Bounded wait that gives up at once after a failure anywhere in the CTA.
-__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                              unsigned int* status) {
-    if (*abort) return false;
-    if (mbar_wait(bar, parity)) return true;
-    record_status(status, AQ_ERR_TIMEOUT);
-    *abort = 1;
-    return false;
 }
 
 // One instantiation per book type and prefix length MB (= m): the decoders' code holds exactly
@@ -665,29 +515,6 @@ __global__ void __launch_bounds__(256) bf16_to_f16_kernel(const uint4* __restric
 }
 
 // ---- host side ------------------------------------------------------------------------------
-
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
-                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
-                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
-                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-aq_status get_encode_fn(EncodeTiledFn* fn) {
-    static std::mutex mu;
-    static EncodeTiledFn cached = nullptr;
-    std::lock_guard<std::mutex> lock(mu);
-    if (!cached) {
-        void* p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
-                                                             cudaEnableDefault, &q);
-            e != cudaSuccess)
-            return cuda_fail(e, "cudaGetDriverEntryPointByVersion");
-        if (q != cudaDriverEntryPointSuccess || !p) return AQ_ERR_CUDA;
-        cached = (EncodeTiledFn)p;
-    }
-    *fn = cached;
-    return AQ_OK;
-}
 
 // Four pairs per cluster (clusters of eight) measured slower than two at every m: only 16
 // clusters of eight fit at once (128 of the 152 SMs), which costs more than the halved

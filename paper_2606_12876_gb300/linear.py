@@ -13,7 +13,8 @@ import torch
 
 from . import (AQ_BF16, AQ_F16, AQ_F32, AQ_LAYOUT_STATIC_WEIGHTS, DTYPES, TORCH_DTYPES, Layout,
                aq_decode, aq_gemm,
-               aq_gemv, aq_gemv_refine, aq_pack, aq_store_books, aq_store_create,
+               aq_gemv, aq_gemv_refine, aq_pack, aq_store_books, aq_store_create, aq_wmse,
+               wmse_workspace_bytes, aq_workspace_init,
                aq_store_device_bytes, aq_store_planes, aq_store_scales, aq_store_set_prefix,
                gemm_workspace_bytes, gemv_workspace_bytes, lib, packed_bytes,
                workspace, _stream)
@@ -199,6 +200,27 @@ class AQLinear:
         ws = self._workspace("gemm", tokens)
         aq_gemm(self.layout, m, self.planes, self.books, self.scales, x, xd, tokens, y, yd, ws)
         return y
+
+    def wmse(self, W, H, lam=None):
+        """Distortion of every prefix (Sec. 2.2 Eq. wmse-task, Sec. 5): a float64 device tensor
+        d with d[k-1] = tr[(W - W^(k)) H (W - W^(k))^T] / d_out, and d[M] = sum_k lam[k-1] d[k-1]
+        when lam (M weights) is given. W: [out][in] in the book dtype; H: [in][in] fp32 or
+        bf16 (its symmetric part is used). All prefixes must be resident."""
+        if self.resident != self.M:
+            raise ValueError("the distortion needs all %d codebooks resident" % self.M)
+        hd = AQ_F32 if H.dtype == torch.float32 else AQ_BF16 if H.dtype == torch.bfloat16 else None
+        if hd is None:
+            raise TypeError("H must be float32 or bfloat16")
+        d = torch.empty(self.M + (1 if lam is not None else 0), dtype=torch.float64,
+                        device=self.device)
+        key = ("wmse", _stream(None))
+        ws = self._ws.get(key)
+        nbytes = wmse_workspace_bytes(self.layout)
+        if ws is None or ws.numel() < nbytes:
+            ws = workspace(nbytes, self.device)
+            self._ws[key] = ws
+        aq_wmse(self.layout, W, self.planes, self.books, self.scales, H, hd, lam, d, ws)
+        return d
 
     def __call__(self, x, m):
         return self.gemv(x, m) if x.shape[0] <= 16 else self.gemm(x, m)
