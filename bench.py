@@ -329,7 +329,7 @@ def measure_wmse(lin, dev, stream, peaks, reps=10):
     peak = peaks.get("bf16_tflops", 1900.0)
     tf = mma_flops / (ms * 1e-3) / 1e12
     return {"workload": "attn_4096", "out": out, "in": inp, "M": M,
-            "compute": "bf16 tcgen05 pair MMA (E_k x folded H), fp32 accumulation, all prefixes per pass",
+            "compute": "E_k written once in bf16, then bf16 tcgen05 pair MMA (E_k x folded H), fp32 accumulation, 2 prefixes per pass",
             "ms": round(ms, 4), "mma_TFLOP_s": round(tf, 1), "frac_bf16_peak": round(tf / peak, 4),
             "definition_TFLOP_s": round(def_flops / (ms * 1e-3) / 1e12, 1),
             "mma_flops": mma_flops, "D": [round(float(v), 6) for v in d[:M].tolist()],

@@ -212,15 +212,16 @@ aq_status aq_gemm(const aq_layout* layout, int m, const void* planes, const void
  *   d       : device, M doubles, 8-byte aligned (M + 1 when lambda is given: d[M] = L);
  *             written, not accumulated; d_out = 0 gives zeros
  *   workspace : device, aq_wmse_workspace_bytes(layout) bytes, 16-byte aligned: a status word,
- *             a bf16 copy of the folded H (d_in^2 * 2 bytes) and per-CTA partial sums. Zero-
- *             fill it once before first use (aq_workspace_init); device-side waits that time
- *             out are reported through it (aq_workspace_status).
- * Computation: E_k = W - W^(k) (fp32, then rounded once to bf16) times H folded to its
- * block-lower-triangular symmetric form (bf16) on the tcgen05 tensor cores with fp32
- * accumulation, for up to four prefixes per pass; per-tile sums are added in fp64 in a fixed
- * order. Accuracy: |D - D_exact| <= 1.25e-2 * D_abs with D_abs = (1/d_out) sum_o |e_o||H||e_o|^T
- * (three bf16 roundings, first order), typically far smaller.
- * Supported: code_bits = 8. Errors: as aq_gemv (AQ_ERR_UNSUPPORTED for 16-bit codes). */
+ *             a bf16 copy of the folded H (d_in^2 * 2 bytes), the residuals E_k of every
+ *             prefix in bf16 (M * d_out * d_in * 2 bytes) and per-CTA partial sums. Zero-fill
+ *             it once before first use (aq_workspace_init); device-side waits that time out
+ *             are reported through it (aq_workspace_status).
+ * Computation: E_k = W - W^(k) (fp32, then rounded once to bf16, written to the workspace)
+ * times H folded to its block-lower-triangular symmetric form (bf16) on the tcgen05 tensor
+ * cores with fp32 accumulation, two prefixes per pass; per-tile sums are added in a fixed
+ * order. Accuracy: |D - D_exact| <= 1.25e-2 * D_abs with
+ * D_abs = (1/d_out) sum_o |e_o||H||e_o|^T (three bf16 roundings, first order), typically far
+ * smaller. Errors: as aq_gemv. */
 size_t aq_wmse_workspace_bytes(const aq_layout* layout);
 aq_status aq_wmse(const aq_layout* layout, const void* w, const void* planes, const void* books,
                   const void* scales, const void* h, int h_dtype, const double* lambda, double* d,

@@ -226,7 +226,6 @@ aq_status aq_wmse(const aq_layout* layout, const void* w, const void* planes, co
     Dims d;
     aq_status st = aq::make_dims(layout, &d);
     if (st != AQ_OK) return st;
-    if (d.B != 8) return AQ_ERR_UNSUPPORTED;
     if (h_dtype != AQ_F32 && h_dtype != AQ_BF16) return AQ_ERR_INVALID_ARG;
     if (!d_out) return AQ_ERR_INVALID_ARG;
     if (((uintptr_t)d_out & 7u) != 0) return AQ_ERR_ALIGNMENT;

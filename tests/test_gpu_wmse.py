@@ -31,10 +31,10 @@ def gpu():
     U.require_gpu()
 
 
-def _case(out, inp, M, dt, seed, noise=0.01, n_mult=2):
+def _case(out, inp, M, dt, seed, noise=0.01, n_mult=2, B=8):
     """A layer, an 'original' weight W near its full reconstruction (rounded to the book type)
     and H = X X^T / n for Gaussian X (n = n_mult * in), as float32."""
-    layer = workloads.make_layer(out, inp, G=8, M=M, B=8, book_dtype=dt, book_std=0.02,
+    layer = workloads.make_layer(out, inp, G=8, M=M, B=B, book_dtype=dt, book_std=0.02,
                                  scale_dtype=dt, seed=seed)
     rng = np.random.Generator(np.random.PCG64(seed + 1))
     W = oracle.reconstruct_exact(layer, M) + noise * rng.standard_normal((out, inp))
@@ -77,6 +77,12 @@ def test_wmse_matches_oracle(case):
     ref = _check(layer, W_bits, H, d, str(case))
     if M > 1:
         assert all(ref[k] > ref[k + 1] for k in range(M - 1)), ref   # the fixture refines
+
+
+def test_sixteen_bit_codes():
+    layer, W_bits, H = _case(160, 520, 2, "bf16", seed=8, B=16)
+    lin, W, Hd = _device(layer, W_bits, H)
+    _check(layer, W_bits, H, lin.wmse(W, Hd).cpu().numpy(), "B=16")
 
 
 def test_bf16_h_and_nonsymmetric_h():
@@ -137,7 +143,5 @@ def test_wmse_argument_errors():
     assert call(lin.layout, d_ptr=None) == aq.AQ_ERR_INVALID_ARG
     assert call(lin.layout, d_ptr=d.data_ptr() + 4) == aq.AQ_ERR_ALIGNMENT
     assert call(lin.layout, wsb=nbytes - 16) == aq.AQ_ERR_WORKSPACE
-    L16 = aq.Layout.make(64, 256, 2, B=16)
-    assert call(L16) == aq.AQ_ERR_UNSUPPORTED
     assert call(lin.layout) == aq.AQ_OK
     assert aq.aq_workspace_status(ws) == aq.AQ_OK

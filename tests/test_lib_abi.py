@@ -146,16 +146,16 @@ def test_store_argument_errors_on_the_host():
 
 def test_wmse_sizes_and_argument_errors_on_the_host():
     L = aq.Layout.make(4096, 4096, 4)
-    # status block, the folded H in bf16, one fp32 partial per CTA and prefix (2 CTAs per
-    # 256 x 128 tile: 16 x 32 tiles)
-    assert aq.wmse_workspace_bytes(L) == 1024 + 4096 * 4096 * 2 + 2 * 16 * 32 * 4 * 4
+    # status block, the folded H in bf16, E_k of the four prefixes in bf16, one fp32 partial
+    # per CTA of a pass and prefix (2 CTAs per 256 x 256 tile: 16 x 16 tiles)
+    assert aq.wmse_workspace_bytes(L) == (1024 + 4096 * 4096 * 2 + 4 * 4096 * 4096 * 2
+                                          + 2 * 16 * 16 * 4 * 4)
     lib = aq.lib()
     d8 = FAKE
     call = lambda L, hdt=aq.AQ_F32, d=d8, ws=FAKE, wsb=None: lib.aq_wmse(
         ctypes.byref(L) if L is not None else None, FAKE, FAKE, FAKE, FAKE, FAKE, hdt, None, d,
         ws, aq.wmse_workspace_bytes(L) if wsb is None and L is not None else (wsb or 0), None)
     assert call(None, wsb=0) == aq.AQ_ERR_INVALID_ARG
-    assert call(_lay(B=16)) == aq.AQ_ERR_UNSUPPORTED
     assert call(_lay(), hdt=aq.AQ_F16) == aq.AQ_ERR_INVALID_ARG
     assert call(_lay(), d=None) == aq.AQ_ERR_INVALID_ARG
     assert call(_lay(), d=FAKE + 4) == aq.AQ_ERR_ALIGNMENT
