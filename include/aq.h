@@ -186,7 +186,7 @@ aq_status aq_gemv_static_scratch(const aq_layout* layout, int m, const void* pla
  * fp32 accumulation in tensor memory; W_m is never written to HBM. The MMA operands are fp16:
  * each decoded weight (fp32 sum of the m codewords) is rounded once to fp16, and bf16
  * activations are first copied to fp16 in the workspace (exact for |x| in fp16's normal
- * range; values beyond +-65504 saturate). Supported: code_bits = 8, m <= 4.
+ * range; values beyond +-65504 saturate). Supported: code_bits = 8 (any m <= num_books <= 8).
  *   x : device, [tokens][d_in] of x_dtype (AQ_F16 or AQ_BF16); y : device, [tokens][d_out]
  *       of y_dtype (AQ_F16, AQ_BF16 or AQ_F32).
  *   workspace : aq_gemm_workspace_bytes(layout, tokens) bytes (a status word and room for the

@@ -55,34 +55,42 @@ constexpr int kPairTokens = 2 * kAcc * kBM;   // 512 tokens per pair tile
 constexpr int kRows = 128;                    // weight rows decoded by one CTA
 constexpr int kBN = 2 * kRows;                // weight rows per pair tile (N of the MMA)
 constexpr int kBK = 64;                       // inputs per stage
-constexpr int kStagesA = 4;                   // activation ring (TMA)
-constexpr int kStagesB = 3;                   // decoded-weight ring
 constexpr int kGemmThreads = 384;
 constexpr int kDecWarp0 = 4, kDecWarps = 8;
-constexpr int kGemmMaxM = 4;
+constexpr int kGemmMaxM = 8;
 
 constexpr int kABlock = kBM * 128;            // one 128-token x 64-input block (16 KiB)
 constexpr int kAStage = kAcc * kABlock;       // 32 KiB
 constexpr int kBStage = kRows * 128;          // 16 KiB
-constexpr int kCodeBuf = kGemmMaxM * kRows * 32;   // one slice of codes, all planes (16 KiB)
 
-// Shared-memory map (offsets from a 1024-byte aligned base; identical in both CTAs of a pair,
-// which the pair MMA relies on: it reads the peer's operands at the same offsets).
-constexpr int kOffA = 0;
-constexpr int kOffB = kOffA + kStagesA * kAStage;
-constexpr int kOffCodes = kOffB + kStagesB * kBStage;
-constexpr int kOffBooks = kOffCodes + 2 * kCodeBuf;
-constexpr int kOffScale = kOffBooks + kGemmMaxM * 4096;
-constexpr int kOffBar = kOffScale + kBN * 4;
-// full_a, empty_a (per A stage), full_b, empty_b, ready, dec_done (per B stage), codes_full[2],
-// codes_empty[2], acc_full
-constexpr int kNumBars = 2 * kStagesA + 4 * kStagesB + 4 + 1;
-constexpr int kOffTmem = kOffBar + kNumBars * 8;
-constexpr int kOffAbort = kOffTmem + 16;
-// The kernel has no static shared memory, so its dynamic shared memory starts on a 1024-byte
-// boundary (checked at run time: the 128-byte swizzled tiles need it).
-constexpr int kGemmSmem = kOffAbort + 16;
-static_assert(kGemmSmem <= 227 * 1024, "shared memory map exceeds the per-CTA limit");
+// Shared-memory map for prefix length MB (offsets from a 1024-byte aligned base; identical in
+// both CTAs of a pair, which the pair MMA relies on: it reads the peer's operands at the same
+// offsets). Up to four books: four activation stages, three weight stages, room for four
+// planes of codes and four codebooks. Longer prefixes need more room for codes and codebooks
+// (MB planes of 128 rows per slice, MB codebooks of 4 KiB): the activation ring drops to three
+// stages, and from seven books the weight ring to two.
+template <int MB>
+struct GemmLayout {
+    static constexpr int kBooks = MB <= 4 ? 4 : MB;
+    static constexpr int kStagesA = MB <= 4 ? 4 : 3;
+    static constexpr int kStagesB = MB <= 6 ? 3 : 2;
+    static constexpr int kCodeBuf = kBooks * kRows * 32;   // one slice of codes, all planes
+    static constexpr int kOffA = 0;
+    static constexpr int kOffB = kOffA + kStagesA * kAStage;
+    static constexpr int kOffCodes = kOffB + kStagesB * kBStage;
+    static constexpr int kOffBooks = kOffCodes + 2 * kCodeBuf;
+    static constexpr int kOffScale = kOffBooks + kBooks * 4096;
+    static constexpr int kOffBar = kOffScale + kBN * 4;
+    // full_a, empty_a (per A stage), full_b, empty_b, ready, dec_done (per B stage),
+    // codes_full[2], codes_empty[2], acc_full
+    static constexpr int kNumBars = 2 * kStagesA + 4 * kStagesB + 4 + 1;
+    static constexpr int kOffTmem = kOffBar + kNumBars * 8;
+    static constexpr int kOffAbort = kOffTmem + 16;
+    // The kernel has no static shared memory, so its dynamic shared memory starts on a
+    // 1024-byte boundary (checked at run time: the 128-byte swizzled tiles need it).
+    static constexpr int kSmem = kOffAbort + 16;
+    static_assert(kSmem <= 227 * 1024, "shared memory map exceeds the per-CTA limit");
+};
 
 __device__ __forceinline__ uint32_t pack2(float lo, float hi, int dt) {
     if (dt == AQ_BF16) {
@@ -141,8 +149,11 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
             const uint16_t* __restrict__ books, const uint16_t* __restrict__ scales, void* y,
             int y_dt, int scale_dt, unsigned int* __restrict__ status, int tokens, int out,
             int in, int ng, int rows_pad, size_t plane_bytes) {
+    using GL = GemmLayout<MB>;
+    constexpr int kStagesA = GL::kStagesA, kStagesB = GL::kStagesB, kCodeBuf = GL::kCodeBuf;
+    constexpr int kOffA = GL::kOffA, kOffB = GL::kOffB, kOffCodes = GL::kOffCodes;
     extern __shared__ __align__(1024) unsigned char smem[];
-    uint64_t* bars = (uint64_t*)(smem + kOffBar);
+    uint64_t* bars = (uint64_t*)(smem + GL::kOffBar);
     uint64_t* full_a = bars;                    // this CTA's activation copies landed
     uint64_t* empty_a = bars + kStagesA;        // the pair MMAs reading the A stage completed
     uint64_t* full_b = bars + 2 * kStagesA;     // this CTA's decoders wrote its weight half
@@ -155,11 +166,11 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
     uint64_t* codes_full = dec_done + kStagesB;
     uint64_t* codes_empty = codes_full + 2;
     uint64_t* acc_full = codes_empty + 2;
-    uint32_t* tmem_slot = (uint32_t*)(smem + kOffTmem);
-    float* scale_s = (float*)(smem + kOffScale);
-    uint4* books_s = (uint4*)(smem + kOffBooks);
+    uint32_t* tmem_slot = (uint32_t*)(smem + GL::kOffTmem);
+    float* scale_s = (float*)(smem + GL::kOffScale);
+    uint4* books_s = (uint4*)(smem + GL::kOffBooks);
     constexpr int m = MB;
-    volatile int& s_abort = *(volatile int*)(smem + kOffAbort);
+    volatile int& s_abort = *(volatile int*)(smem + GL::kOffAbort);
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     // rank = role in the pair (0: leader, issues the MMAs; 1: peer). A cluster = NP CTA pairs
@@ -545,11 +556,17 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
     const int np = gemm_pairs_per_cluster(m, tokens);
     using Kern = void (*)(const CUtensorMap, const uint8_t*, const uint16_t*, const uint16_t*,
                           void*, int, int, unsigned int*, int, int, int, int, int, size_t);
-    const Kern k1[4] = {gemm_kernel<BDT, 1, 1>, gemm_kernel<BDT, 2, 1>, gemm_kernel<BDT, 3, 1>,
-                        gemm_kernel<BDT, 4, 1>};
-    const Kern k2[4] = {nullptr, gemm_kernel<BDT, 2, 2>, gemm_kernel<BDT, 3, 2>,
-                        gemm_kernel<BDT, 4, 2>};
+    const Kern k1[kGemmMaxM] = {gemm_kernel<BDT, 1, 1>, gemm_kernel<BDT, 2, 1>, gemm_kernel<BDT, 3, 1>,
+                                gemm_kernel<BDT, 4, 1>, gemm_kernel<BDT, 5, 1>, gemm_kernel<BDT, 6, 1>,
+                                gemm_kernel<BDT, 7, 1>, gemm_kernel<BDT, 8, 1>};
+    const Kern k2[kGemmMaxM] = {nullptr, gemm_kernel<BDT, 2, 2>, gemm_kernel<BDT, 3, 2>,
+                                gemm_kernel<BDT, 4, 2>, gemm_kernel<BDT, 5, 2>, gemm_kernel<BDT, 6, 2>,
+                                gemm_kernel<BDT, 7, 2>, gemm_kernel<BDT, 8, 2>};
+    const int smem_sizes[kGemmMaxM] = {GemmLayout<1>::kSmem, GemmLayout<2>::kSmem, GemmLayout<3>::kSmem,
+                                       GemmLayout<4>::kSmem, GemmLayout<5>::kSmem, GemmLayout<6>::kSmem,
+                                       GemmLayout<7>::kSmem, GemmLayout<8>::kSmem};
     const Kern kern = (np == 2 ? k2 : k1)[m - 1];
+    const int smem = smem_sizes[m - 1];
     const int csize = 2 * np;         // CTAs per cluster
     static std::mutex mu;
     static bool attr_done[2 * kGemmMaxM][64] = {};
@@ -559,7 +576,7 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
     {
         std::lock_guard<std::mutex> lock(mu);
         if (dev >= 0 && dev < 64 && !attr_done[slot][dev]) {
-            if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
+            if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
                 e != cudaSuccess)
                 return cuda_fail(e, "cudaFuncSetAttribute");
             if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
@@ -574,7 +591,7 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
     const int tok_tile = np * kPairTokens;
     cfg.gridDim = dim3(csize * ((d.out + kBN - 1) / kBN), (tokens + tok_tile - 1) / tok_tile);
     cfg.blockDim = dim3(kGemmThreads);
-    cfg.dynamicSmemBytes = kGemmSmem;
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
