@@ -121,9 +121,9 @@ aq_status aq_decode(const aq_layout* layout, int m, const void* planes, const vo
  *   y         : device, [batch][d_out] of y_dtype (AQ_F16, AQ_BF16 or AQ_F32), row-major
  *   workspace : device scratch of at least aq_gemv_workspace_bytes(layout, batch) bytes:
  *               a status word and fp32 partial sums for every row: one per 256-input
- *               slice and token, or, with 2^8-entry books at batch 1 (batch 2..4), one per
- *               slice, token and codebook of the largest prefix up to 8 (up to 4) served
- *               that way. Zero-fill it once before its first use (aq_workspace_init); every
+ *               slice and token, or, with 2^8-entry books at batch 1..2 (batch 3..4), one
+ *               per slice, token and codebook of the largest prefix up to 8 (up to 4)
+ *               served that way. Zero-fill it once before its first use (aq_workspace_init); every
  *               call leaves it ready for the next one.
  *               Calls that may overlap on the GPU must not share a workspace.
  * Two kernels are enqueued, both with programmatic dependent launch: the product (fp32

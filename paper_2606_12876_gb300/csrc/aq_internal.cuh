@@ -40,11 +40,12 @@ constexpr size_t kWsStatusBytes = 256;
 inline size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 inline size_t ws_partial_offset(const Dims&) { return kWsStatusBytes; }
 
-// The table-lookup GEMV (2^8-entry books; batch 1 with prefixes up to kLutMaxM, batch 2..4
-// with prefixes up to kLutMultiM) writes one partial plane per (slice, book, token); every
+// The table-lookup GEMV (2^8-entry books; batch 1 and 2 with prefixes up to kLutMaxM, batch
+// 3..4 with prefixes up to kLutMultiM: their two 64 KiB tables and five or more codebooks
+// leave room for a single code stage) writes one partial plane per (slice, book, token); every
 // other GEMV one per (slice, token).
 constexpr int kLutMaxM = 8, kLutMultiM = 4;
-inline int lut_max_m(int batch) { return batch == 1 ? kLutMaxM : batch <= 4 ? kLutMultiM : 0; }
+inline int lut_max_m(int batch) { return batch <= 2 ? kLutMaxM : batch <= 4 ? kLutMultiM : 0; }
 inline bool uses_lut(const Dims& d, int m, int batch) { return d.B == 8 && m <= lut_max_m(batch); }
 
 // Records a failed CUDA call (thread-local text for aq_last_error) and returns AQ_ERR_CUDA.

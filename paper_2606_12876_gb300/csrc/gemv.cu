@@ -10,7 +10,7 @@
 // scales the row and stores y, with the rows spread evenly over the GPU.
 //
 // Three product kernels, chosen by batch, code width and prefix:
-//  * gemv_lut (B = 8; 1 token with m <= 8, or 2..4 tokens with m <= 4). By linearity,
+//  * gemv_lut (B = 8; 1 or 2 tokens with m <= 8, or 3..4 tokens with m <= 4). By linearity,
 //    x_g . (sum_k C_k[b_k]) = sum_k T_k[g][b_k] with T_k[g][j] = x_g . C_k[j]. A persistent
 //    CTA (one per SM) walks a contiguous range of work items; for each (slice, book) it builds
 //    that book's T for the 32 groups in shared memory (32 KiB per token), then every code
@@ -21,7 +21,7 @@
 //    planes into a shared-memory ring with TMA bulk copies (the CTA's rows of a slice are
 //    contiguous in every plane), overlapping HBM reads with the table build and the lookups
 //    of the sixteen consumer warps.
-//  * gemv_mma (B = 8, 5..16 tokens, m <= 4). The decoded group (fp32 sum of the m
+//  * gemv_mma (B = 8, 5..16 tokens, any m <= 8). The decoded group (fp32 sum of the m
 //    codewords, rounded once to tf32) is an A fragment of a tensor-core multiply with 8 or
 //    16 tokens of activations (mma.sync m16n8k8).
 //  * gemv_direct (any other case: 16-bit codes, larger m). Decode each group in fp32 (sum of
@@ -493,7 +493,7 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
     }
 }
 
-// ------------------------------------------------------------------ tensor-core kernel (B = 8, 2..16 tokens, m <= 4)
+// ------------------------------------------------------------------ tensor-core kernel (B = 8, 2..16 tokens)
 
 // Partials for 2..16 tokens with the multiply on the tensor cores (mma.sync m16n8k8, tf32
 // operands, fp32 accumulation). Each warp takes one 32-row block of the CTA's slice: the
@@ -506,7 +506,7 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
 // each element is added to its fp32 sum by one mixed-type add (16-bit operand, fp32 sum).
 // (Eight bank-disjoint copies of each book, which make the gathers conflict-free, measured
 // slower: at m = 3, 4 their 32 KiB per book leave one CTA per SM.)
-constexpr int kMmaMaxM = 4;       // prefixes compiled for this kernel
+constexpr int kMmaMaxM = 8;       // prefixes compiled for this kernel
 constexpr int kMmaXStride = 260;   // floats per staged token row (4 of padding: conflict-free)
 constexpr int kMmaCodeRow = 36;    // bytes per staged code row (4 of padding: conflict-free)
 
@@ -858,22 +858,23 @@ aq_status run_mma(const Dims& d, const GemvArgs& a, cudaStream_t st) {
                       d.in, d.rows_pad, d.RBc, rbpc, d.plane_bytes);
 }
 
+template <int NT, int BDT>
+aq_status dispatch_mma_nt(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
+    switch (m) {
+        case 1: return run_mma<NT, BDT, 1>(d, a, st);
+        case 2: return run_mma<NT, BDT, 2>(d, a, st);
+        case 3: return run_mma<NT, BDT, 3>(d, a, st);
+        case 4: return run_mma<NT, BDT, 4>(d, a, st);
+        case 5: return run_mma<NT, BDT, 5>(d, a, st);
+        case 6: return run_mma<NT, BDT, 6>(d, a, st);
+        case 7: return run_mma<NT, BDT, 7>(d, a, st);
+        default: return run_mma<NT, BDT, 8>(d, a, st);
+    }
+}
+
 template <int BDT>
 aq_status dispatch_mma(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
-    if (a.batch <= 8) {
-        switch (m) {
-            case 1: return run_mma<1, BDT, 1>(d, a, st);
-            case 2: return run_mma<1, BDT, 2>(d, a, st);
-            case 3: return run_mma<1, BDT, 3>(d, a, st);
-            default: return run_mma<1, BDT, 4>(d, a, st);
-        }
-    }
-    switch (m) {
-        case 1: return run_mma<2, BDT, 1>(d, a, st);
-        case 2: return run_mma<2, BDT, 2>(d, a, st);
-        case 3: return run_mma<2, BDT, 3>(d, a, st);
-        default: return run_mma<2, BDT, 4>(d, a, st);
-    }
+    return a.batch <= 8 ? dispatch_mma_nt<1, BDT>(d, m, a, st) : dispatch_mma_nt<2, BDT>(d, m, a, st);
 }
 
 template <int B, int BDT, int SDT>
