@@ -100,9 +100,7 @@ aq_status check_ptrs(std::initializer_list<const void*> ps) {
 }
 
 // GEMM workspace: status word, then room for an fp16 copy of bf16 activations.
-size_t gemm_ws_bytes(const Dims& d, int tokens) {
-    return aq::kWsStatusBytes + (size_t)tokens * (size_t)d.in * 2;
-}
+size_t gemm_ws_bytes(const Dims& d, int tokens) { return aq::gemm_ws_need(d, tokens); }
 
 size_t gemv_ws_bytes(const Dims& d, int batch) {
     // Partial planes: S per token, or S per book and token for the largest prefix the

@@ -48,6 +48,21 @@ constexpr int kLutMaxM = 8, kLutMultiM = 4;
 inline int lut_max_m(int batch) { return batch <= 2 ? kLutMaxM : batch <= 4 ? kLutMultiM : 0; }
 inline bool uses_lut(const Dims& d, int m, int batch) { return d.B == 8 && m <= lut_max_m(batch); }
 
+// Prefill GEMM workspace: [status word][fp16 copy of bf16 activations][dense W_m, fp16]. From
+// kGemmDenseTokens tokens, prefixes of two or more books decode W_m once into the workspace
+// and run the pair MMAs on it (decoding in the GEMM's inner loop is bound by shared-memory
+// gathers, and at that length every weight tile is decoded again for every 512 tokens).
+constexpr int kGemmDenseTokens = 2048;
+inline bool gemm_uses_dense(int m, int tokens) { return m >= 2 && tokens >= kGemmDenseTokens; }
+inline size_t gemm_w16_offset(const Dims& d, int tokens) {
+    return round_up(kWsStatusBytes + (size_t)tokens * (size_t)d.in * 2, 1024);
+}
+inline size_t gemm_ws_need(const Dims& d, int tokens) {
+    if (d.B == 8 && d.M >= 2 && tokens >= kGemmDenseTokens)
+        return gemm_w16_offset(d, tokens) + (size_t)d.out * (size_t)d.in * 2;
+    return kWsStatusBytes + (size_t)tokens * (size_t)d.in * 2;
+}
+
 // Records a failed CUDA call (thread-local text for aq_last_error) and returns AQ_ERR_CUDA.
 aq_status cuda_fail(cudaError_t e, const char* what);
 // AQ_OK if e is cudaSuccess, else cuda_fail(e, what).

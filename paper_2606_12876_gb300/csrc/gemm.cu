@@ -143,12 +143,19 @@ __device__ __forceinline__ uint4 decode_group(uint32_t books, const uint32_t (&c
 // own 128 rows. Sharing pays when the gathers bound the kernel (m >= 2) and every pair has
 // tokens; larger clusters leave more SMs idle (36 clusters of four, or fewer of eight, fit on
 // the 152 SMs), which at m = 1 costs more than the decode they save.
-template <int BDT, int MB, int NP>
+//
+// DENSE: the weights were decoded beforehand (dense_w_kernel: fp16 sums of the m codewords,
+// the same values the decoders would write) and each CTA's weight tile arrives by TMA (wmap,
+// 128-byte swizzle, the layout the decoders write) like the activations; the decoder warps
+// only run the epilogue. Instantiated with MB = NP = 1.
+template <int BDT, int MB, int NP, bool DENSE = false>
 __global__ void __launch_bounds__(kGemmThreads, 1)
-gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ planes,
+gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
+            const uint8_t* __restrict__ planes,
             const uint16_t* __restrict__ books, const uint16_t* __restrict__ scales, void* y,
             int y_dt, int scale_dt, unsigned int* __restrict__ status, int tokens, int out,
             int in, int ng, int rows_pad, size_t plane_bytes) {
+    static_assert(!DENSE || (MB == 1 && NP == 1), "dense tiles: one instantiation");
     using GL = GemmLayout<MB>;
     constexpr int kStagesA = GL::kStagesA, kStagesB = GL::kStagesB, kCodeBuf = GL::kCodeBuf;
     constexpr int kOffA = GL::kOffA, kOffB = GL::kOffB, kOffCodes = GL::kOffCodes;
@@ -184,10 +191,24 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
     constexpr int kSlab = DR * 128;             // their 64-input slab of a weight stage
     const uint32_t rank4 = cluster_rank();
     const uint32_t rank = rank4 & 1u, pair = SHARE ? rank4 >> 1 : 0u;
-    const int n0 = (blockIdx.x >> kClusterLog) * kBN;   // first output row of the pair tile
+    // Tile of the cluster: row tile tn, token tile tt. With decoding in the loop the grid runs
+    // all row tiles of one token tile together (blockIdx.x fastest); the dense variant reads
+    // 2 bytes of weight per element instead of m/8 of codes, so there the clusters of one row
+    // tile run together and its weight tiles are read from HBM once and then from L2.
+    int tn, tt;
+    if constexpr (DENSE) {
+        const int ntt = (int)gridDim.y;
+        const int cid = (int)blockIdx.y * (int)(gridDim.x >> kClusterLog) + (int)(blockIdx.x >> kClusterLog);
+        tn = cid / ntt;
+        tt = cid - tn * ntt;
+    } else {
+        tn = (int)(blockIdx.x >> kClusterLog);
+        tt = (int)blockIdx.y;
+    }
+    const int n0 = tn * kBN;                    // first output row of the pair tile
     const int r0 = n0 + (int)rank * kRows;      // first row of this CTA's weight operand
     const int rd0 = r0 + (int)pair * DR;        // first row decoded by this CTA
-    const int t0 = (blockIdx.y * NP + (int)pair) * kPairTokens;   // first token
+    const int t0 = (tt * NP + (int)pair) * kPairTokens;   // first token
     const int nk = (in + kBK - 1) / kBK;        // K steps
     const int nsl = (nk + 3) / 4;               // 256-input slices
     const int rows_valid = max(0, min(DR, rows_pad - rd0));   // packed rows present
@@ -196,7 +217,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
     // pair therefore starts at its own 256-input slice and wraps around (only the fp32
     // accumulation order differs). Every role walks the slices in this order; `it` counts
     // stages in processing order and drives the ring.
-    const int rot = (blockIdx.x >> kClusterLog) % nsl;   // the same in both pairs of a cluster
+    const int rot = tn % nsl;                   // the same in both pairs of a cluster
 
     // Same answer in both CTAs of the pair (identical layouts), so both leave before any
     // cluster-wide step.
@@ -211,10 +232,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
         }
         for (int s = 0; s < kStagesB; ++s) {
             // (peer) the copier with the partner's bytes, or the decoder warps
-            mbar_init(&full_b[s], SHARE ? 1 : kDecWarps);
+            mbar_init(&full_b[s], (SHARE || DENSE) ? 1 : kDecWarps);
             mbar_init(&empty_b[s], NP);           // commits of the pairs writing the stage
             // (leader) the copier or the decoder warps, plus the two relays
-            mbar_init(&ready[s], SHARE ? 3 : kDecWarps + 2);
+            mbar_init(&ready[s], DENSE ? 2 : SHARE ? 3 : kDecWarps + 2);
             mbar_init(&dec_done[s], kDecWarps);   // (SHARE) one arrival per decoder warp
         }
         for (int c = 0; c < 2; ++c) {
@@ -241,20 +262,23 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
         // ---------------- producer
         if (lane == 0) {
             asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&xmap) : "memory");
+            if constexpr (DENSE) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&wmap) : "memory");
             int issued_a = 0, issued_c = 0;
             bool stop = false;
             for (int js = 0; js < nsl && !stop; ++js) {
                 const int sl = rot + js < nsl ? rot + js : rot + js - nsl;
-                const int cb = js & 1;                    // codes of slice sl
-                if (js >= 2 && !wait_or_abort(&codes_empty[cb], ((js >> 1) - 1) & 1, &s_abort, status))
-                    break;
-                mbar_arrive_expect_tx(&codes_full[cb], (uint32_t)(m * rows_valid * 32));
-                if (rows_valid > 0)
-                    for (int k = 0; k < m; ++k)
-                        bulk_g2s(smem + kOffCodes + cb * kCodeBuf + k * (DR * 32),
-                                 planes + (size_t)k * plane_bytes + ((size_t)sl * rows_pad + rd0) * 32,
-                                 (uint32_t)(rows_valid * 32), &codes_full[cb]);
-                ++issued_c;
+                if constexpr (!DENSE) {
+                    const int cb = js & 1;                // codes of slice sl
+                    if (js >= 2 && !wait_or_abort(&codes_empty[cb], ((js >> 1) - 1) & 1, &s_abort, status))
+                        break;
+                    mbar_arrive_expect_tx(&codes_full[cb], (uint32_t)(m * rows_valid * 32));
+                    if (rows_valid > 0)
+                        for (int k = 0; k < m; ++k)
+                            bulk_g2s(smem + kOffCodes + cb * kCodeBuf + k * (DR * 32),
+                                     planes + (size_t)k * plane_bytes + ((size_t)sl * rows_pad + rd0) * 32,
+                                     (uint32_t)(rows_valid * 32), &codes_full[cb]);
+                    ++issued_c;
+                }
                 const int nj = min(4, nk - sl * 4);
                 for (int j = 0; j < nj; ++j) {
                     const int it = issued_a, st = it % kStagesA;
@@ -269,12 +293,27 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
                     for (int i = 0; i < kAcc; ++i)
                         tma_load_2d(a + i * kABlock, &xmap, (sl * 4 + j) * kBK,
                                     t0 + i * 2 * kBM + (int)rank * kBM, &full_a[st]);
+                    if constexpr (DENSE) {
+                        // this CTA's 128 weight rows of the stage, into the weight ring
+                        const int sb = it % kStagesB;
+                        if (it >= kStagesB &&
+                            !wait_or_abort(&empty_b[sb], ((it / kStagesB) - 1) & 1, &s_abort, status)) {
+                            stop = true;
+                            ++issued_a;
+                            break;
+                        }
+                        mbar_arrive_expect_tx(&full_b[sb], (uint32_t)kBStage);
+                        tma_load_2d(smem + kOffB + sb * kBStage, &wmap, (sl * 4 + j) * kBK, r0, &full_b[sb]);
+                    }
                     ++issued_a;
                 }
             }
             // No copy may still be in flight when the CTA exits.
             for (int j = max(0, issued_a - kStagesA); j < issued_a; ++j)
                 mbar_wait(&full_a[j % kStagesA], (j / kStagesA) & 1);
+            if constexpr (DENSE)
+                for (int j = max(0, issued_a - kStagesB); j < issued_a; ++j)
+                    mbar_wait(&full_b[j % kStagesB], (j / kStagesB) & 1);
             for (int j = max(0, issued_c - 2); j < issued_c; ++j)
                 mbar_wait(&codes_full[j & 1], (j >> 1) & 1);
         }
@@ -327,6 +366,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
                     !wait_or_abort(&ready[sb], ((it / kStagesB) - 1) & 1, &s_abort, status))
                     break;
                 if (!wait_or_abort(&full_a[sa], (it / kStagesA) & 1, &s_abort, status)) break;
+                if constexpr (DENSE)
+                    if (!wait_or_abort(&full_b[sb], (it / kStagesB) & 1, &s_abort, status)) break;
                 mbar_arrive(&ready[sb]);
             }
         }
@@ -361,8 +402,9 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
         const int c0 = cs * GPT;
         const int row = rd0 + n;
         const int nn = (int)pair * DR + n;          // its row in the weight operand tile
-        for (int i = dt; i < m * 256; i += kDecWarps * 32)
-            books_s[i] = __ldg((const uint4*)books + i);
+        if constexpr (!DENSE)
+            for (int i = dt; i < m * 256; i += kDecWarps * 32)
+                books_s[i] = __ldg((const uint4*)books + i);
         for (int i = dt; i < kBN; i += kDecWarps * 32)
             scale_s[i] = (n0 + i < out) ? bits_to_f32_rt(scales[n0 + i], scale_dt) : 0.0f;
         named_barrier(1, kDecWarps * 32);
@@ -373,7 +415,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict_
         const uint32_t books_u = smem_u32(books_s);
         const uint32_t b_tile = smem_u32(smem + kOffB) + (nn >> 3) * 1024 + (nn & 7) * 128;
         int it = 0;                                 // stages decoded so far (ring position)
-        for (int js = 0; js < nsl; ++js) {
+        for (int js = 0; js < (DENSE ? 0 : nsl); ++js) {
             const int sl = rot + js < nsl ? rot + js : rot + js - nsl;
             const int cb = js & 1;
             // q[k][j]: the word holding the codes (one byte each) of the thread's groups
@@ -554,7 +596,7 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
     // Pairs per cluster sharing the decode: sharing pays where the gathers bound the kernel
     // (m >= 2) and every pair of a cluster has tokens (one 512-token tile per pair).
     const int np = gemm_pairs_per_cluster(m, tokens);
-    using Kern = void (*)(const CUtensorMap, const uint8_t*, const uint16_t*, const uint16_t*,
+    using Kern = void (*)(const CUtensorMap, const CUtensorMap, const uint8_t*, const uint16_t*, const uint16_t*,
                           void*, int, int, unsigned int*, int, int, int, int, int, size_t);
     const Kern k1[kGemmMaxM] = {gemm_kernel<BDT, 1, 1>, gemm_kernel<BDT, 2, 1>, gemm_kernel<BDT, 3, 1>,
                                 gemm_kernel<BDT, 4, 1>, gemm_kernel<BDT, 5, 1>, gemm_kernel<BDT, 6, 1>,
@@ -602,10 +644,155 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
     attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    return cuda_ok(cudaLaunchKernelEx(&cfg, kern, map, (const uint8_t*)planes,
+    CUtensorMap unused;                 // the weight map is read only by the dense variant
+    std::memset(&unused, 0, sizeof(unused));
+    return cuda_ok(cudaLaunchKernelEx(&cfg, kern, map, unused, (const uint8_t*)planes,
                                       (const uint16_t*)books, (const uint16_t*)scales, y, y_dt,
                                       d.scale_dt, (unsigned int*)ws, tokens, d.out, d.in, d.ng,
                                       d.rows_pad, d.plane_bytes),
+                   "cudaLaunchKernelEx");
+}
+
+// ---- dense variant: W_m decoded once into the workspace, then TMA-fed pair MMAs -----------
+
+// W16[o][i] = fp16(sum_{k<m} C_k[b_k[o, i/8]][i mod 8]): the unscaled fp32 sum of the m
+// codewords in book order, rounded once to fp16 (the values the GEMM's decoders write; the
+// epilogue applies the row scale). Each warp owns one 32-row block of one 256-input slice:
+// lane L stages its row's codes of the m planes, then the warp walks the 32 rows with lane L
+// producing group s*32 + L, so every store is 512 contiguous bytes.
+constexpr int kDenseWarps = 8;
+
+template <int BDT>
+__global__ void __launch_bounds__(kDenseWarps * 32)
+dense_w_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
+               uint16_t* __restrict__ w16, int m, int out, int in, int ng, int rows_pad, int RBc,
+               size_t plane_bytes) {
+    extern __shared__ __align__(16) unsigned char smem_d[];
+    uint4* books_s = (uint4*)smem_d;                 // [m][256] codewords
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    unsigned char* codes_s = smem_d + (size_t)m * 4096 + (size_t)warp * m * 32 * 32;
+    pdl_wait();
+    pdl_launch_dependents();
+    for (int i = threadIdx.x; i < m * 256; i += blockDim.x) books_s[i] = __ldg((const uint4*)books + i);
+    const int s = blockIdx.y;
+    const int rb = blockIdx.x * kDenseWarps + warp;
+    const bool active = rb < RBc;
+    if (active) {
+        const int o = rb * 32 + lane;
+        for (int k = 0; k < m; ++k) {
+            const uint4* src = (const uint4*)(planes + k * plane_bytes + ((size_t)s * rows_pad + o) * 32);
+            uint4* dst = (uint4*)(codes_s + ((size_t)k * 32 + lane) * 32);
+            dst[0] = ld_stream_v4(src);
+            dst[1] = ld_stream_v4(src + 1);
+        }
+    }
+    __syncthreads();
+    const int g = s * 32 + lane;
+    if (!active || g >= ng) return;
+    const uint32_t books_u = smem_u32(books_s);
+    for (int r = 0; r < 32; ++r) {
+        const int o = rb * 32 + r;
+        if (o >= out) break;
+        const int p = (lane - r) & 31;               // position of group `lane` in row o
+        float a[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) a[e] = -0.0f;
+        for (int k = 0; k < m; ++k) {
+            const uint32_t code = codes_s[((size_t)k * 32 + r) * 32 + p];
+            const uint4 c = lds128(books_u + ((uint32_t)k << 12) + (code << 4));
+            add_widen2<BDT>(c.x, a[0], a[1]);
+            add_widen2<BDT>(c.y, a[2], a[3]);
+            add_widen2<BDT>(c.z, a[4], a[5]);
+            add_widen2<BDT>(c.w, a[6], a[7]);
+        }
+        *(uint4*)(w16 + (size_t)o * in + (size_t)g * 8) =
+            make_uint4(f16x2(make_float2(a[0], a[1])), f16x2(make_float2(a[2], a[3])),
+                       f16x2(make_float2(a[4], a[5])), f16x2(make_float2(a[6], a[7])));
+    }
+}
+
+template <int BDT>
+aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* books,
+                         const void* scales, const void* x, int tokens, void* y, int y_dt,
+                         void* ws, uint16_t* w16, cudaStream_t st) {   // x: fp16 [tokens][in]
+    {   // decode W_m once
+        const size_t smem = (size_t)m * 4096 + (size_t)kDenseWarps * m * 32 * 32;
+        auto kern = dense_w_kernel<BDT>;
+        if (smem > 48 * 1024)
+            if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+                e != cudaSuccess)
+                return cuda_fail(e, "cudaFuncSetAttribute");
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((d.RBc + kDenseWarps - 1) / kDenseWarps, d.S);
+        cfg.blockDim = dim3(kDenseWarps * 32);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = st;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (aq_status e = cuda_ok(cudaLaunchKernelEx(&cfg, kern, (const uint8_t*)planes, (const uint16_t*)books,
+                                                     w16, m, d.out, d.in, d.ng, d.rows_pad, d.RBc, d.plane_bytes),
+                                  "cudaLaunchKernelEx");
+            e != AQ_OK)
+            return e;
+    }
+    EncodeTiledFn encode;
+    if (aq_status e = get_encode_fn(&encode); e != AQ_OK) return e;
+    CUtensorMap xm, wm;
+    std::memset(&xm, 0, sizeof(xm));
+    std::memset(&wm, 0, sizeof(wm));
+    const cuuint64_t strides[1] = {(cuuint64_t)d.in * 2};
+    const cuuint32_t estr[2] = {1, 1};
+    {
+        const cuuint64_t dims[2] = {(cuuint64_t)d.in, (cuuint64_t)tokens};
+        const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)kBM};
+        if (encode(&xm, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(x), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return AQ_ERR_CUDA;
+    }
+    {
+        const cuuint64_t dims[2] = {(cuuint64_t)d.in, (cuuint64_t)d.out};
+        const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)kRows};
+        if (encode(&wm, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, (void*)w16, dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return AQ_ERR_CUDA;
+    }
+    auto kern = gemm_kernel<BDT, 1, 1, true>;
+    constexpr int smem = GemmLayout<1>::kSmem;
+    static std::mutex mu;
+    static bool attr_done[64] = {};
+    int dev = 0;
+    if (cudaError_t e = cudaGetDevice(&dev); e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+            if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+                e != cudaSuccess)
+                return cuda_fail(e, "cudaFuncSetAttribute");
+            attr_done[dev] = true;
+        }
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * ((d.out + kBN - 1) / kBN), (tokens + kPairTokens - 1) / kPairTokens);
+    cfg.blockDim = dim3(kGemmThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = 2;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cuda_ok(cudaLaunchKernelEx(&cfg, kern, xm, wm, (const uint8_t*)planes, (const uint16_t*)books,
+                                      (const uint16_t*)scales, y, y_dt, d.scale_dt, (unsigned int*)ws,
+                                      tokens, d.out, d.in, d.ng, d.rows_pad, d.plane_bytes),
                    "cudaLaunchKernelEx");
 }
 
@@ -640,6 +827,12 @@ aq_status launch_gemm(const Dims& d, int m, const void* planes, const void* book
             e != AQ_OK)
             return e;
         xh = dst;
+    }
+    if (gemm_uses_dense(m, tokens)) {
+        uint16_t* w16 = (uint16_t*)((char*)ws + gemm_w16_offset(d, tokens));
+        return d.book_dt == AQ_BF16
+                   ? run_gemm_dense<AQ_BF16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, w16, st)
+                   : run_gemm_dense<AQ_F16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, w16, st);
     }
     return d.book_dt == AQ_BF16
                ? run_gemm<AQ_BF16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, st)

@@ -49,6 +49,24 @@ def test_gemm_matches_oracle(case, y_dtype):
         U.assert_product_close(U.to_f64(y), oracle.product_exact(layer, xb, dt, m), "m=%d" % m)
 
 
+@pytest.mark.parametrize("case", [(2100, 300, 520, 5, "bf16"), (2048, 256, 1032, 3, "f16")],
+                         ids=lambda c: "x".join(map(str, c)))
+def test_gemm_dense_path_long_inputs(case):
+    """From 2048 tokens, prefixes of two or more books decode W_m once into the workspace
+    (fp16) and run TMA-fed pair MMAs on it: every prefix within the product tolerance."""
+    tok, out, inp, M, dt = case
+    layer = workloads.make_layer(out, inp, G=8, M=M, B=8, book_dtype=dt, book_std=0.05,
+                                 scale_dtype=dt, seed=tok + M)
+    lin = AQLinear.from_layer(layer)
+    xb = workloads.make_x(tok, inp, dt, seed=8)
+    x = x_to_device(xb, dt)
+    rows = np.r_[0:64, tok // 2:tok // 2 + 64, tok - 64:tok]
+    for m in range(1, M + 1):
+        y = lin.gemm(x, m, y_dtype=aq.AQ_F32)
+        ys = U.to_f64(y[torch.as_tensor(rows, device="cuda")])
+        U.assert_product_close(ys, oracle.product_exact(layer, xb[rows], dt, m), "m=%d" % m)
+
+
 def test_gemm_mixed_activation_and_book_types():
     """bf16 activations with fp16 books, and fp16 activations with bf16 books."""
     for bd, xd in (("f16", "bf16"), ("bf16", "f16")):

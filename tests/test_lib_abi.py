@@ -162,3 +162,14 @@ def test_wmse_sizes_and_argument_errors_on_the_host():
     assert call(_lay(), ws=None) == aq.AQ_ERR_WORKSPACE
     assert call(_lay(), wsb=aq.wmse_workspace_bytes(_lay()) - 16) == aq.AQ_ERR_WORKSPACE
     assert call(_lay(), ws=FAKE + 8) == aq.AQ_ERR_ALIGNMENT
+
+
+def test_gemm_workspace_sizes():
+    """Status word + fp16 activation copy; from 2048 tokens (two or more books) also room for
+    W_m decoded once in fp16."""
+    L = aq.Layout.make(300, 520, 4)
+    assert aq.gemm_workspace_bytes(L, 2047) == 256 + 2047 * 520 * 2
+    off = (256 + 2048 * 520 * 2 + 1023) // 1024 * 1024
+    assert aq.gemm_workspace_bytes(L, 2048) == off + 300 * 520 * 2
+    L1 = aq.Layout.make(300, 520, 1)
+    assert aq.gemm_workspace_bytes(L1, 4096) == 256 + 4096 * 520 * 2
