@@ -236,7 +236,7 @@ def measure_gemm(dev, stream, peaks, reps=5, tokens=4096):
     dense_ms = timed(lambda: torch.matmul(x, wd.t()))
     del wd
     return {"workload": name, "tokens": tokens, "out": out, "in": inp, "M": 4,
-            "compute": "fp16 tcgen05 MMA, fp32 accumulation, weights decoded in shared memory",
+            "compute": "fp16 tcgen05 pair MMA, fp32 accumulation; weights decoded in shared memory (m = 1), or W_m decoded once in fp16 and loaded by TMA (m >= 2 at 2048+ tokens)",
             "per_m": rows, "dense_bf16_torch_ms": round(dense_ms, 4),
             "dense_bf16_TFLOP_s": round(flops / (dense_ms * 1e-3) / 1e12, 1),
             "peak_TFLOP_s": peak, "peak_source": "measured" if "bf16_tflops" in peaks else "fallback"}
