@@ -192,8 +192,8 @@ def pack(layer):
     _codes_ok(codes, B)
     rows_pad = (out + 31) // 32 * 32
     ng_pad = (inp // G + 31) // 32 * 32
-    esz = 1 if B <= 8 else 2
-    buf = np.zeros(M * rows_pad * ng_pad * esz, dtype=np.uint8)
+    nbytes = M * rows_pad * ng_pad * (1 if B <= 8 else 2) // (2 if B <= 4 else 1)
+    buf = np.zeros(nbytes, dtype=np.uint8)
     rc = lib().oracle_pack(out, inp, G, M, B, _p(codes), _p(buf))
     if rc:
         raise ValueError("oracle_pack rejected the shape")

@@ -254,8 +254,10 @@ int oracle_product_dense(int out, int in, const uint16_t* w, int w_dtype, const 
 //   planes are a prefix of the buffer. Inside a plane the order is [slice][row][position],
 //   32 positions per (slice,row); position p of row o in slice s holds the code of group
 //   s*32 + ((p + o) mod 32). Padding rows and groups hold code 0.
-// Element size is 1 byte for B <= 8 and 2 bytes for B <= 16. planes must hold
-// M*rows_pad*ng_pad elements.
+// Element size is 1 byte for 4 < B <= 8 and 2 bytes for B <= 16; for B <= 4 two codes
+// share a byte: position p lives in byte p / 2 of its (slice, row) unit, in the low four bits
+// for even p and the high four bits for odd p (a unit is then 16 bytes). planes must hold
+// M*rows_pad*ng_pad codes.
 int oracle_pack(int out, int in, int G, int M, int B, const void* codes, void* planes) {
     if (out < 0 || in < 0 || G <= 0 || M <= 0 || B <= 0 || B > 16 || in % G) return 1;
     const long ng = in / G;
@@ -263,6 +265,7 @@ int oracle_pack(int out, int in, int G, int M, int B, const void* codes, void* p
     const long ng_pad = (ng + 31) / 32 * 32;
     const long plane = rows_pad * ng_pad;
     const long S = ng_pad / 32;
+    if (B <= 4) std::memset(planes, 0, (size_t)(M * plane / 2));
     for (long k = 0; k < M; ++k)
         for (long s = 0; s < S; ++s)
             for (long o = 0; o < rows_pad; ++o)
@@ -271,7 +274,8 @@ int oracle_pack(int out, int in, int G, int M, int B, const void* codes, void* p
                     uint32_t v = 0;
                     if (o < out && g < ng) v = code_at(codes, B, (o * ng + g) * M + k);
                     const long dst = k * plane + (s * rows_pad + o) * 32 + p;
-                    if (B <= 8) ((uint8_t*)planes)[dst] = (uint8_t)v;
+                    if (B <= 4) ((uint8_t*)planes)[dst / 2] |= (uint8_t)((v & 15u) << (4 * (p % 2)));
+                    else if (B <= 8) ((uint8_t*)planes)[dst] = (uint8_t)v;
                     else ((uint16_t*)planes)[dst] = (uint16_t)v;
                 }
     return 0;

@@ -433,6 +433,32 @@ def pin_pack_positions():
                     assert planes[k, s, o, p] == want
 
 
+def pin_pack_positions_4bit():
+    """4-bit codes: two per byte, position p of a (slice, row) unit in byte p // 2, low four
+    bits for even p; the row rotation as for wider codes. Written out with plain loops."""
+    out, inp, M = 37, 520, 3
+    ng = inp // 8
+    codes = np.zeros((out, ng, M), np.uint8)
+    for o in range(out):
+        for g in range(ng):
+            for k in range(M):
+                codes[o, g, k] = (3 * o + 5 * g + 7 * k) % 16
+    layer = dict(out=out, **{"in": inp}, G=8, M=M, B=4, codes=codes)
+    planes = oracle.pack(layer)
+    rows_pad, ng_pad = 64, 96
+    assert planes.size == M * rows_pad * ng_pad // 2
+    planes = planes.reshape(M, ng_pad // 32, rows_pad, 16)
+    for k in range(M):
+        for s in range(ng_pad // 32):
+            for o in range(rows_pad):
+                for p in range(32):
+                    g = s * 32 + (p + o) % 32
+                    want = int(codes[o, g, k]) if (o < out and g < ng) else 0
+                    byte = int(planes[k, s, o, p // 2])
+                    got = (byte >> (4 * (p % 2))) & 15
+                    assert got == want, (k, s, o, p)
+
+
 def pin_pack_prefix_property():
     """The first m planes of a packed M-book layer equal the packed m-book truncation."""
     layer = workloads.make_layer(40, 272, G=8, M=4, B=8, seed=2)

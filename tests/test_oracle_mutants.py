@@ -30,6 +30,7 @@ MUTANTS = [
      "sum += bits_to_double(x[t * in + (in - 1 - i)], x_dtype) * wrow[i];"),
     ("pack_rotation_wrong", "((p + o) % 32)", "((p + 32 - o % 32) % 32)"),
     ("avg_bits_without_M", "(double)M * (double)d_out", "(double)d_out"),
+    ("pack_4bit_nibble_order", "<< (4 * (p % 2))", "<< (4 * (1 - p % 2))"),
     ("reconstruct_drops_scale", "w_out[o * in + g * G + e] = s * acc;",
      "w_out[o * in + g * G + e] = acc;"),
 ]
