@@ -55,7 +55,7 @@ typedef struct aq_layout {
     int32_t in_features;    /* d_in >= 8, a multiple of group_size */
     int32_t group_size;     /* g; only 8 is supported */
     int32_t num_books;      /* M, 1..8 */
-    int32_t code_bits;      /* B; 8 (uint8 codes) or 16 (uint16 codes) */
+    int32_t code_bits;      /* B; 4 (two codes per byte), 8 (uint8 codes) or 16 (uint16) */
     int32_t book_dtype;     /* AQ_F16 or AQ_BF16: element type of the codebooks */
     int32_t scale_dtype;    /* AQ_F16 or AQ_BF16: element type of the scales */
     int32_t flags;          /* 0 or AQ_LAYOUT_STATIC_WEIGHTS */
@@ -88,7 +88,11 @@ const char* aq_last_error(void);
  *   Position p of row o in slice s holds the code of group s*32 + ((p + o) mod 32): each
  *   row's 32 codes of a slice are rotated by the row index, so 32 consecutive rows read a
  *   position p together touch 32 different groups. Padding rows/groups hold code 0.
- *   Plane k starts at byte k*aq_plane_bytes(); the first m planes are a contiguous prefix. */
+ *   Plane k starts at byte k*aq_plane_bytes(); the first m planes are a contiguous prefix.
+ *   4-bit codes (B = 4, the 16-entry codebooks of the paper's 4x4-bit ablation, App. G.1)
+ *   share bytes: position p of a (slice, row) unit is in byte p/2, in the low four bits for
+ *   even p and the high four bits for odd p, so a unit is 16 bytes and a plane
+ *   rows_pad*ng_pad/2 bytes. */
 
 /* Bytes of one code plane; 0 if the layout is invalid. */
 size_t aq_plane_bytes(const aq_layout* layout);
@@ -97,7 +101,7 @@ size_t aq_plane_bytes(const aq_layout* layout);
 size_t aq_packed_bytes(const aq_layout* layout, int m);
 
 /* Pack natural codes into planes (the codes b_{i,j,m} of Sec. 3.2).
- *   codes  : device, (d_out, d_in/8, M) row-major, uint8 (B = 8) or uint16 (B = 16);
+ *   codes  : device, (d_out, d_in/8, M) row-major, uint8 (B = 4, 8) or uint16 (B = 16);
  *            code values must be < 2^B.
  *   planes : device, aq_packed_bytes(layout, M) bytes, fully written (padding = 0). */
 aq_status aq_pack(const aq_layout* layout, const void* codes, void* planes, void* stream);
@@ -187,11 +191,13 @@ aq_status aq_gemv_static_scratch(const aq_layout* layout, int m, const void* pla
  * see workspace below). The MMA operands are fp16:
  * each decoded weight (fp32 sum of the m codewords) is rounded once to fp16, and bf16
  * activations are first copied to fp16 in the workspace (exact for |x| in fp16's normal
- * range; values beyond +-65504 saturate). Supported: code_bits = 8 (any m <= num_books <= 8).
+ * range; values beyond +-65504 saturate). Supported: code_bits = 8 and 4 (4-bit layouts always
+ * decode W_m into the workspace first), any m <= num_books <= 8.
  *   x : device, [tokens][d_in] of x_dtype (AQ_F16 or AQ_BF16); y : device, [tokens][d_out]
  *       of y_dtype (AQ_F16, AQ_BF16 or AQ_F32).
  *   workspace : aq_gemm_workspace_bytes(layout, tokens) bytes (a status word, room for the
- *               fp16 activation copy and, from 2048 tokens when num_books >= 2, room for W_m
+ *               fp16 activation copy and, from 2048 tokens when num_books >= 2 (for 4-bit
+ *               codes always), room for W_m
  *               decoded once in fp16, d_out*d_in*2 bytes: at that length calls with m >= 2
  *               decode W_m into it and multiply by TMA-fed tensor-core tiles, which is faster
  *               than decoding every weight tile again for every 512 tokens), zero-filled

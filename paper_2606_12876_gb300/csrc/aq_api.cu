@@ -17,7 +17,7 @@ aq_status make_dims(const aq_layout* L, Dims* d) {
         (L->scale_dtype != AQ_F16 && L->scale_dtype != AQ_BF16))
         return AQ_ERR_INVALID_ARG;
     if (L->group_size != 8) return AQ_ERR_UNSUPPORTED;
-    if (L->code_bits != 8 && L->code_bits != 16) return AQ_ERR_UNSUPPORTED;
+    if (L->code_bits != 4 && L->code_bits != 8 && L->code_bits != 16) return AQ_ERR_UNSUPPORTED;
     if (L->num_books > 8) return AQ_ERR_UNSUPPORTED;
     d->out = L->out_features;
     d->in = L->in_features;
@@ -33,9 +33,9 @@ aq_status make_dims(const aq_layout* L, Dims* d) {
     d->S = d->ng_pad / 32;
     d->rows_pad = (int)(((long long)d->out + 31) / 32 * 32);
     d->RBc = d->rows_pad / 32;
-    d->esz = d->B / 8;
+    d->esz = d->B / 8;                  // 0 for 4-bit codes (two per byte)
     d->plane_elems = (size_t)d->rows_pad * (size_t)d->ng_pad;
-    d->plane_bytes = d->plane_elems * d->esz;
+    d->plane_bytes = d->plane_elems * (size_t)d->B / 8;
     return AQ_OK;
 }
 

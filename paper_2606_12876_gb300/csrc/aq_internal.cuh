@@ -20,7 +20,7 @@ struct Dims {
     int S;         // slices of 32 groups
     int rows_pad;  // out rounded up to 32
     int RBc;       // 32-row blocks, rows_pad/32
-    int esz;       // bytes per code (1 or 2)
+    int esz;       // bytes per code (1 or 2; 0 for 4-bit codes, two per byte)
     size_t plane_elems, plane_bytes;
 };
 
@@ -52,13 +52,16 @@ inline bool uses_lut(const Dims& d, int m, int batch) { return d.B == 8 && m <= 
 // kGemmDenseTokens tokens, prefixes of two or more books decode W_m once into the workspace
 // and run the pair MMAs on it (decoding in the GEMM's inner loop is bound by shared-memory
 // gathers, and at that length every weight tile is decoded again for every 512 tokens).
+// 4-bit layouts always take the dense form (the in-loop decoders read 8-bit codes).
 constexpr int kGemmDenseTokens = 2048;
-inline bool gemm_uses_dense(int m, int tokens) { return m >= 2 && tokens >= kGemmDenseTokens; }
+inline bool gemm_uses_dense(const Dims& d, int m, int tokens) {
+    return d.B == 4 || (m >= 2 && tokens >= kGemmDenseTokens);
+}
 inline size_t gemm_w16_offset(const Dims& d, int tokens) {
     return round_up(kWsStatusBytes + (size_t)tokens * (size_t)d.in * 2, 1024);
 }
 inline size_t gemm_ws_need(const Dims& d, int tokens) {
-    if (d.B == 8 && d.M >= 2 && tokens >= kGemmDenseTokens)
+    if (d.B == 4 || (d.B == 8 && d.M >= 2 && tokens >= kGemmDenseTokens))
         return gemm_w16_offset(d, tokens) + (size_t)d.out * (size_t)d.in * 2;
     return kWsStatusBytes + (size_t)tokens * (size_t)d.in * 2;
 }
@@ -250,6 +253,21 @@ __device__ __forceinline__ void unrotate_codes(const uint32_t (&w)[8], int o, ui
     for (int i = 0; i < 8; ++i) t[i] = (rw & 4) ? v[(i + 4) & 7] : v[i];
 #pragma unroll
     for (int j = 0; j < 8; ++j) u[j] = rb ? __funnelshift_l(t[(j + 7) & 7], t[j], rb) : t[j];
+}
+
+// Bytes of one (row, slice) unit of a code plane: 32 codes of B bits (B = 4, 8 or 16).
+constexpr int unit_bytes(int B) { return 32 * B / 8; }
+// Bytes of shared memory for the first m codebooks when they are staged there (B <= 8:
+// 2^B codewords of 16 bytes each); 16-bit codebooks are read through L2.
+constexpr size_t staged_books_bytes(int B, int m) { return B <= 8 ? (size_t)m * (16u << B) : 0; }
+
+// The code at position p (0..31) of a staged (row, slice) unit. B = 4 packs two codes per
+// byte: position p in byte p / 2, low four bits for even p, high four bits for odd p.
+template <int B>
+__device__ __forceinline__ uint32_t unit_code(const unsigned char* u, int p) {
+    if constexpr (B == 4) return (uint32_t)(u[p >> 1] >> ((p & 1) * 4)) & 15u;
+    else if constexpr (B == 8) return u[p];
+    else return ((const uint16_t*)u)[p];
 }
 
 // Record a device-side failure in the workspace status word (first error wins).

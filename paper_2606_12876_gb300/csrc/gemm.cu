@@ -662,28 +662,29 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
 // producing group s*32 + L, so every store is 512 contiguous bytes.
 constexpr int kDenseWarps = 8;
 
-template <int BDT>
+template <int B, int BDT>
 __global__ void __launch_bounds__(kDenseWarps * 32)
 dense_w_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
                uint16_t* __restrict__ w16, int m, int out, int in, int ng, int rows_pad, int RBc,
                size_t plane_bytes) {
+    constexpr int UNIT = unit_bytes(B);
     extern __shared__ __align__(16) unsigned char smem_d[];
-    uint4* books_s = (uint4*)smem_d;                 // [m][256] codewords
+    uint4* books_s = (uint4*)smem_d;                 // [m][2^B] codewords
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    unsigned char* codes_s = smem_d + (size_t)m * 4096 + (size_t)warp * m * 32 * 32;
+    unsigned char* codes_s = smem_d + staged_books_bytes(B, m) + (size_t)warp * m * 32 * UNIT;
     pdl_wait();
     pdl_launch_dependents();
-    for (int i = threadIdx.x; i < m * 256; i += blockDim.x) books_s[i] = __ldg((const uint4*)books + i);
+    for (int i = threadIdx.x; i < (m << B); i += blockDim.x) books_s[i] = __ldg((const uint4*)books + i);
     const int s = blockIdx.y;
     const int rb = blockIdx.x * kDenseWarps + warp;
     const bool active = rb < RBc;
     if (active) {
         const int o = rb * 32 + lane;
         for (int k = 0; k < m; ++k) {
-            const uint4* src = (const uint4*)(planes + k * plane_bytes + ((size_t)s * rows_pad + o) * 32);
-            uint4* dst = (uint4*)(codes_s + ((size_t)k * 32 + lane) * 32);
-            dst[0] = ld_stream_v4(src);
-            dst[1] = ld_stream_v4(src + 1);
+            const uint4* src = (const uint4*)(planes + k * plane_bytes + ((size_t)s * rows_pad + o) * UNIT);
+            uint4* dst = (uint4*)(codes_s + ((size_t)k * 32 + lane) * UNIT);
+#pragma unroll
+            for (int q = 0; q < UNIT / 16; ++q) dst[q] = ld_stream_v4(src + q);
         }
     }
     __syncthreads();
@@ -698,8 +699,8 @@ dense_w_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ 
 #pragma unroll
         for (int e = 0; e < 8; ++e) a[e] = -0.0f;
         for (int k = 0; k < m; ++k) {
-            const uint32_t code = codes_s[((size_t)k * 32 + r) * 32 + p];
-            const uint4 c = lds128(books_u + ((uint32_t)k << 12) + (code << 4));
+            const uint32_t code = unit_code<B>(codes_s + ((size_t)k * 32 + r) * UNIT, p);
+            const uint4 c = lds128(books_u + (((uint32_t)k << B) + code) * 16u);
             add_widen2<BDT>(c.x, a[0], a[1]);
             add_widen2<BDT>(c.y, a[2], a[3]);
             add_widen2<BDT>(c.z, a[4], a[5]);
@@ -711,13 +712,13 @@ dense_w_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ 
     }
 }
 
-template <int BDT>
+template <int B, int BDT>
 aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* books,
                          const void* scales, const void* x, int tokens, void* y, int y_dt,
                          void* ws, uint16_t* w16, cudaStream_t st) {   // x: fp16 [tokens][in]
     {   // decode W_m once
-        const size_t smem = (size_t)m * 4096 + (size_t)kDenseWarps * m * 32 * 32;
-        auto kern = dense_w_kernel<BDT>;
+        const size_t smem = staged_books_bytes(B, m) + (size_t)kDenseWarps * m * 32 * unit_bytes(B);
+        auto kern = dense_w_kernel<B, BDT>;
         if (smem > 48 * 1024)
             if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
                 e != cudaSuccess)
@@ -802,7 +803,7 @@ aq_status launch_gemm(const Dims& d, int m, const void* planes, const void* book
                       const void* scales, const void* x, int x_dt, int tokens, void* y, int y_dt,
                       void* ws, cudaStream_t st) {
     if (d.out == 0 || tokens == 0) return AQ_OK;
-    if (d.B != 8 || m > kGemmMaxM) return AQ_ERR_UNSUPPORTED;
+    if ((d.B != 8 && d.B != 4) || m > kGemmMaxM) return AQ_ERR_UNSUPPORTED;
     const void* xh = x;
     if (x_dt == AQ_BF16) {
         // fp16 copy of the activations after the status word of the workspace
@@ -828,11 +829,15 @@ aq_status launch_gemm(const Dims& d, int m, const void* planes, const void* book
             return e;
         xh = dst;
     }
-    if (gemm_uses_dense(m, tokens)) {
+    if (gemm_uses_dense(d, m, tokens)) {
         uint16_t* w16 = (uint16_t*)((char*)ws + gemm_w16_offset(d, tokens));
+        if (d.B == 4)   // the in-loop decoders read 8-bit codes; 4-bit layouts always go dense
+            return d.book_dt == AQ_BF16
+                       ? run_gemm_dense<4, AQ_BF16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, w16, st)
+                       : run_gemm_dense<4, AQ_F16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, w16, st);
         return d.book_dt == AQ_BF16
-                   ? run_gemm_dense<AQ_BF16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, w16, st)
-                   : run_gemm_dense<AQ_F16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, w16, st);
+                   ? run_gemm_dense<8, AQ_BF16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, w16, st)
+                   : run_gemm_dense<8, AQ_F16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, w16, st);
     }
     return d.book_dt == AQ_BF16
                ? run_gemm<AQ_BF16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, st)

@@ -24,7 +24,7 @@
 //  * gemv_mma (B = 8, 5..16 tokens, any m <= 8). The decoded group (fp32 sum of the m
 //    codewords, rounded once to tf32) is an A fragment of a tensor-core multiply with 8 or
 //    16 tokens of activations (mma.sync m16n8k8).
-//  * gemv_direct (any other case: 16-bit codes, larger m). Decode each group in fp32 (sum of
+//  * gemv_direct (any other case: 4- and 16-bit codes, larger m). Decode each group in fp32 (sum of
 //    m codewords), then multiply by the tokens' 8 activations. Lane L owns row 32*rb+L and
 //    walks the 32 groups of the slice in a common order, so the activation loads are
 //    warp-uniform broadcasts.
@@ -413,13 +413,12 @@ __global__ void __launch_bounds__(256)
 gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
                    const uint16_t* __restrict__ x, int x_dt, float* __restrict__ partials, int m, int batch, int in, int rows_pad, int RBc,
                    int rb_per_chunk, size_t plane_bytes) {
-    constexpr int ESZ = B / 8;
-    constexpr int UNIT = 32 * ESZ;
+    constexpr int UNIT = unit_bytes(B);
     constexpr int kWarps = 8;
     extern __shared__ __align__(128) unsigned char smem[];
     float* xs = (float*)smem;                                        // [NB][256]
-    uint16_t* books_s = (uint16_t*)(smem + NB * 1024);               // B = 8: [m][256][8]
-    const size_t books_bytes = (B == 8) ? (size_t)m * 4096 : 0;
+    uint16_t* books_s = (uint16_t*)(smem + NB * 1024);               // B <= 8: [m][2^B][8]
+    const size_t books_bytes = staged_books_bytes(B, m);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     unsigned char* codes_s = smem + NB * 1024 + books_bytes + (size_t)warp * m * 32 * UNIT;
     const int s = blockIdx.y, chunk = blockIdx.x;
@@ -433,8 +432,8 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
         if (t < batch && col < in) v = bits_to_f32_rt(x[(size_t)t * in + col], x_dt);
         xs[i] = v;
     }
-    if constexpr (B == 8) {
-        for (int i = tid; i < m * 256; i += 256)
+    if constexpr (B <= 8) {
+        for (int i = tid; i < (m << B); i += 256)
             ((uint4*)books_s)[i] = __ldg((const uint4*)books + i);
     }
     __syncthreads();
@@ -459,11 +458,9 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
 #pragma unroll
             for (int e = 0; e < 8; ++e) wv[e] = 0.0f;
             for (int k = 0; k < m; ++k) {
-                uint32_t code;
-                if constexpr (B == 8) code = codes_s[((size_t)k * 32 + lane) * UNIT + p];
-                else code = ((const uint16_t*)(codes_s + ((size_t)k * 32 + lane) * UNIT))[p];
+                const uint32_t code = unit_code<B>(codes_s + ((size_t)k * 32 + lane) * UNIT, p);
                 uint4 cwv;
-                if constexpr (B == 8) cwv = ((const uint4*)books_s)[k * 256 + code];
+                if constexpr (B <= 8) cwv = ((const uint4*)books_s)[(k << B) + code];
                 else cwv = __ldg((const uint4*)books + ((size_t)k << 16) + code);
                 float c[8];
                 unpack8<BDT>(cwv, c);
@@ -825,8 +822,8 @@ template <int NB, int B, int BDT, int SDT>
 aq_status run_direct(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     DeviceInfo di;
     if (aq_status e = device_info(&di); e != AQ_OK) return e;
-    const size_t smem = (size_t)NB * 1024 + (B == 8 ? (size_t)m * 4096 : 0) +
-                        (size_t)8 * m * 32 * 32 * (B / 8);
+    const size_t smem = (size_t)NB * 1024 + staged_books_bytes(B, m) +
+                        (size_t)8 * m * 32 * unit_bytes(B);
     auto kern = gemv_direct_kernel<NB, B, BDT, SDT>;
     int occ = 0;
     if (aq_status e = prepare(kern, smem, 256, m, &occ); e != AQ_OK) return e;
@@ -922,6 +919,14 @@ static aq_status launch_product(const Dims& d, int m, const void* planes, const 
     }
     if (d.B == 8 && batch >= 2 && m <= kMmaMaxM)
         return bb ? dispatch_mma<AQ_BF16>(d, m, a, st) : dispatch_mma<AQ_F16>(d, m, a, st);
+    if (d.B == 4) {
+        switch (bb * 2 + sb) {
+            case 0: return dispatch_direct<4, AQ_F16, AQ_F16>(d, m, a, st);
+            case 1: return dispatch_direct<4, AQ_F16, AQ_BF16>(d, m, a, st);
+            case 2: return dispatch_direct<4, AQ_BF16, AQ_F16>(d, m, a, st);
+            default: return dispatch_direct<4, AQ_BF16, AQ_BF16>(d, m, a, st);
+        }
+    }
     switch ((d.B == 16) * 4 + bb * 2 + sb) {
         case 0: return dispatch_direct<8, AQ_F16, AQ_F16>(d, m, a, st);
         case 1: return dispatch_direct<8, AQ_F16, AQ_BF16>(d, m, a, st);

@@ -27,6 +27,28 @@ __global__ void pack_kernel(const CT* __restrict__ codes, CT* __restrict__ plane
     }
 }
 
+// 4-bit codes: one thread per packed byte (positions 2b and 2b + 1 of a unit). Output byte
+// index = ((k*S + s)*rows_pad + o)*16 + b; even positions in the low four bits.
+__global__ void pack4_kernel(const uint8_t* __restrict__ codes, uint8_t* __restrict__ planes,
+                             int out, int ng, int M, int rows_pad, int S, size_t total) {
+    for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        const int b = (int)(idx & 15);
+        size_t rest = idx >> 4;
+        const int o = (int)(rest % rows_pad);
+        rest /= rows_pad;
+        const int s = (int)(rest % S);
+        const int k = (int)(rest / S);
+        uint32_t v = 0;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int g = s * 32 + ((2 * b + h + o) & 31);
+            if (o < out && g < ng) v |= ((uint32_t)codes[((size_t)o * ng + g) * M + k] & 15u) << (4 * h);
+        }
+        planes[idx] = (uint8_t)v;
+    }
+}
+
 constexpr int kDecWarps = 8;
 
 // Decode: each warp owns one 32-row block of one slice. Lane L stages its own row's codes
@@ -39,18 +61,17 @@ __global__ void __launch_bounds__(kDecWarps * 32)
 decode_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
               const uint16_t* __restrict__ scales, uint16_t* __restrict__ w, int m, int out,
               int in, int ng, int rows_pad, int RBc, size_t plane_bytes) {
-    constexpr int ESZ = B / 8;                       // bytes per code
-    constexpr int UNIT = 32 * ESZ;                   // bytes of one (row, slice) unit
+    constexpr int UNIT = unit_bytes(B);              // bytes of one (row, slice) unit
     extern __shared__ __align__(16) unsigned char smem[];
-    uint16_t* books_s = (uint16_t*)smem;             // B = 8: [m][256][8]
-    const size_t books_bytes = (B == 8) ? (size_t)m * 256 * 8 * 2 : 0;
+    uint16_t* books_s = (uint16_t*)smem;             // B <= 8: [m][2^B][8]
+    const size_t books_bytes = staged_books_bytes(B, m);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     unsigned char* codes_s = smem + books_bytes + (size_t)warp * m * 32 * UNIT;
 
-    if constexpr (B == 8) {
+    if constexpr (B <= 8) {
         const uint4* src = (const uint4*)books;
         uint4* dst = (uint4*)books_s;
-        for (int i = threadIdx.x; i < m * 256; i += blockDim.x) dst[i] = src[i];
+        for (int i = threadIdx.x; i < (m << B); i += blockDim.x) dst[i] = src[i];
     }
     const int s = blockIdx.y;
     const int rb = blockIdx.x * kDecWarps + warp;
@@ -78,11 +99,9 @@ decode_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ b
 #pragma unroll
         for (int e = 0; e < 8; ++e) acc[e] = 0.0f;
         for (int k = 0; k < m; ++k) {
-            uint32_t code;
-            if constexpr (B == 8) code = codes_s[((size_t)k * 32 + r) * UNIT + p];
-            else code = ((const uint16_t*)(codes_s + ((size_t)k * 32 + r) * UNIT))[p];
+            const uint32_t code = unit_code<B>(codes_s + ((size_t)k * 32 + r) * UNIT, p);
             uint4 cw;
-            if constexpr (B == 8) cw = ((const uint4*)books_s)[k * 256 + code];
+            if constexpr (B <= 8) cw = ((const uint4*)books_s)[(k << B) + code];
             else cw = __ldg((const uint4*)books + ((size_t)k << 16) + code);
             float c[8];
             unpack8<BDT>(cw, c);
@@ -105,7 +124,7 @@ decode_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ b
 template <int B, int BDT, int SDT>
 aq_status run_decode(const Dims& d, int m, const void* planes, const void* books,
                      const void* scales, void* w, cudaStream_t st) {
-    const size_t smem = (B == 8 ? (size_t)m * 4096 : 0) + (size_t)kDecWarps * m * 32 * 32 * (B / 8);
+    const size_t smem = staged_books_bytes(B, m) + (size_t)kDecWarps * m * 32 * unit_bytes(B);
     auto kern = decode_kernel<B, BDT, SDT>;
     if (smem > 48 * 1024)
         if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -127,7 +146,13 @@ aq_status launch_pack(const Dims& d, const void* codes, void* planes, cudaStream
     const int threads = 256;
     const size_t want = (total + threads - 1) / threads;
     const int blocks = (int)(want < 65535 * 16 ? want : 65535 * 16);
-    if (d.esz == 1)
+    if (d.B == 4) {
+        const size_t bytes = total / 2;
+        const size_t want4 = (bytes + threads - 1) / threads;
+        const int blocks4 = (int)(want4 < 65535 * 16 ? want4 : 65535 * 16);
+        pack4_kernel<<<blocks4, threads, 0, st>>>((const uint8_t*)codes, (uint8_t*)planes, d.out,
+                                                  d.ng, d.M, d.rows_pad, d.S, bytes);
+    } else if (d.esz == 1)
         pack_kernel<uint8_t><<<blocks, threads, 0, st>>>((const uint8_t*)codes, (uint8_t*)planes,
                                                          d.out, d.ng, d.M, d.rows_pad, d.S, total);
     else
@@ -141,6 +166,14 @@ aq_status launch_decode(const Dims& d, int m, const void* planes, const void* bo
                         const void* scales, void* w, cudaStream_t st) {
     if (d.out == 0) return AQ_OK;
     const int key = (d.B == 16) * 4 + (d.book_dt == AQ_BF16) * 2 + (d.scale_dt == AQ_BF16);
+    if (d.B == 4) {
+        switch (key) {
+            case 0: return run_decode<4, AQ_F16, AQ_F16>(d, m, planes, books, scales, w, st);
+            case 1: return run_decode<4, AQ_F16, AQ_BF16>(d, m, planes, books, scales, w, st);
+            case 2: return run_decode<4, AQ_BF16, AQ_F16>(d, m, planes, books, scales, w, st);
+            default: return run_decode<4, AQ_BF16, AQ_BF16>(d, m, planes, books, scales, w, st);
+        }
+    }
     switch (key) {
         case 0: return run_decode<8, AQ_F16, AQ_F16>(d, m, planes, books, scales, w, st);
         case 1: return run_decode<8, AQ_F16, AQ_BF16>(d, m, planes, books, scales, w, st);

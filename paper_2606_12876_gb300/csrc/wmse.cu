@@ -114,19 +114,18 @@ wmse_resid_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict
                   const uint16_t* __restrict__ scales, const uint16_t* __restrict__ w,
                   uint16_t* __restrict__ e_out, int M, int out, int in, int ng, int rows_pad,
                   int RBc, size_t plane_bytes) {
-    constexpr int ESZ = B / 8;                       // bytes per code
-    constexpr int UNIT = 32 * ESZ;                   // bytes of one (row, slice) code unit
+    constexpr int UNIT = unit_bytes(B);              // bytes of one (row, slice) code unit
     extern __shared__ __align__(16) unsigned char smem[];
-    uint16_t* books_s = (uint16_t*)smem;             // B = 8: [M][256][8]
-    const size_t books_bytes = (B == 8) ? (size_t)M * 4096 : 0;
+    uint16_t* books_s = (uint16_t*)smem;             // B <= 8: [M][2^B][8]
+    const size_t books_bytes = staged_books_bytes(B, M);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     unsigned char* codes_s = smem + books_bytes + (size_t)warp * M * 32 * UNIT;
     pdl_wait();
     pdl_launch_dependents();
-    if constexpr (B == 8) {
+    if constexpr (B <= 8) {
         const uint4* src = (const uint4*)books;
         uint4* dst = (uint4*)books_s;
-        for (int i = threadIdx.x; i < M * 256; i += blockDim.x) dst[i] = src[i];
+        for (int i = threadIdx.x; i < (M << B); i += blockDim.x) dst[i] = src[i];
     }
     const int s = blockIdx.y;
     const int rb = blockIdx.x * kRWarps + warp;
@@ -164,11 +163,9 @@ wmse_resid_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict
 #pragma unroll
         for (int e = 0; e < 8; ++e) acc[e] = -0.0f;
         for (int k = 0; k < M; ++k) {
-            uint32_t code;
-            if constexpr (B == 8) code = codes_s[((size_t)k * 32 + r) * UNIT + p];
-            else code = ((const uint16_t*)(codes_s + ((size_t)k * 32 + r) * UNIT))[p];
+            const uint32_t code = unit_code<B>(codes_s + ((size_t)k * 32 + r) * UNIT, p);
             uint4 cw;
-            if constexpr (B == 8) cw = ((const uint4*)books_s)[k * 256 + code];
+            if constexpr (B <= 8) cw = ((const uint4*)books_s)[(k << B) + code];
             else cw = __ldg((const uint4*)books + ((size_t)k << 16) + code);
             add_widen2<BDT>(cw.x, acc[0], acc[1]);
             add_widen2<BDT>(cw.y, acc[2], acc[3]);
@@ -516,7 +513,7 @@ aq_status encode(CUtensorMap* map, const void* base, int rank, const cuuint64_t*
 template <int B, int BDT, int SDT>
 aq_status run_resid(const Dims& d, const void* w, const void* planes, const void* books,
                     const void* scales, uint16_t* E, cudaStream_t st) {
-    const size_t smem = (B == 8 ? (size_t)d.M * 4096 : 0) + (size_t)kRWarps * d.M * 32 * 32 * (B / 8);
+    const size_t smem = staged_books_bytes(B, d.M) + (size_t)kRWarps * d.M * 32 * unit_bytes(B);
     auto kern = wmse_resid_kernel<B, BDT, SDT>;
     if (smem > 48 * 1024)
         if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -539,6 +536,14 @@ aq_status run_resid(const Dims& d, const void* w, const void* planes, const void
 aq_status launch_resid(const Dims& d, const void* w, const void* planes, const void* books,
                        const void* scales, uint16_t* E, cudaStream_t st) {
     const int key = (d.B == 16) * 4 + (d.book_dt == AQ_BF16) * 2 + (d.scale_dt == AQ_BF16);
+    if (d.B == 4) {
+        switch (key) {
+            case 0: return run_resid<4, AQ_F16, AQ_F16>(d, w, planes, books, scales, E, st);
+            case 1: return run_resid<4, AQ_F16, AQ_BF16>(d, w, planes, books, scales, E, st);
+            case 2: return run_resid<4, AQ_BF16, AQ_F16>(d, w, planes, books, scales, E, st);
+            default: return run_resid<4, AQ_BF16, AQ_BF16>(d, w, planes, books, scales, E, st);
+        }
+    }
     switch (key) {
         case 0: return run_resid<8, AQ_F16, AQ_F16>(d, w, planes, books, scales, E, st);
         case 1: return run_resid<8, AQ_F16, AQ_BF16>(d, w, planes, books, scales, E, st);

@@ -32,7 +32,8 @@ def _u16_to_device(a, device):
 class AQLinear:
     """Packed planes, codebooks and scales of one layer on `device`.
 
-    books: [M][2^B][8] fp16/bf16 bit patterns (uint16); codes: (out, in/8, M) uint8/uint16;
+    books: [M][2^B][8] fp16/bf16 bit patterns (uint16), B = 4, 8 or 16; codes: (out, in/8, M)
+    uint8 (B <= 8) or uint16;
     scales: [out] bit patterns. The natural codes are packed on the GPU by aq_pack. After
     packing the stream is synchronised and the layout is marked AQ_LAYOUT_STATIC_WEIGHTS: the
     layer's weights are read-only from then on, so calls may prefetch them early.
@@ -41,7 +42,7 @@ class AQLinear:
     def __init__(self, books, codes, scales, book_dtype="f16", scale_dtype="f16",
                  device="cuda", keep_codes=False):
         out, ng, M = codes.shape
-        B = 8 if codes.dtype == np.uint8 else 16
+        B = int(np.asarray(books).shape[1]).bit_length() - 1     # books: [M][2^B][8]
         self.layout = Layout.make(out, ng * 8, M, B=B, book_dtype=book_dtype,
                                   scale_dtype=scale_dtype)
         self.out, self.inp, self.M, self.B = out, ng * 8, M, B
@@ -50,7 +51,7 @@ class AQLinear:
         self.books = _u16_to_device(books, self.device)
         self.scales = _u16_to_device(scales, self.device)
         codes_t = torch.from_numpy(np.ascontiguousarray(codes).view(
-            np.int8 if B == 8 else np.int16)).to(self.device)
+            np.int8 if B <= 8 else np.int16)).to(self.device)
         self.planes = torch.empty(packed_bytes(self.layout, M), dtype=torch.uint8,
                                   device=self.device)
         aq_pack(self.layout, codes_t, self.planes)

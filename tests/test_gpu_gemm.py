@@ -67,6 +67,19 @@ def test_gemm_dense_path_long_inputs(case):
         U.assert_product_close(ys, oracle.product_exact(layer, xb[rows], dt, m), "m=%d" % m)
 
 
+@pytest.mark.parametrize("tok", [40, 700])
+def test_gemm_4bit_codes(tok):
+    """4-bit codes (16-entry codebooks): W_m decoded into the workspace, then the pair MMAs."""
+    layer = workloads.make_layer(300, 520, G=8, M=4, B=4, book_dtype="bf16", book_std=0.05,
+                                 scale_dtype="bf16", seed=tok)
+    lin = AQLinear.from_layer(layer)
+    xb = workloads.make_x(tok, 520, "bf16", seed=9)
+    x = x_to_device(xb, "bf16")
+    for m in range(1, 5):
+        y = lin.gemm(x, m, y_dtype=aq.AQ_F32)
+        U.assert_product_close(U.to_f64(y), oracle.product_exact(layer, xb, "bf16", m), "m=%d" % m)
+
+
 def test_gemm_mixed_activation_and_book_types():
     """bf16 activations with fp16 books, and fp16 activations with bf16 books."""
     for bd, xd in (("f16", "bf16"), ("bf16", "f16")):

@@ -26,6 +26,7 @@ def gpu():
 CASES = [  # out, in, M, B, dtype, batch (table lookups, tensor cores, direct, 16-bit codes)
     (300, 1032, 4, 8, "f16", 1), (257, 1032, 3, 8, "bf16", 3), (1000, 2048, 4, 8, "f16", 8),
     (60, 1032, 8, 8, "f16", 2), (96, 520, 2, 16, "f16", 1), (130, 264, 2, 16, "bf16", 5),
+    (257, 1032, 4, 4, "f16", 1),
 ]
 
 

@@ -29,6 +29,7 @@ def gpu():
 
 CASES = [  # out, in, M, B, dtype (planes of exactly one granule; small and ragged; 16-bit codes)
     (4096, 4096, 4, 8, "f16"), (300, 1032, 4, 8, "bf16"), (96, 520, 3, 16, "f16"),
+    (200, 520, 4, 4, "bf16"),
 ]
 
 

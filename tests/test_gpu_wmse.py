@@ -85,6 +85,12 @@ def test_sixteen_bit_codes():
     _check(layer, W_bits, H, lin.wmse(W, Hd).cpu().numpy(), "B=16")
 
 
+def test_four_bit_codes():
+    layer, W_bits, H = _case(130, 264, 4, "f16", seed=12, B=4)
+    lin, W, Hd = _device(layer, W_bits, H)
+    _check(layer, W_bits, H, lin.wmse(W, Hd).cpu().numpy(), "B=4")
+
+
 def test_bf16_h_and_nonsymmetric_h():
     """H given in bf16, and a non-symmetric H (only its symmetric part counts)."""
     layer, W_bits, H = _case(200, 520, 3, "bf16", seed=3)

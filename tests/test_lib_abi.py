@@ -46,11 +46,11 @@ def test_version_and_status_strings():
 
 
 @pytest.mark.parametrize("out,inp,M,B", [(1, 8, 1, 8), (37, 560, 3, 8), (64, 256, 4, 8),
-                                          (50, 136, 2, 16), (4096, 4096, 4, 8)])
+                                          (50, 136, 2, 16), (4096, 4096, 4, 8), (37, 560, 3, 4)])
 def test_packed_sizes_match_oracle_layout(out, inp, M, B):
     L = aq.Layout.make(out, inp, M, B=B)
     layer = dict(out=out, **{"in": inp}, G=8, M=M, B=B,
-                 codes=np.zeros((out, inp // 8, M), np.uint8 if B == 8 else np.uint16))
+                 codes=np.zeros((out, inp // 8, M), np.uint8 if B <= 8 else np.uint16))
     total = oracle.pack(layer).size
     assert aq.plane_bytes(L) * M == total
     for m in range(1, M + 1):
@@ -73,7 +73,8 @@ def _lay(**kw):
 
 
 @pytest.mark.parametrize("kw,status", [
-    (dict(G=4), aq.AQ_ERR_UNSUPPORTED), (dict(B=4), aq.AQ_ERR_UNSUPPORTED),
+    (dict(G=4), aq.AQ_ERR_UNSUPPORTED), (dict(B=5), aq.AQ_ERR_UNSUPPORTED),
+    (dict(B=12), aq.AQ_ERR_UNSUPPORTED),
     (dict(B=17), aq.AQ_ERR_INVALID_ARG), (dict(M=9), aq.AQ_ERR_UNSUPPORTED),
     (dict(M=0), aq.AQ_ERR_INVALID_ARG), (dict(inp=260), aq.AQ_ERR_INVALID_ARG),
     (dict(inp=0), aq.AQ_ERR_INVALID_ARG), (dict(out=-1), aq.AQ_ERR_INVALID_ARG),
@@ -173,3 +174,11 @@ def test_gemm_workspace_sizes():
     assert aq.gemm_workspace_bytes(L, 2048) == off + 300 * 520 * 2
     L1 = aq.Layout.make(300, 520, 1)
     assert aq.gemm_workspace_bytes(L1, 4096) == 256 + 4096 * 520 * 2
+
+
+def test_gemm_workspace_for_4bit_codes():
+    """4-bit layouts always decode W_m into the workspace first."""
+    L = aq.Layout.make(300, 520, 4, B=4)
+    off = (256 + 40 * 520 * 2 + 1023) // 1024 * 1024
+    assert aq.gemm_workspace_bytes(L, 40) == off + 300 * 520 * 2
+    assert aq.plane_bytes(L) == 320 * 96 // 2
