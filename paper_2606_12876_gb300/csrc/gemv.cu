@@ -24,6 +24,8 @@
 //  * gemv_mma (B = 8, 5..16 tokens, any m <= 8). The decoded group (fp32 sum of the m
 //    codewords, rounded once to tf32) is an A fragment of a tensor-core multiply with 8 or
 //    16 tokens of activations (mma.sync m16n8k8).
+//  * gemv_lut4 (B = 4, 1 token): the whole product in one kernel; each warp builds the
+//    16-entry tables of its slices and looks up one entry per 4-bit code.
 //  * gemv_direct (any other case: 4- and 16-bit codes, larger m). Decode each group in fp32 (sum of
 //    m codewords), then multiply by the tokens' 8 activations. Lane L owns row 32*rb+L and
 //    walks the 32 groups of the slice in a common order, so the activation loads are
@@ -692,6 +694,86 @@ splitk_reduce_kernel(const float* __restrict__ partials, const uint16_t* __restr
     }
 }
 
+// ------------------------------------------------------------------ 4-bit codes, one token
+
+// y = x W_m^T for one token with 4-bit codes in one kernel (no split-K partials): a CTA owns
+// 32 rows (lane L is row 32*blockIdx.x + L) and its warp w walks the slices w, w+8, ... For a
+// slice the warp first builds the tables T_k[j][g] = x_g . C_k[j] of every book k < m (16
+// entries x 32 groups, 2 KiB per book): lane g computes group g's 16m entries from its own
+// eight activations. Then each lane reads its row's 16-byte code unit per book and adds one
+// table entry per code; position p of row o holds group (p + o) mod 32, so at every step the
+// 32 lanes read 32 different groups, word g of a 128-byte table row: no bank conflicts. At the
+// end the warps' sums are added in a fixed order (warp 0, 1, ...), scaled by s[o] and, for a
+// refinement, added to y_prev in fp32 before the one rounding to y's type.
+// Warps per CTA: 16 while their tables fit (up to six books), else 8.
+inline int lut4_warps(int m) { return m <= 6 ? 16 : 8; }
+
+template <int BDT, int XDT, int SDT>
+__global__ void __launch_bounds__(512)
+gemv_lut4_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
+                 const uint16_t* __restrict__ scales, const uint16_t* __restrict__ x, void* y,
+                 int y_dt, const void* y_prev, int m, int out, int in, int ng, int S,
+                 int rows_pad, size_t plane_bytes) {
+    extern __shared__ __align__(16) float t4[];      // [warps][m][16][32], then [warps][32]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    float* T = t4 + (size_t)warp * m * 512;
+    float* red = t4 + (size_t)nw * m * 512;
+    const int o = blockIdx.x * 32 + lane;
+    pdl_wait();
+    pdl_launch_dependents();
+    // four accumulators (code words q = 0..3 of a unit) keep the adds independent
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    for (int s = warp; s < S; s += nw) {
+        const int g = s * 32 + lane;                 // this lane's group for the table build
+        float xv[8];
+        if (g < ng) unpack8<XDT>(__ldg((const uint4*)(x + (size_t)g * 8)), xv);
+        else
+#pragma unroll
+            for (int e = 0; e < 8; ++e) xv[e] = 0.0f;
+        __syncwarp();                                // the previous slice's lookups are done
+        for (int k = 0; k < m; ++k) {
+            uint4 cw[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) cw[j] = __ldg((const uint4*)books + (k * 16 + j));
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                float c[8];
+                unpack8<BDT>(cw[j], c);
+                float t = xv[0] * c[0];
+#pragma unroll
+                for (int e = 1; e < 8; ++e) t = fmaf(xv[e], c[e], t);
+                T[(k * 16 + j) * 32 + lane] = t;
+            }
+        }
+        __syncwarp();
+        for (int k = 0; k < m; ++k) {
+            const uint4 u = ld_stream_v4(planes + (size_t)k * plane_bytes + ((size_t)s * rows_pad + o) * 16);
+            const uint32_t wd[4] = {u.x, u.y, u.z, u.w};
+            const float* Tk = T + k * 512;
+#pragma unroll
+            for (int b = 0; b < 8; ++b)              // position p = 8q + b: nibble b of word q
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int p = 8 * q + b;
+                    const uint32_t j = (wd[q] >> (4 * b)) & 15u;
+                    acc[q] += Tk[j * 32 + ((p + lane) & 31)];
+                }
+        }
+    }
+    red[warp * 32 + lane] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+    __syncthreads();
+    if (warp == 0 && o < out) {
+        float sum = 0.0f;
+        for (int w = 0; w < nw; ++w) sum += red[w * 32 + lane];
+        float v = sum * bits_to_f32<SDT>(scales[o]);
+        if (y_prev)
+            v = (y_dt == AQ_F32 ? ((const float*)y_prev)[o]
+                                : bits_to_f32_rt(((const uint16_t*)y_prev)[o], y_dt)) + v;
+        if (y_dt == AQ_F32) ((float*)y)[o] = v;
+        else ((uint16_t*)y)[o] = y_dt == AQ_F16 ? f32_to_bits<AQ_F16>(v) : f32_to_bits<AQ_BF16>(v);
+    }
+}
+
 // ------------------------------------------------------------------ host side
 
 // Launch with the programmatic-stream-serialization attribute (PDL), so the kernel's CTAs may
@@ -885,6 +967,37 @@ aq_status dispatch_direct(const Dims& d, int m, const GemvArgs& a, cudaStream_t 
 
 }  // namespace
 
+template <int BDT, int XDT, int SDT>
+aq_status run_lut4(const Dims& d, int m, const void* planes, const void* books,
+                   const void* scales, const void* x, void* y, int y_dt, const void* y_prev,
+                   cudaStream_t st) {
+    const int nw = lut4_warps(m);
+    const size_t smem = ((size_t)nw * m * 512 + nw * 32) * 4;
+    auto kern = gemv_lut4_kernel<BDT, XDT, SDT>;
+    int occ = 0;
+    if (aq_status e = prepare(kern, smem, nw * 32, m, &occ); e != AQ_OK) return e;
+    return launch_pdl(kern, dim3(d.RBc), dim3(nw * 32), smem, st, (const uint8_t*)planes,
+                      (const uint16_t*)books, (const uint16_t*)scales, (const uint16_t*)x, y,
+                      y_dt, y_prev, m, d.out, d.in, d.ng, d.S, d.rows_pad, d.plane_bytes);
+}
+
+// 4-bit codes, one token: the whole product in one kernel (tables per slice and warp).
+static aq_status launch_lut4(const Dims& d, int m, const void* planes, const void* books,
+                             const void* scales, const void* x, int x_dt, void* y, int y_dt,
+                             const void* y_prev, cudaStream_t st) {
+    const int key = (d.book_dt == AQ_BF16) * 4 + (x_dt == AQ_BF16) * 2 + (d.scale_dt == AQ_BF16);
+    switch (key) {
+        case 0: return run_lut4<AQ_F16, AQ_F16, AQ_F16>(d, m, planes, books, scales, x, y, y_dt, y_prev, st);
+        case 1: return run_lut4<AQ_F16, AQ_F16, AQ_BF16>(d, m, planes, books, scales, x, y, y_dt, y_prev, st);
+        case 2: return run_lut4<AQ_F16, AQ_BF16, AQ_F16>(d, m, planes, books, scales, x, y, y_dt, y_prev, st);
+        case 3: return run_lut4<AQ_F16, AQ_BF16, AQ_BF16>(d, m, planes, books, scales, x, y, y_dt, y_prev, st);
+        case 4: return run_lut4<AQ_BF16, AQ_F16, AQ_F16>(d, m, planes, books, scales, x, y, y_dt, y_prev, st);
+        case 5: return run_lut4<AQ_BF16, AQ_F16, AQ_BF16>(d, m, planes, books, scales, x, y, y_dt, y_prev, st);
+        case 6: return run_lut4<AQ_BF16, AQ_BF16, AQ_F16>(d, m, planes, books, scales, x, y, y_dt, y_prev, st);
+        default: return run_lut4<AQ_BF16, AQ_BF16, AQ_BF16>(d, m, planes, books, scales, x, y, y_dt, y_prev, st);
+    }
+}
+
 // The product kernel of aq_gemv: fp32 partial sums per (slice, token, row) into the workspace.
 static aq_status launch_product(const Dims& d, int m, const void* planes, const void* books,
                                 const void* scales, const void* x, int x_dt, int batch, void* y,
@@ -961,6 +1074,8 @@ aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* book
                       const void* scales, const void* x, int x_dt, int batch, void* y,
                       int y_dt, void* ws, cudaStream_t st, const void* y_prev) {
     if (d.out == 0 || batch == 0) return AQ_OK;
+    if (d.B == 4 && batch == 1)
+        return launch_lut4(d, m, planes, books, scales, x, x_dt, y, y_dt, y_prev, st);
     if (aq_status e = launch_product(d, m, planes, books, scales, x, x_dt, batch, y, y_dt, ws, st);
         e != AQ_OK)
         return e;
