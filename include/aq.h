@@ -133,7 +133,8 @@ aq_status aq_decode(const aq_layout* layout, int m, const void* planes, const vo
  * Two kernels are enqueued, both with programmatic dependent launch: the product (fp32
  * partial sums per 256-input slice, and per codebook at batch 1..4 with 2^8-entry books, into
  * the workspace) and a split-K reduction that sums each row's partials, scales it and
- * writes y. Each waits for the preceding grid before reading memory. The partials of each
+ * writes y (4-bit codes at batch 1: one kernel that writes y itself). Each waits for the
+ * preceding grid before reading memory. The partials of each
  * row are summed in a fixed order, so the result does not depend on scheduling.
  * Accuracy: |y - y_exact| <= 1e-2*(1+|y_exact|) per element and relative Frobenius error
  * <= 2e-3, with y_exact the fp64 product of the exactly widened stored values. */
