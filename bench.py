@@ -142,6 +142,20 @@ class ClockSampler:
                 "samples": len(rows)}
 
 
+def cpu_model():
+    """The host CPU's model name (lscpu), or the machine type."""
+    import platform
+    import subprocess
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                return line.split(":", 1)[1].strip() + " (%s)" % platform.machine()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return platform.machine()
+
+
 def cpu_oracle_rate(layer, x_bits, ms, budget_s, rows=None):
     """Time the oracle on (a row sample of) one step: returns (GB/s, seconds/step, steps)."""
     import oracle
@@ -436,13 +450,26 @@ def own_arm(args):
     ms_step = ms_total / args.steps
 
     # Per prefix: a graph of `steps` launches of that prefix alone (rotating weight copies),
-    # CUDA events around the graph only, so back-to-back launches keep their overlap.
-    per_m_us = {}
+    # CUDA events around the graph only, so back-to-back launches keep their overlap; the
+    # median of 5 replays. Single-call latency: one eager call between synchronisations,
+    # events around it, median of 7.
+    per_m_us, single_us = {}, {}
     for m in ms:
         g = capture(lambda i, m=m: call(i, m), args.steps)
         g.replay()
-        per_m_us[m] = time_graph(g) * 1e3 / args.steps
+        per_m_us[m] = statistics.median(time_graph(g) for _ in range(5)) * 1e3 / args.steps
         del g
+        lat = []
+        with torch.cuda.stream(stream):
+            for i in range(7):
+                torch.cuda.synchronize(dev)
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                call(i, m)
+                e1.record()
+                torch.cuda.synchronize(dev)
+                lat.append(e0.elapsed_time(e1) * 1e3)
+        single_us[m] = statistics.median(lat)
 
 
     # Refinement step (aq_gemv_refine): the increment from prefix m-1 to m, reading plane m-1
@@ -464,10 +491,12 @@ def own_arm(args):
         us = per_m_us[m]
         gbs = bytes_m[m] / (us * 1e-6) / 1e9
         per_m.append({"m": m, "bits_per_weight": m, "us": round(us, 3), "GB_s": round(gbs, 1),
-                      "frac_hbm": round(gbs / hbm_peak, 4), "bytes": bytes_m[m],
+                      "frac_hbm": round(gbs / hbm_peak, 4),
+                      "frac_hbm_spec_8TBs": round(gbs / 8000.0, 4),
+                      "single_call_us": round(single_us[m], 3), "bytes": bytes_m[m],
                       "refine_from_m_minus_1_us": round(refine_us[m], 3),
                       "refine_GB_s": round(refine_bytes / (refine_us[m] * 1e-6) / 1e9, 1)})
-    dom = max(per_m, key=lambda r: r["us"])
+    dom = per_m[-1]       # the full prefix: the most bytes per call (and the longest call)
 
     # end to end through the public API: pinned host x -> device, 4 GEMVs, y -> pinned host
     e2e = None
@@ -505,8 +534,16 @@ def own_arm(args):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
         rate, per, n = cpu_oracle_rate(layer, x_bits, ms, 10.0)
-        cpu = {"value": rate, "unit": "GB/s", "cores": oracle.num_threads(), "kind": "oracle",
-               "sample": "%d full steps (4096x4096, batch 1, m=1..4), %.2f s/step" % (n, per)}
+        cores = oracle.num_threads()
+        # one thread, on the first 256 rows (scaled by bytes like the full-row rate)
+        oracle.set_num_threads(1)
+        rate1, per1, n1 = cpu_oracle_rate(layer, x_bits, ms, 3.0, rows=(0, 256))
+        oracle.set_num_threads(cores)
+        cpu = {"value": rate, "unit": "GB/s", "cores": cores, "kind": "oracle",
+               "sample": "%d full steps (4096x4096, batch 1, m=1..4), %.2f s/step" % (n, per),
+               "one_thread": {"value": rate1, "unit": "GB/s",
+                              "sample": "%d steps on rows 0..255, %.3f s/step" % (n1, per1)},
+               "cpu_model": cpu_model()}
 
     if rank == 0:
         line = {

@@ -52,6 +52,8 @@ def lib():
         L.oracle_bits_to_f64_array.argtypes = [vp, vp, ctypes.c_long, i32]
         L.oracle_num_threads.restype = i32
         L.oracle_num_threads.argtypes = []
+        L.oracle_set_num_threads.restype = None
+        L.oracle_set_num_threads.argtypes = [i32]
         _lib = L
     return _lib
 
@@ -234,6 +236,12 @@ def bits_value(v, dtype):
 
 def num_threads():
     return lib().oracle_num_threads()
+
+
+def set_num_threads(n):
+    """Threads the oracle's OpenMP loops use from now on (timing only; results do not depend
+    on it)."""
+    lib().oracle_set_num_threads(int(n))
 
 
 def widen(bits, dtype):

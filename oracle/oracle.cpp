@@ -299,6 +299,8 @@ int oracle_num_threads(void);
 #ifdef _OPENMP
 #include <omp.h>
 extern "C" int oracle_num_threads(void) { return omp_get_max_threads(); }
+extern "C" void oracle_set_num_threads(int n) { omp_set_num_threads(n > 0 ? n : 1); }
 #else
 extern "C" int oracle_num_threads(void) { return 1; }
+extern "C" void oracle_set_num_threads(int) {}
 #endif
