@@ -496,7 +496,7 @@ def own_arm(args):
                       "single_call_us": round(single_us[m], 3), "bytes": bytes_m[m],
                       "refine_from_m_minus_1_us": round(refine_us[m], 3),
                       "refine_GB_s": round(refine_bytes / (refine_us[m] * 1e-6) / 1e9, 1)})
-    dom = per_m[-1]       # the full prefix: the most bytes per call (and the longest call)
+    dom = per_m[-1]       # the full prefix: the most bytes per call
 
     # end to end through the public API: pinned host x -> device, 4 GEMVs, y -> pinned host
     e2e = None
