@@ -130,7 +130,8 @@ def workloads_values(bits, dtype):
 
 
 def _tiny_layers():
-    shapes = [(1, 8, 1, 8), (3, 16, 2, 8), (8, 24, 4, 8), (5, 8, 3, 16), (33, 40, 2, 8)]
+    shapes = [(1, 8, 1, 8), (3, 16, 2, 8), (8, 24, 4, 8), (5, 8, 3, 16), (33, 40, 2, 8),
+              (7, 24, 3, 4)]
     for idx, (out, inp, M, B) in enumerate(shapes):
         for bd in ("f16", "bf16"):
             yield workloads.make_layer(out, inp, G=8, M=M, B=B, book_dtype=bd, book_std=0.3,
