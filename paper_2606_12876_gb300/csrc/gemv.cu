@@ -714,16 +714,25 @@ gemv_lut4_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict_
                  const uint16_t* __restrict__ scales, const uint16_t* __restrict__ x, void* y,
                  int y_dt, const void* y_prev, int m, int out, int in, int ng, int S,
                  int rows_pad, size_t plane_bytes) {
-    extern __shared__ __align__(16) float t4[];      // [warps][m][16][32], then [warps][32]
+    // [warps][m][16][32] tables, [warps][32] sums, [m][16] codewords
+    extern __shared__ __align__(16) float t4[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
     float* T = t4 + (size_t)warp * m * 512;
     float* red = t4 + (size_t)nw * m * 512;
+    uint4* books_s = (uint4*)(red + nw * 32);
     const int o = blockIdx.x * 32 + lane;
     pdl_wait();
     pdl_launch_dependents();
+    for (int i = threadIdx.x; i < m * 16; i += blockDim.x) books_s[i] = __ldg((const uint4*)books + i);
+    __syncthreads();
     // four accumulators (code words q = 0..3 of a unit) keep the adds independent
     float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
     for (int s = warp; s < S; s += nw) {
+        // the row's code units of this slice, requested before the tables are built
+        uint4 u[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            if (k < m) u[k] = ld_stream_v4(planes + (size_t)k * plane_bytes + ((size_t)s * rows_pad + o) * 16);
         const int g = s * 32 + lane;                 // this lane's group for the table build
         float xv[8];
         if (g < ng) unpack8<XDT>(__ldg((const uint4*)(x + (size_t)g * 8)), xv);
@@ -734,7 +743,7 @@ gemv_lut4_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict_
         for (int k = 0; k < m; ++k) {
             uint4 cw[16];
 #pragma unroll
-            for (int j = 0; j < 16; ++j) cw[j] = __ldg((const uint4*)books + (k * 16 + j));
+            for (int j = 0; j < 16; ++j) cw[j] = books_s[k * 16 + j];
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
                 float c[8];
@@ -746,9 +755,10 @@ gemv_lut4_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict_
             }
         }
         __syncwarp();
-        for (int k = 0; k < m; ++k) {
-            const uint4 u = ld_stream_v4(planes + (size_t)k * plane_bytes + ((size_t)s * rows_pad + o) * 16);
-            const uint32_t wd[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            if (k >= m) break;
+            const uint32_t wd[4] = {u[k].x, u[k].y, u[k].z, u[k].w};
             const float* Tk = T + k * 512;
 #pragma unroll
             for (int b = 0; b < 8; ++b)              // position p = 8q + b: nibble b of word q
@@ -972,7 +982,7 @@ aq_status run_lut4(const Dims& d, int m, const void* planes, const void* books,
                    const void* scales, const void* x, void* y, int y_dt, const void* y_prev,
                    cudaStream_t st) {
     const int nw = lut4_warps(m);
-    const size_t smem = ((size_t)nw * m * 512 + nw * 32) * 4;
+    const size_t smem = ((size_t)nw * m * 512 + nw * 32) * 4 + (size_t)m * 16 * 16;
     auto kern = gemv_lut4_kernel<BDT, XDT, SDT>;
     int occ = 0;
     if (aq_status e = prepare(kern, smem, nw * 32, m, &occ); e != AQ_OK) return e;
