@@ -299,9 +299,16 @@ size_t aq_store_device_bytes(const aq_store* store);
 aq_status aq_store_destroy(aq_store* store);
 
 /* ---------------------------------------------------------------- workspace helpers
+ * aq_selftest_wait: self-test of the library's failure detection (no counterpart in the
+ * paper). Enqueues a one-thread kernel that waits, through the same time-bounded mbarrier wait
+ * the compute kernels use (about 2 s), for a barrier phase that nothing completes; when the
+ * wait gives up it records AQ_ERR_TIMEOUT in the workspace status word and returns, leaving
+ * the context usable. aq_workspace_status then reports AQ_ERR_TIMEOUT once.
+ *   workspace : device, at least 256 bytes, 16-byte aligned, zero-filled.
  * aq_workspace_init: enqueue a zero-fill of bytes at workspace (cudaMemsetAsync).
  * aq_workspace_status: SYNCHRONISES stream, then returns the device-side status a kernel
  * recorded in the workspace (AQ_OK if none) and clears it. */
+aq_status aq_selftest_wait(void* workspace, size_t workspace_bytes, void* stream);
 aq_status aq_workspace_init(void* workspace, size_t bytes, void* stream);
 aq_status aq_workspace_status(void* workspace, void* stream);
 

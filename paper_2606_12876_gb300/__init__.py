@@ -26,7 +26,7 @@ EXPORTS = ["aq_abi_version", "aq_status_string", "aq_last_error", "aq_plane_byte
            "aq_gemm", "aq_workspace_init", "aq_workspace_status", "aq_gemv_static_scratch",
            "aq_gemv_refine", "aq_store_create", "aq_store_set_prefix", "aq_store_prefix",
            "aq_store_planes", "aq_store_books", "aq_store_scales", "aq_store_device_bytes",
-           "aq_store_destroy", "aq_wmse_workspace_bytes", "aq_wmse"]
+           "aq_store_destroy", "aq_wmse_workspace_bytes", "aq_wmse", "aq_selftest_wait"]
 
 
 class AQError(RuntimeError):
@@ -88,6 +88,7 @@ def lib():
             "aq_store_device_bytes": (sz, [vp]),
             "aq_store_destroy": (i32, [vp]),
             "aq_wmse_workspace_bytes": (sz, [lp]),
+            "aq_selftest_wait": (i32, [vp, sz, vp]),
             "aq_wmse": (i32, [lp, vp, vp, vp, vp, vp, i32, ctypes.POINTER(ctypes.c_double), vp,
                               vp, sz, vp]),
         }

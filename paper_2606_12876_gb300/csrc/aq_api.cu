@@ -260,6 +260,13 @@ aq_status aq_gemm(const aq_layout* layout, int m, const void* planes, const void
                            as_stream(stream));
 }
 
+aq_status aq_selftest_wait(void* workspace, size_t workspace_bytes, void* stream) {
+    if (!workspace) return AQ_ERR_INVALID_ARG;
+    if (workspace_bytes < aq::kWsStatusBytes) return AQ_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;
+    return aq::launch_selftest_wait((unsigned int*)workspace, as_stream(stream));
+}
+
 aq_status aq_workspace_init(void* workspace, size_t bytes, void* stream) {
     if (!workspace) return AQ_ERR_INVALID_ARG;
     if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;

@@ -87,6 +87,8 @@ aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* book
 aq_status launch_gemm(const Dims& d, int m, const void* planes, const void* books,
                       const void* scales, const void* x, int x_dt, int tokens, void* y, int y_dt,
                       void* ws, cudaStream_t st);
+// aq_selftest_wait: one bounded wait that nothing completes (records AQ_ERR_TIMEOUT).
+aq_status launch_selftest_wait(unsigned int* status, cudaStream_t st);
 // Per-prefix distortion (aq_wmse): workspace bytes, and the launch (validated arguments).
 size_t wmse_ws_bytes(const Dims& d);
 aq_status launch_wmse(const Dims& d, const void* w, const void* planes, const void* books,

@@ -140,6 +140,28 @@ aq_status run_decode(const Dims& d, int m, const void* planes, const void* books
 
 }  // namespace
 
+namespace {
+
+// Self-test of the bounded waits: thread 0 waits, through the same bounded wait the compute
+// kernels use, on a shared-memory mbarrier that nothing arrives at; when the wait gives up it
+// records AQ_ERR_TIMEOUT in the status word and the kernel returns.
+__global__ void selftest_wait_kernel(unsigned int* status) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        mbar_fence_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && !mbar_wait(&bar, 0)) record_status(status, AQ_ERR_TIMEOUT);
+}
+
+}  // namespace
+
+aq_status launch_selftest_wait(unsigned int* status, cudaStream_t st) {
+    selftest_wait_kernel<<<1, 32, 0, st>>>(status);
+    return cuda_ok(cudaGetLastError(), "kernel launch");
+}
+
 aq_status launch_pack(const Dims& d, const void* codes, void* planes, cudaStream_t st) {
     const size_t total = (size_t)d.M * d.plane_elems;
     if (total == 0) return AQ_OK;

@@ -182,3 +182,10 @@ def test_gemm_workspace_for_4bit_codes():
     off = (256 + 40 * 520 * 2 + 1023) // 1024 * 1024
     assert aq.gemm_workspace_bytes(L, 40) == off + 300 * 520 * 2
     assert aq.plane_bytes(L) == 320 * 96 // 2
+
+
+def test_selftest_wait_argument_errors_on_the_host():
+    lib = aq.lib()
+    assert lib.aq_selftest_wait(None, 256, None) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_selftest_wait(FAKE, 16, None) == aq.AQ_ERR_WORKSPACE
+    assert lib.aq_selftest_wait(FAKE + 8, 256, None) == aq.AQ_ERR_ALIGNMENT
