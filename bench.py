@@ -58,16 +58,30 @@ def layer_bytes(out, inp, m, B=8, G=8, batch=1, xsize=2, ysize=2):
             + batch * inp * xsize + batch * out * ysize)
 
 
+def lut_kernel_source():
+    """The source text that decides what gemv_lut_kernel reads: the kernel's section of gemv.cu,
+    its launcher run_lut (grid, ring slots, work split), and the device helpers of
+    aq_internal.cuh."""
+    csrc = os.path.join(ROOT, "paper_2606_12876_gb300", "csrc")
+    g = open(os.path.join(csrc, "gemv.cu")).read()
+    h = open(os.path.join(csrc, "aq_internal.cuh")).read()
+    rule = "// " + "-" * 66
+    a = g.index(rule + " LUT kernel")
+    b = g.index(rule, a + len(rule))
+    r0 = g.index("aq_status run_lut(const Dims& d")
+    r1 = g.index("\n}\n", r0)
+    d0 = h.index("// ---- device helpers")
+    return g[a:b] + g[r0:r1] + h[d0:]
+
+
 def profiled_traffic(workload, m):
     """DRAM bytes per launch measured by ncu (profiles/gemv_lut_traffic.txt), or None when the
-    kernel sources changed since that capture."""
+    kernel's source (lut_kernel_source) changed since that capture."""
     import hashlib
     path = os.path.join(ROOT, "profiles", "gemv_lut_traffic.txt")
     if not os.path.exists(path):
         return None
-    h = hashlib.sha256()
-    for f in ("gemv.cu", "aq_internal.cuh"):
-        h.update(open(os.path.join(ROOT, "paper_2606_12876_gb300", "csrc", f), "rb").read())
+    h = hashlib.sha256(lut_kernel_source().encode())
     rec, traffic = None, None
     for line in open(path):
         parts = line.split()
