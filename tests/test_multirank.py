@@ -61,3 +61,4 @@ def test_reference_arm_runs_on_rank_zero_only(monkeypatch):
     with contextlib.redirect_stdout(out):
         assert bench.reference_arm(A()) is None
     assert out.getvalue() == ""
+
