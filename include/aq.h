@@ -5,8 +5,8 @@
  * A linear layer W (d_out x d_in) is stored once as M additive codebooks C_0..C_{M-1}
  * (each 2^B codewords of g = 8 values), per-output-row scales s, and one B-bit code per
  * (row, group of g inputs, codebook). At call time a prefix length m (1 <= m <= M) selects
- * how many codebooks are summed (Sec. 5: "partial reconstruction using the first k
- * codebooks"; the number of active codebooks is a deployment parameter):
+ * how many codebooks are summed (Sec. 5: the weights are rebuilt from the leading k
+ * codebooks only, and how many are active is chosen at deployment):
  *
  *     W_m[o, g*8 + e] = s[o] * sum_{k<m} C_k[ b_k[o, g] ][e]         (Sec. 3.2 and Sec. 5)
  *     y[t, o]         = sum_i x[t, i] * W_m[o, i]                     (Sec. 2.2, Y = W X)
