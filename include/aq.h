@@ -171,12 +171,16 @@ aq_status aq_gemv_refine(const aq_layout* layout, int m, const void* planes, con
  * can synchronise the device or fail under memory pressure. Nothing is allocated: the scratch
  * comes from a fixed AQ_STATIC_SCRATCH_BYTES buffer that the library holds, as a device
  * array, on every GPU that loads it, until the process exits.
- *   - Arguments and results are those of aq_gemv (same checks, same status codes).
+ *   - Arguments and host-side status codes are those of aq_gemv (same checks).
  *   - Returns AQ_ERR_WORKSPACE when aq_gemv_workspace_bytes(layout, batch) is larger than
  *     AQ_STATIC_SCRATCH_BYTES; use aq_gemv with a workspace for such sizes.
  *   - The first call on a device looks up the buffer's device address; make that first call
- *     on each device before capturing any stream on it.
- *   - Each call enqueues a clear of the buffer's status word, then the GEMV.
+ *     on each device before capturing any stream on it. The address is cached for the life of
+ *     the device's primary context: do not use this entry point after cudaDeviceReset.
+ *   - Each call enqueues the GEMV kernels only (nothing is cleared in between).
+ *   - A device-side failure (a bounded wait that gave up, AQ_ERR_TIMEOUT) is recorded in the
+ *     buffer's status word and stays there, across later calls, until
+ *     aq_gemv_static_scratch_status reads and clears it.
  *   - Every call on a device shares the one buffer, which keeps the last call's contents:
  *     calls that may overlap on the GPU (other streams, other host threads) race on it and
  *     must be ordered by the caller. */
@@ -184,6 +188,11 @@ aq_status aq_gemv_refine(const aq_layout* layout, int m, const void* planes, con
 aq_status aq_gemv_static_scratch(const aq_layout* layout, int m, const void* planes,
                                  const void* books, const void* scales, const void* x,
                                  int x_dtype, int batch, void* y, int y_dtype, void* stream);
+
+/* The device-side status of the aq_gemv_static_scratch calls on the current device: as
+ * aq_workspace_status for the library's fixed buffer. SYNCHRONISES stream, returns the status
+ * a kernel recorded (AQ_OK if none) and clears it. (No counterpart in the paper.) */
+aq_status aq_gemv_static_scratch_status(void* stream);
 
 /* ---------------------------------------------------------------- GEMM (prefill)
  * Same product for many tokens: y[t, o] = sum_i x[t, i] * W_m[o, i], t < tokens. Decoded

@@ -24,6 +24,7 @@ TORCH_DTYPES = {AQ_F16: torch.float16, AQ_BF16: torch.bfloat16, AQ_F32: torch.fl
 EXPORTS = ["aq_abi_version", "aq_status_string", "aq_last_error", "aq_plane_bytes", "aq_packed_bytes", "aq_pack",
            "aq_decode", "aq_gemv_workspace_bytes", "aq_gemv", "aq_gemm_workspace_bytes",
            "aq_gemm", "aq_workspace_init", "aq_workspace_status", "aq_gemv_static_scratch",
+           "aq_gemv_static_scratch_status",
            "aq_gemv_refine", "aq_store_create", "aq_store_set_prefix", "aq_store_prefix",
            "aq_store_planes", "aq_store_books", "aq_store_scales", "aq_store_device_bytes",
            "aq_store_destroy", "aq_wmse_workspace_bytes", "aq_wmse", "aq_selftest_wait"]
@@ -78,6 +79,7 @@ def lib():
             "aq_workspace_init": (i32, [vp, sz, vp]),
             "aq_workspace_status": (i32, [vp, vp]),
             "aq_gemv_static_scratch": (i32, [lp, i32, vp, vp, vp, vp, i32, i32, vp, i32, vp]),
+            "aq_gemv_static_scratch_status": (i32, [vp]),
             "aq_gemv_refine": (i32, [lp, i32, vp, vp, vp, vp, i32, i32, vp, vp, i32, vp, sz, vp]),
             "aq_store_create": (i32, [lp, ctypes.POINTER(vp)]),
             "aq_store_set_prefix": (i32, [vp, i32, vp, vp, vp, vp]),
@@ -196,6 +198,12 @@ def aq_gemv_static_scratch(layout, m, planes, books, scales, x, x_dtype, batch, 
     _check(lib().aq_gemv_static_scratch(ctypes.byref(layout), m, _ptr(planes), _ptr(books),
                                         _ptr(scales), _ptr(x), x_dtype, batch, _ptr(y), y_dtype,
                                         _stream(stream)), "aq_gemv_static_scratch")
+
+
+def aq_gemv_static_scratch_status(stream=None):
+    """The device-side status of the aq_gemv_static_scratch calls on the current device
+    (synchronises the stream; clears the status)."""
+    return lib().aq_gemv_static_scratch_status(_stream(stream))
 
 
 def aq_store_create(layout):

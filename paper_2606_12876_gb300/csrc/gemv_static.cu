@@ -19,7 +19,9 @@ constexpr size_t kStaticScratchBytes = AQ_STATIC_SCRATCH_BYTES;
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
 // In host code, g_static_scratch names a host-side stand-in, not the device buffer; the device
-// address is looked up once per device (with that device current) and cached here.
+// address is looked up once per device (with that device current) and cached here. The cache
+// belongs to the device's primary context: after cudaDeviceReset the address is stale, so
+// this entry point must not be used across a reset.
 std::mutex g_mu;
 void* g_scratch_addr[64] = {};
 
@@ -52,16 +54,20 @@ extern "C" aq_status aq_gemv_static_scratch(const aq_layout* layout, int m, cons
 
     const size_t need = aq_gemv_workspace_bytes(layout, batch);
     if (need == 0 || need > kStaticScratchBytes) return AQ_ERR_WORKSPACE;  // beyond the fixed buffer
-    aq::Dims d;
-    if (aq_status e = aq::make_dims(layout, &d); e != AQ_OK) return e;
 
     void* scratch = nullptr;
     if (aq_status e = static_scratch_address(&scratch); e != AQ_OK) return e;
-    // The buffer keeps whatever the previous call left; the status word must start at zero,
-    // so clear it (the partial sums are always written before they are read).
-    if (cudaError_t e = cudaMemsetAsync(scratch, 0, aq::ws_partial_offset(d), (cudaStream_t)stream);
-        e != cudaSuccess)
-        return aq::cuda_fail(e, "cudaMemsetAsync");
+    // Nothing is cleared here: the partial sums are always written before they are read, and
+    // the status word (zero when the library is loaded) is set only when a device-side wait
+    // gives up; it stays set until aq_gemv_static_scratch_status reads and clears it. So a
+    // call enqueues the GEMV kernels alone, which keeps the overlap of consecutive calls
+    // (programmatic dependent launch) that a memset between them would break.
     return aq_gemv(layout, m, planes, books, scales, x, x_dtype, batch, y, y_dtype, scratch,
                    kStaticScratchBytes, stream);
+}
+
+extern "C" aq_status aq_gemv_static_scratch_status(void* stream) {
+    void* scratch = nullptr;
+    if (aq_status e = static_scratch_address(&scratch); e != AQ_OK) return e;
+    return aq_workspace_status(scratch, stream);
 }

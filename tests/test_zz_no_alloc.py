@@ -39,6 +39,34 @@ def test_static_scratch_matches_workspace_gemv(case):
                 lin.scales.data_ptr(), x.data_ptr(), xc, batch, y.data_ptr(), aq.AQ_F32, stream)
             assert rc == aq.AQ_OK, aq.status_string(rc)
             U.assert_product_close(U.to_f64(y), ref, "m=%d" % m)
+    # no device-side wait gave up in any of these calls
+    assert aq.lib().aq_gemv_static_scratch_status(stream) == aq.AQ_OK
+
+
+def test_static_scratch_leaves_device_memory_alone():
+    """A burst of calls changes the device's free memory by nothing: the entry point allocates
+    neither memory of its own nor through the caching allocator (y is allocated up front)."""
+    U.require_gpu()
+    layer = workloads.make_layer(1000, 2048, G=8, M=3, B=8, book_std=0.05, seed=21)
+    lin = AQLinear.from_layer(layer)
+    x = x_to_device(workloads.make_x(1, 2048, "f16", seed=2), "f16")
+    y = torch.empty(1, 1000, dtype=torch.float16, device="cuda")
+    stream = torch.cuda.current_stream().cuda_stream
+
+    def call():
+        rc = aq.lib().aq_gemv_static_scratch(
+            ctypes.byref(lin.layout), 3, lin.planes.data_ptr(), lin.books.data_ptr(),
+            lin.scales.data_ptr(), x.data_ptr(), aq.AQ_F16, 1, y.data_ptr(), aq.AQ_F16, stream)
+        assert rc == aq.AQ_OK, aq.status_string(rc)
+
+    call()                          # first call on the device: looks up the buffer's address
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for _ in range(50):
+        call()
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    assert aq.lib().aq_gemv_static_scratch_status(stream) == aq.AQ_OK
 
 
 def test_static_scratch_rejects_sizes_beyond_the_buffer():
