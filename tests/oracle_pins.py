@@ -347,6 +347,38 @@ def pin_wmse_bruteforce_tiny():
         assert abs(D[k - 1] - tot / 3) <= 1e-10 * abs(tot / 3), (k, D[k - 1], tot / 3)
 
 
+def pin_wmse_abs_bruteforce_tiny():
+    """The magnitude behind the distortion tolerance, (1/d_out) sum_o |e_o| |H| |e_o|^T, as a
+    triple sum over rows and input pairs in plain Python on a 3 x 16 layer."""
+    layer, W, X = _wmse_case(out=3, inp=16, M=2, seed=17, dt="f16")
+    H = X @ X.T / X.shape[1] - 0.3          # entries of both signs
+    A = oracle.wmse_abs(layer, W, H)
+    for k in (1, 2):
+        E = W - _onehot_reconstruction(layer, k)
+        tot = 0.0
+        for o in range(3):
+            for i in range(16):
+                for j in range(16):
+                    tot += abs(E[o, i]) * abs(H[i, j]) * abs(E[o, j])
+        assert abs(A[k - 1] - tot / 3) <= 1e-10 * (tot / 3), (k, A[k - 1], tot / 3)
+
+
+def pin_wmse_abs_equals_wmse_for_nonnegative_terms():
+    """With W - W^(k) and H elementwise non-negative every term of the trace is non-negative,
+    so the magnitude equals the distortion itself; in general it bounds |D^(k)| from above."""
+    layer, _, X = _wmse_case(out=16, inp=48, M=3, seed=19, dt="f16")
+    top = max(float(np.max(_onehot_reconstruction(layer, k))) for k in range(1, 4))
+    rng = _rng(20)
+    W = top + 0.01 + rng.random((16, 48))   # above every reconstruction: e >= 0
+    H = np.abs(X @ X.T / X.shape[1])
+    D, A = oracle.wmse(layer, W, H), oracle.wmse_abs(layer, W, H)
+    assert np.all(np.abs(A - D) <= 1e-12 * A), (A, D)
+    H2 = X @ X.T / X.shape[1] - 0.5
+    W2 = _onehot_reconstruction(layer, 3) + 0.1 * rng.standard_normal((16, 48))
+    D2, A2 = oracle.wmse(layer, W2, H2), oracle.wmse_abs(layer, W2, H2)
+    assert np.all(np.abs(D2) <= A2 * (1 + 1e-12)) and np.any(np.abs(D2) < 0.9 * A2), (D2, A2)
+
+
 def pin_wmse_vanishes_at_the_exact_weight():
     """W = W^(M): the full prefix has zero distortion; a shorter prefix leaves the dropped
     codebooks' contribution, which is positive for a positive definite H."""

@@ -45,6 +45,11 @@ PY_MUTANTS = [
      "E = W + reconstruct_exact(layer, k)\n        res.append(float(np.sum((E @ H)"),
     ("wmse_squares_H", "np.sum((E @ H) * E)", "np.sum((E @ H @ H) * E)"),
     ("dbyd_shifted_weights", "total += lam[k] * D[k]", "total += lam[k] * D[k - 1]"),
+    ("wmse_abs_keeps_sign_of_H", "A = np.abs(np.asarray(H, dtype=np.float64))",
+     "A = np.asarray(H, dtype=np.float64)"),
+    ("wmse_abs_drops_normalisation", "np.sum((E @ A) * E)) / out", "np.sum((E @ A) * E))"),
+    ("wmse_abs_prefix_off_by_one", "E = np.abs(np.asarray(W, dtype=np.float64) - reconstruct_exact(layer, k))",
+     "E = np.abs(np.asarray(W, dtype=np.float64) - reconstruct_exact(layer, max(1, k - 1)))"),
 ]
 
 
