@@ -195,24 +195,29 @@ aq_status aq_gemv_static_scratch(const aq_layout* layout, int m, const void* pla
 aq_status aq_gemv_static_scratch_status(void* stream);
 
 /* ---------------------------------------------------------------- GEMM (prefill)
- * Same product for many tokens: y[t, o] = sum_i x[t, i] * W_m[o, i], t < tokens. Decoded
- * weight tiles are built in shared memory and multiplied on the tcgen05 tensor cores with
- * fp32 accumulation in tensor memory (up to 2047 tokens, or m = 1, W_m is never written to HBM;
- * see workspace below). The MMA operands are fp16:
- * each decoded weight (fp32 sum of the m codewords) is rounded once to fp16, and bf16
- * activations are first copied to fp16 in the workspace (exact for |x| in fp16's normal
- * range; values beyond +-65504 saturate). Supported: code_bits = 8 and 4 (4-bit layouts always
+ * Same product for many tokens (Sec. 2.2 Y = W X with W_m of Sec. 3.2 / Sec. 5):
+ * y[t, o] = sum_i x[t, i] * W_m[o, i], t < tokens. Decoded weight tiles are built in shared
+ * memory and multiplied on the tcgen05 tensor cores with fp32 accumulation in tensor memory
+ * (up to 2047 tokens, or m = 1, W_m is never written to HBM; see workspace below). The MMA
+ * operands are fp16, over the whole range of the inputs: each decoded weight (fp32 sum of the
+ * m codewords) is rounded once to fp16 after the codebooks were scaled by a power of two
+ * 2^-f that keeps the largest possible sum below 2^15; bf16 activations are copied to fp16 in
+ * the workspace, each token row scaled by a power of two 2^-e_t that puts its largest |x| in
+ * [2^14, 2^15); the epilogue multiplies by 2^(e_t + f). The scalings are exact, so inputs
+ * already inside fp16's range give the same bits as without them, and bf16 values far outside
+ * it (activation outliers, large codebook entries) are multiplied with fp16's 11-bit
+ * significand instead of saturating. Supported: code_bits = 8 and 4 (4-bit layouts always
  * decode W_m into the workspace first), any m <= num_books <= 8.
  *   x : device, [tokens][d_in] of x_dtype (AQ_F16 or AQ_BF16); y : device, [tokens][d_out]
  *       of y_dtype (AQ_F16, AQ_BF16 or AQ_F32).
- *   workspace : aq_gemm_workspace_bytes(layout, tokens) bytes (a status word, room for the
- *               fp16 activation copy and, from 2048 tokens when num_books >= 2 (for 4-bit
- *               codes always), room for W_m
- *               decoded once in fp16, d_out*d_in*2 bytes: at that length calls with m >= 2
- *               decode W_m into it and multiply by TMA-fed tensor-core tiles, which is faster
- *               than decoding every weight tile again for every 512 tokens), zero-filled
- *               before first use; its first word receives a device-side status (see
- *               aq_workspace_status).
+ *   workspace : aq_gemm_workspace_bytes(layout, tokens) bytes (a 256-byte status block, one
+ *               float per token for the activation factors, room for the fp16 activation
+ *               copy and, from 2048 tokens when num_books >= 2 (for 4-bit codes always), room
+ *               for W_m decoded once in fp16, d_out*d_in*2 bytes: at that length calls with
+ *               m >= 2 decode W_m into it and multiply by TMA-fed tensor-core tiles, which is
+ *               faster than decoding every weight tile again for every 512 tokens),
+ *               zero-filled before first use; its first word receives a device-side status
+ *               (see aq_workspace_status).
  * Accuracy: as aq_gemv for fp32 outputs; fp16/bf16 outputs add one rounding of y. */
 size_t aq_gemm_workspace_bytes(const aq_layout* layout, int tokens);
 aq_status aq_gemm(const aq_layout* layout, int m, const void* planes, const void* books,

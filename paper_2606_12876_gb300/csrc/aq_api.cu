@@ -46,6 +46,10 @@ thread_local char g_last_error[256] = "";
 aq_status cuda_fail(cudaError_t e, const char* what) {
     snprintf(g_last_error, sizeof(g_last_error), "%s: %s (%s)", what, cudaGetErrorName(e),
              cudaGetErrorString(e));
+    // A failed launch or runtime call leaves its error as the thread's last error; take it
+    // back, so that a later launch checked with cudaGetLastError is not blamed for it (a sticky
+    // error, one that corrupted the context, is reported again by every later call anyway).
+    (void)cudaGetLastError();
     return AQ_ERR_CUDA;
 }
 

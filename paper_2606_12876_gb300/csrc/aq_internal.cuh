@@ -48,22 +48,27 @@ constexpr int kLutMaxM = 8, kLutMultiM = 4;
 inline int lut_max_m(int batch) { return batch <= 2 ? kLutMaxM : batch <= 4 ? kLutMultiM : 0; }
 inline bool uses_lut(const Dims& d, int m, int batch) { return d.B == 8 && m <= lut_max_m(batch); }
 
-// Prefill GEMM workspace: [status word][fp16 copy of bf16 activations][dense W_m, fp16]. From
-// kGemmDenseTokens tokens, prefixes of two or more books decode W_m once into the workspace
-// and run the pair MMAs on it (decoding in the GEMM's inner loop is bound by shared-memory
-// gathers, and at that length every weight tile is decoded again for every 512 tokens).
-// 4-bit layouts always take the dense form (the in-loop decoders read 8-bit codes).
+// Prefill GEMM workspace: [status block, 256 B: status word at 0, the dense form's weight
+// factor (float) at kWsWfacOffset][per-token activation factors, float][fp16 copy of bf16
+// activations][dense W_m, fp16]. From kGemmDenseTokens tokens, prefixes of two or more books
+// decode W_m once into the workspace and run the pair MMAs on it (decoding in the GEMM's inner
+// loop is bound by shared-memory gathers, and at that length every weight tile is decoded
+// again for every 512 tokens). 4-bit layouts always take the dense form (the in-loop decoders
+// read 8-bit codes).
 constexpr int kGemmDenseTokens = 2048;
+constexpr size_t kWsWfacOffset = 128;
 inline bool gemm_uses_dense(const Dims& d, int m, int tokens) {
     return d.B == 4 || (m >= 2 && tokens >= kGemmDenseTokens);
 }
+inline size_t gemm_xfac_offset() { return kWsStatusBytes; }
+inline size_t gemm_x16_offset(int tokens) { return kWsStatusBytes + round_up((size_t)tokens * 4, 256); }
 inline size_t gemm_w16_offset(const Dims& d, int tokens) {
-    return round_up(kWsStatusBytes + (size_t)tokens * (size_t)d.in * 2, 1024);
+    return round_up(gemm_x16_offset(tokens) + (size_t)tokens * (size_t)d.in * 2, 1024);
 }
 inline size_t gemm_ws_need(const Dims& d, int tokens) {
     if (d.B == 4 || (d.B == 8 && d.M >= 2 && tokens >= kGemmDenseTokens))
         return gemm_w16_offset(d, tokens) + (size_t)d.out * (size_t)d.in * 2;
-    return kWsStatusBytes + (size_t)tokens * (size_t)d.in * 2;
+    return gemm_x16_offset(tokens) + (size_t)tokens * (size_t)d.in * 2;
 }
 
 // Records a failed CUDA call (thread-local text for aq_last_error) and returns AQ_ERR_CUDA.
@@ -271,6 +276,14 @@ __device__ __forceinline__ uint32_t unit_code(const unsigned char* u, int p) {
     else if constexpr (B == 8) return u[p];
     else return ((const uint16_t*)u)[p];
 }
+
+// floor(log2(v)) for a finite v > 0 (subnormals count as 2^-126), from the exponent field.
+__device__ __forceinline__ int exponent_of(float v) {
+    const int e = (int)((__float_as_uint(v) >> 23) & 0xffu);
+    return (e == 0 ? 1 : e) - 127;
+}
+// 2^e as a float, for -126 <= e <= 127.
+__device__ __forceinline__ float pow2f(int e) { return __uint_as_float((uint32_t)(e + 127) << 23); }
 
 // Record a device-side failure in the workspace status word (first error wins).
 __device__ __forceinline__ void record_status(unsigned int* status, unsigned int code) {

@@ -86,9 +86,10 @@ struct GemmLayout {
     static constexpr int kNumBars = 2 * kStagesA + 4 * kStagesB + 4 + 1;
     static constexpr int kOffTmem = kOffBar + kNumBars * 8;
     static constexpr int kOffAbort = kOffTmem + 16;
+    static constexpr int kOffWmax = kOffAbort + 16;        // per-book largest |entry| (8 words)
     // The kernel has no static shared memory, so its dynamic shared memory starts on a
     // 1024-byte boundary (checked at run time: the 128-byte swizzled tiles need it).
-    static constexpr int kSmem = kOffAbort + 16;
+    static constexpr int kSmem = kOffWmax + 32;
     static_assert(kSmem <= 227 * 1024, "shared memory map exceeds the per-CTA limit");
 };
 
@@ -105,6 +106,52 @@ __device__ __forceinline__ uint32_t f16x2(float2 v) {   // {lo, hi} -> packed fp
     uint32_t h;
     asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(h) : "f"(v.y), "f"(v.x));
     return h;
+}
+
+// fp16 range for any input (R9). The MMA operands are fp16; bf16 activations and bf16
+// codebooks can hold values far outside fp16's range (and fp16 books' sums can exceed it).
+// Both are therefore scaled by powers of two, which is exact: each token row of bf16
+// activations by 2^-e_t so that its largest |x| lies in [2^14, 2^15) (bf16_rows_to_f16_kernel),
+// and the codebooks by 2^-f so that the largest possible |sum of m codewords| (the sum over
+// the books of their largest |entry|) lies below 2^15 (for bf16 books also at least 2^14, so
+// that small weights do not fall into fp16's subnormal range; fp16 books are only scaled down,
+// and a single fp16 book not at all). The epilogue multiplies by 2^(e_t + f). Where nothing
+// was out of range the result is bit-identical to the unscaled computation.
+
+// Largest |entry| of a codeword of eight 16-bit values, as the bits of a non-negative float
+// (monotonic in the value, so unsigned maxima of them are maxima of the values).
+template <int BDT>
+__device__ __forceinline__ unsigned int codeword_max_bits(const uint4& c) {
+    float f[8];
+    unpack8<BDT>(c, f);
+    float mx = 0.0f;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) mx = fmaxf(mx, fabsf(f[e]));
+    return __float_as_uint(mx);
+}
+
+// f of the codebooks of prefix m from the per-book largest |entry| (float bits).
+template <int BDT>
+__device__ __forceinline__ int book_exponent(const unsigned int* wmax, int m) {
+    if (BDT == AQ_F16 && m == 1) return 0;   // one fp16 codeword is an fp16 value already
+    float tot = 0.0f;
+    for (int k = 0; k < m; ++k) tot += __uint_as_float(wmax[k]);
+    if (!(tot > 0.0f)) return 0;             // all-zero books (or NaN entries)
+    int f = exponent_of(fminf(tot, 3.0e38f)) - 14;
+    if (BDT == AQ_F16 && f < 0) f = 0;
+    return max(-100, min(100, f));
+}
+
+// A codeword times sc (a power of two), back in its own type.
+template <int BDT>
+__device__ __forceinline__ uint4 scale_codeword(const uint4& c, float sc) {
+    float f[8];
+    unpack8<BDT>(c, f);
+    uint16_t h[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) h[e] = f32_to_bits<BDT>(f[e] * sc);
+    return make_uint4(h[0] | ((uint32_t)h[1] << 16), h[2] | ((uint32_t)h[3] << 16),
+                      h[4] | ((uint32_t)h[5] << 16), h[6] | ((uint32_t)h[7] << 16));
 }
 
 // Decoded group (eight fp16 weights): sum of the MB codewords in fp32, in book order, rounded
@@ -153,8 +200,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
             const uint8_t* __restrict__ planes,
             const uint16_t* __restrict__ books, const uint16_t* __restrict__ scales, void* y,
-            int y_dt, int scale_dt, unsigned int* __restrict__ status, int tokens, int out,
-            int in, int ng, int rows_pad, size_t plane_bytes) {
+            int y_dt, int scale_dt, unsigned int* __restrict__ status,
+            const float* __restrict__ xfac, int tokens, int out, int in, int ng, int rows_pad,
+            size_t plane_bytes) {
     static_assert(!DENSE || (MB == 1 && NP == 1), "dense tiles: one instantiation");
     using GL = GemmLayout<MB>;
     constexpr int kStagesA = GL::kStagesA, kStagesB = GL::kStagesB, kCodeBuf = GL::kCodeBuf;
@@ -402,11 +450,30 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
         const int c0 = cs * GPT;
         const int row = rd0 + n;
         const int nn = (int)pair * DR + n;          // its row in the weight operand tile
-        if constexpr (!DENSE)
-            for (int i = dt; i < m * 256; i += kDecWarps * 32)
-                books_s[i] = __ldg((const uint4*)books + i);
+        // Books staged times 2^-f (fp16 range, above), 2^f folded into the row scales; the
+        // dense variant's writer staged its books the same way and left 2^f in the workspace.
+        float wfac = 1.0f;
+        if constexpr (!DENSE) {
+            unsigned int* wmax_s = (unsigned int*)(smem + GL::kOffWmax);
+            if (dt < 8) wmax_s[dt] = 0u;
+            named_barrier(1, kDecWarps * 32);
+            uint4 cw[MB];               // codeword dt of every book (256 per book, 256 threads)
+#pragma unroll
+            for (int k = 0; k < MB; ++k) {
+                cw[k] = __ldg((const uint4*)books + k * 256 + dt);
+                atomicMax(&wmax_s[k], codeword_max_bits<BDT>(cw[k]));
+            }
+            named_barrier(1, kDecWarps * 32);
+            const int f = book_exponent<BDT>(wmax_s, MB);
+            wfac = pow2f(f);
+#pragma unroll
+            for (int k = 0; k < MB; ++k)
+                books_s[k * 256 + dt] = f ? scale_codeword<BDT>(cw[k], pow2f(-f)) : cw[k];
+        } else {
+            wfac = *(const volatile float*)((const char*)status + kWsWfacOffset);
+        }
         for (int i = dt; i < kBN; i += kDecWarps * 32)
-            scale_s[i] = (n0 + i < out) ? bits_to_f32_rt(scales[n0 + i], scale_dt) : 0.0f;
+            scale_s[i] = (n0 + i < out) ? bits_to_f32_rt(scales[n0 + i], scale_dt) * wfac : 0.0f;
         named_barrier(1, kDecWarps * 32);
 
         const int r = row & 31;                     // rotation of this row's codes
@@ -494,9 +561,13 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
             const int q = warp & 3;                       // tensor-memory lane quarter
             const int i = (warp - kDecWarp0) >> 2;        // token block (accumulator)
             const int t = t0 + i * 2 * kBM + (int)rank * kBM + q * 32 + lane;
+            const float xf = (xfac && t < tokens) ? xfac[t] : 1.0f;   // 2^e_t (bf16 activations)
             for (int nc = 0; nc < kBN; nc += 32) {
                 float v[32];
                 tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + i * kBN + nc, v);
+                if (xf != 1.0f)
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) v[e] *= xf;   // exact: a power of two
                 if (t < tokens) {
                     const size_t base = (size_t)t * out + n0 + nc;
                     if (vec && n0 + nc + 32 <= out) {
@@ -546,24 +617,54 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     }
 }
 
-// bf16 -> fp16 copy of the activations (8 values per thread; saturating at +-65504).
-__global__ void __launch_bounds__(256) bf16_to_f16_kernel(const uint4* __restrict__ src,
-                                                          uint4* __restrict__ dst, size_t n8) {
+// bf16 -> fp16 copy of the activations, one token row per CTA (grid-stride over the rows): the
+// row is multiplied by 2^-e_t, e_t chosen so that its largest |x| lies in [2^14, 2^15), which is
+// exact (a power of two; bf16's 8 significant bits fit fp16's 11 wherever the scaled value is
+// in fp16's normal range), and 2^e_t is stored for the epilogue. An all-zero row keeps e_t = 0.
+__global__ void __launch_bounds__(256) bf16_rows_to_f16_kernel(const uint16_t* __restrict__ src,
+                                                               uint16_t* __restrict__ dst,
+                                                               float* __restrict__ xfac, int in,
+                                                               int tokens) {
+    __shared__ unsigned int red[8];
     pdl_wait();
     pdl_launch_dependents();
-    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n8;
-         i += (size_t)gridDim.x * blockDim.x) {
-        const uint4 v = src[i];
-        float f[8];
-        unpack8<AQ_BF16>(v, f);
-        uint32_t o[4];
+    const int n8 = in / 8, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int t = blockIdx.x; t < tokens; t += gridDim.x) {
+        const uint4* row = (const uint4*)(src + (size_t)t * in);
+        unsigned int mx = 0;            // largest |bf16| bit pattern of the row
+        for (int i = threadIdx.x; i < n8; i += blockDim.x) {
+            const uint4 v = row[i];
+            const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            uint32_t h;
-            asm("cvt.rn.satfinite.f16x2.f32 %0, %1, %2;" : "=r"(h) : "f"(f[2 * e + 1]), "f"(f[2 * e]));
-            o[e] = h;
+            for (int e = 0; e < 4; ++e) mx = max(mx, max(w[e] & 0x7fffu, (w[e] >> 16) & 0x7fffu));
         }
-        dst[i] = make_uint4(o[0], o[1], o[2], o[3]);
+        mx = __reduce_max_sync(0xffffffffu, mx);
+        if (lane == 0) red[warp] = mx;
+        __syncthreads();
+        mx = red[0];
+        for (int w = 1; w < 8; ++w) mx = max(mx, red[w]);
+        __syncthreads();                // red is reused by the next row
+        int et = 0;
+        if (mx != 0) {
+            const int eb = (int)((mx >> 7) & 0xffu);           // biased bf16 exponent
+            et = max(-100, min(100, (eb == 0 ? 1 : eb) - 127 - 14));
+        }
+        const float sc = pow2f(-et);
+        uint4* out = (uint4*)(dst + (size_t)t * in);
+        for (int i = threadIdx.x; i < n8; i += blockDim.x) {
+            const uint4 v = row[i];
+            float f[8];
+            unpack8<AQ_BF16>(v, f);
+            uint32_t o[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                uint32_t h;
+                asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(h) : "f"(f[2 * e + 1] * sc), "f"(f[2 * e] * sc));
+                o[e] = h;
+            }
+            out[i] = make_uint4(o[0], o[1], o[2], o[3]);
+        }
+        if (threadIdx.x == 0) xfac[t] = pow2f(et);
     }
 }
 
@@ -578,8 +679,8 @@ int gemm_pairs_per_cluster(int m, int tokens) {
 
 template <int BDT>
 aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
-                   const void* scales, const void* x, int tokens, void* y, int y_dt, void* ws,
-                   cudaStream_t st) {   // x: fp16 [tokens][in]
+                   const void* scales, const void* x, const float* xfac, int tokens, void* y,
+                   int y_dt, void* ws, cudaStream_t st) {   // x: fp16 [tokens][in]
     EncodeTiledFn encode;
     if (aq_status e = get_encode_fn(&encode); e != AQ_OK) return e;
     CUtensorMap map;
@@ -597,7 +698,7 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
     // (m >= 2) and every pair of a cluster has tokens (one 512-token tile per pair).
     const int np = gemm_pairs_per_cluster(m, tokens);
     using Kern = void (*)(const CUtensorMap, const CUtensorMap, const uint8_t*, const uint16_t*, const uint16_t*,
-                          void*, int, int, unsigned int*, int, int, int, int, int, size_t);
+                          void*, int, int, unsigned int*, const float*, int, int, int, int, int, size_t);
     const Kern k1[kGemmMaxM] = {gemm_kernel<BDT, 1, 1>, gemm_kernel<BDT, 2, 1>, gemm_kernel<BDT, 3, 1>,
                                 gemm_kernel<BDT, 4, 1>, gemm_kernel<BDT, 5, 1>, gemm_kernel<BDT, 6, 1>,
                                 gemm_kernel<BDT, 7, 1>, gemm_kernel<BDT, 8, 1>};
@@ -648,9 +749,9 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
     std::memset(&unused, 0, sizeof(unused));
     return cuda_ok(cudaLaunchKernelEx(&cfg, kern, map, unused, (const uint8_t*)planes,
                                       (const uint16_t*)books, (const uint16_t*)scales, y, y_dt,
-                                      d.scale_dt, (unsigned int*)ws, tokens, d.out, d.in, d.ng,
+                                      d.scale_dt, (unsigned int*)ws, xfac, tokens, d.out, d.in, d.ng,
                                       d.rows_pad, d.plane_bytes),
-                   "cudaLaunchKernelEx");
+                   "cudaLaunchKernelEx (GEMM)");
 }
 
 // ---- dense variant: W_m decoded once into the workspace, then TMA-fed pair MMAs -----------
@@ -665,16 +766,30 @@ constexpr int kDenseWarps = 8;
 template <int B, int BDT>
 __global__ void __launch_bounds__(kDenseWarps * 32)
 dense_w_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
-               uint16_t* __restrict__ w16, int m, int out, int in, int ng, int rows_pad, int RBc,
-               size_t plane_bytes) {
+               uint16_t* __restrict__ w16, float* __restrict__ wfac_out, int m, int out, int in,
+               int ng, int rows_pad, int RBc, size_t plane_bytes) {
     constexpr int UNIT = unit_bytes(B);
     extern __shared__ __align__(16) unsigned char smem_d[];
     uint4* books_s = (uint4*)smem_d;                 // [m][2^B] codewords
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     unsigned char* codes_s = smem_d + staged_books_bytes(B, m) + (size_t)warp * m * 32 * UNIT;
+    __shared__ unsigned int wmax[8];
     pdl_wait();
     pdl_launch_dependents();
-    for (int i = threadIdx.x; i < (m << B); i += blockDim.x) books_s[i] = __ldg((const uint4*)books + i);
+    // Books staged times 2^-f (fp16 range, as in the GEMM's decoders); 2^f goes to the
+    // workspace for the GEMM's epilogue (every CTA finds the same f; CTA 0 writes it).
+    if (threadIdx.x < 8) wmax[threadIdx.x] = 0u;
+    __syncthreads();
+    for (int i = threadIdx.x; i < (m << B); i += blockDim.x) {
+        const uint4 c = __ldg((const uint4*)books + i);
+        atomicMax(&wmax[i >> B], codeword_max_bits<BDT>(c));
+        books_s[i] = c;
+    }
+    __syncthreads();
+    const int f = book_exponent<BDT>(wmax, m);
+    if (f)
+        for (int i = threadIdx.x; i < (m << B); i += blockDim.x) books_s[i] = scale_codeword<BDT>(books_s[i], pow2f(-f));
+    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *wfac_out = pow2f(f);
     const int s = blockIdx.y;
     const int rb = blockIdx.x * kDenseWarps + warp;
     const bool active = rb < RBc;
@@ -714,12 +829,14 @@ dense_w_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ 
 
 template <int B, int BDT>
 aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* books,
-                         const void* scales, const void* x, int tokens, void* y, int y_dt,
-                         void* ws, uint16_t* w16, cudaStream_t st) {   // x: fp16 [tokens][in]
+                         const void* scales, const void* x, const float* xfac, int tokens, void* y,
+                         int y_dt, void* ws, uint16_t* w16, cudaStream_t st) {   // x: fp16 [tokens][in]
     {   // decode W_m once
         const size_t smem = staged_books_bytes(B, m) + (size_t)kDenseWarps * m * 32 * unit_bytes(B);
         auto kern = dense_w_kernel<B, BDT>;
-        if (smem > 48 * 1024)
+        // (the kernel also has a few bytes of static shared memory, so the default 48 KiB
+        // limit on the total is raised already from 32 KiB of dynamic memory)
+        if (smem > 32 * 1024)
             if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
                 e != cudaSuccess)
                 return cuda_fail(e, "cudaFuncSetAttribute");
@@ -734,8 +851,9 @@ aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* b
         cfg.attrs = attr;
         cfg.numAttrs = 1;
         if (aq_status e = cuda_ok(cudaLaunchKernelEx(&cfg, kern, (const uint8_t*)planes, (const uint16_t*)books,
-                                                     w16, m, d.out, d.in, d.ng, d.rows_pad, d.RBc, d.plane_bytes),
-                                  "cudaLaunchKernelEx");
+                                                     w16, (float*)((char*)ws + kWsWfacOffset), m, d.out,
+                                                     d.in, d.ng, d.rows_pad, d.RBc, d.plane_bytes),
+                                  "cudaLaunchKernelEx (dense W_m)");
             e != AQ_OK)
             return e;
     }
@@ -793,8 +911,8 @@ aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* b
     cfg.numAttrs = 2;
     return cuda_ok(cudaLaunchKernelEx(&cfg, kern, xm, wm, (const uint8_t*)planes, (const uint16_t*)books,
                                       (const uint16_t*)scales, y, y_dt, d.scale_dt, (unsigned int*)ws,
-                                      tokens, d.out, d.in, d.ng, d.rows_pad, d.plane_bytes),
-                   "cudaLaunchKernelEx");
+                                      xfac, tokens, d.out, d.in, d.ng, d.rows_pad, d.plane_bytes),
+                   "cudaLaunchKernelEx (dense GEMM)");
 }
 
 }  // namespace
@@ -805,14 +923,15 @@ aq_status launch_gemm(const Dims& d, int m, const void* planes, const void* book
     if (d.out == 0 || tokens == 0) return AQ_OK;
     if ((d.B != 8 && d.B != 4) || m > kGemmMaxM) return AQ_ERR_UNSUPPORTED;
     const void* xh = x;
+    const float* xfac = nullptr;
     if (x_dt == AQ_BF16) {
-        // fp16 copy of the activations after the status word of the workspace
-        void* dst = (char*)ws + kWsStatusBytes;
-        const size_t n8 = (size_t)tokens * d.in / 8;
+        // fp16 copy of the activations, each token row scaled into fp16's range, and the
+        // per-token factors, in the workspace
+        void* dst = (char*)ws + gemm_x16_offset(tokens);
+        float* fac = (float*)((char*)ws + gemm_xfac_offset());
         DeviceInfo di;
         if (aq_status e = device_info(&di); e != AQ_OK) return e;
-        const size_t want = (n8 + 255) / 256;
-        const int blocks = (int)(want < (size_t)di.sms * 8 ? want : (size_t)di.sms * 8);
+        const int blocks = tokens < di.sms * 8 ? tokens : di.sms * 8;
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(blocks);
         cfg.blockDim = dim3(256);
@@ -822,26 +941,27 @@ aq_status launch_gemm(const Dims& d, int m, const void* planes, const void* book
         attr[0].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
-        if (aq_status e = cuda_ok(cudaLaunchKernelEx(&cfg, bf16_to_f16_kernel, (const uint4*)x,
-                                                     (uint4*)dst, n8),
-                                  "cudaLaunchKernelEx");
+        if (aq_status e = cuda_ok(cudaLaunchKernelEx(&cfg, bf16_rows_to_f16_kernel, (const uint16_t*)x,
+                                                     (uint16_t*)dst, fac, d.in, tokens),
+                                  "cudaLaunchKernelEx (activation copy)");
             e != AQ_OK)
             return e;
         xh = dst;
+        xfac = fac;
     }
     if (gemm_uses_dense(d, m, tokens)) {
         uint16_t* w16 = (uint16_t*)((char*)ws + gemm_w16_offset(d, tokens));
         if (d.B == 4)   // the in-loop decoders read 8-bit codes; 4-bit layouts always go dense
             return d.book_dt == AQ_BF16
-                       ? run_gemm_dense<4, AQ_BF16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, w16, st)
-                       : run_gemm_dense<4, AQ_F16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, w16, st);
+                       ? run_gemm_dense<4, AQ_BF16>(d, m, planes, books, scales, xh, xfac, tokens, y, y_dt, ws, w16, st)
+                       : run_gemm_dense<4, AQ_F16>(d, m, planes, books, scales, xh, xfac, tokens, y, y_dt, ws, w16, st);
         return d.book_dt == AQ_BF16
-                   ? run_gemm_dense<8, AQ_BF16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, w16, st)
-                   : run_gemm_dense<8, AQ_F16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, w16, st);
+                   ? run_gemm_dense<8, AQ_BF16>(d, m, planes, books, scales, xh, xfac, tokens, y, y_dt, ws, w16, st)
+                   : run_gemm_dense<8, AQ_F16>(d, m, planes, books, scales, xh, xfac, tokens, y, y_dt, ws, w16, st);
     }
     return d.book_dt == AQ_BF16
-               ? run_gemm<AQ_BF16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, st)
-               : run_gemm<AQ_F16>(d, m, planes, books, scales, xh, tokens, y, y_dt, ws, st);
+               ? run_gemm<AQ_BF16>(d, m, planes, books, scales, xh, xfac, tokens, y, y_dt, ws, st)
+               : run_gemm<AQ_F16>(d, m, planes, books, scales, xh, xfac, tokens, y, y_dt, ws, st);
 }
 
 }  // namespace aq

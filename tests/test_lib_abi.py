@@ -165,21 +165,26 @@ def test_wmse_sizes_and_argument_errors_on_the_host():
     assert call(_lay(), ws=FAKE + 8) == aq.AQ_ERR_ALIGNMENT
 
 
+def _x16(tokens):
+    """Offset of the fp16 activation copy: status block, then one float per token."""
+    return 256 + (tokens * 4 + 255) // 256 * 256
+
+
 def test_gemm_workspace_sizes():
-    """Status word + fp16 activation copy; from 2048 tokens (two or more books) also room for
-    W_m decoded once in fp16."""
+    """Status block + per-token activation factors + fp16 activation copy; from 2048 tokens
+    (two or more books) also room for W_m decoded once in fp16."""
     L = aq.Layout.make(300, 520, 4)
-    assert aq.gemm_workspace_bytes(L, 2047) == 256 + 2047 * 520 * 2
-    off = (256 + 2048 * 520 * 2 + 1023) // 1024 * 1024
+    assert aq.gemm_workspace_bytes(L, 2047) == _x16(2047) + 2047 * 520 * 2
+    off = (_x16(2048) + 2048 * 520 * 2 + 1023) // 1024 * 1024
     assert aq.gemm_workspace_bytes(L, 2048) == off + 300 * 520 * 2
     L1 = aq.Layout.make(300, 520, 1)
-    assert aq.gemm_workspace_bytes(L1, 4096) == 256 + 4096 * 520 * 2
+    assert aq.gemm_workspace_bytes(L1, 4096) == _x16(4096) + 4096 * 520 * 2
 
 
 def test_gemm_workspace_for_4bit_codes():
     """4-bit layouts always decode W_m into the workspace first."""
     L = aq.Layout.make(300, 520, 4, B=4)
-    off = (256 + 40 * 520 * 2 + 1023) // 1024 * 1024
+    off = (_x16(40) + 40 * 520 * 2 + 1023) // 1024 * 1024
     assert aq.gemm_workspace_bytes(L, 40) == off + 300 * 520 * 2
     assert aq.plane_bytes(L) == 320 * 96 // 2
 
