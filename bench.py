@@ -33,7 +33,9 @@ WORKLOAD = "attn_4096"
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--steps", type=int, default=40000,
+                    help="timed steps (replays of a graph of at most 200 steps; the default "
+                         "keeps the timed region about a second long)")
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="own", choices=["own", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -49,6 +51,13 @@ def parse():
                     help="tokens of the prefill GEMM case (smaller values: profiling runs)")
     ap.add_argument("--skip-gemv", action="store_true",
                     help="only the GEMM case (profiling runs; prints no bench line)")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the per-configuration GEMV table (8B block, 1024^2, large books)")
+    ap.add_argument("--profile-gemv", metavar="WORKLOAD[:LAYER]",
+                    help="only three aq_gemv calls of one workload layer (for ncu captures; "
+                         "prints no bench line), with --batch and --m")
+    ap.add_argument("--batch", type=int, default=1)
+    ap.add_argument("--m", type=int, default=1)
     return ap.parse_args()
 
 
@@ -130,7 +139,7 @@ class ClockSampler:
             os.close(fd)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.dev), "--query-gpu=" + self.FIELDS,
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
             time.sleep(0.3)
         except (OSError, FileNotFoundError):
@@ -365,6 +374,123 @@ def measure_wmse(lin, dev, stream, peaks, reps=10):
             "peak_source": "measured" if "bf16_tflops" in peaks else "fallback"}
 
 
+def graph_us(calls, n, stream, reps=5):
+    """us per call of a CUDA graph of n calls (calls(i) enqueues call i; weight copies rotate
+    inside it): median over reps replays, events around the graph only, so back-to-back calls
+    keep their overlap."""
+    import torch
+    for i in range(3):
+        calls(i)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(n):
+            calls(i)
+    g.replay()
+    torch.cuda.synchronize()
+    ts = []
+    for _ in range(reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record()
+            g.replay()
+            e1.record()
+        torch.cuda.synchronize()
+        ts.append(e0.elapsed_time(e1) * 1e3 / n)
+    del g
+    return statistics.median(ts)
+
+
+def fp32_alu_peak_tflops(sm_mhz, sms=152):
+    """CUDA-core fp32 peak: 128 FMA lanes per SM, 2 flops per FMA, at the SM clock."""
+    return sms * 128 * 2 * sm_mhz * 1e6 / 1e12
+
+
+def measure_configs(dev, stream, hbm_peak, sm_mhz):
+    """Batch-1..16 GEMV over the paper-shaped layers (per prefix m): the 1024^2 layer
+    (batch 1), the Llama-3-8B block (each linear and the summed block, batch 1 and 8, bf16
+    activations), the 8192^2 layer with 2^16-entry books (batch 1 and 16) and the 4096^2
+    attention projection at batch 4 and 16. us per call from graphs of back-to-back calls over
+    weight copies that together exceed 3x L2; GB/s = algorithmic bytes / time; for batch > 1
+    also the fraction of the CUDA-core fp32 FMA roofline (2 * batch flops per weight)."""
+    import torch
+    import paper_2606_12876_gb300 as aq
+    from paper_2606_12876_gb300.linear import AQLinear, x_to_device
+    import workloads
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    alu_peak = fp32_alu_peak_tflops(sm_mhz)
+    res = {"alu_peak_TFLOP_s": round(alu_peak, 1),
+           "alu_peak_basis": "152 SMs x 128 fp32 lanes x 2 flops x %.0f MHz (median SM clock "
+                             "of the headline run)" % sm_mhz}
+
+    def layer_entry(lin, xdt, batch, ms):
+        xc = aq.AQ_F16 if xdt == "f16" else aq.AQ_BF16
+        x = x_to_device(workloads.make_x(batch, lin.inp, xdt, seed=batch), xdt)
+        y = torch.empty(batch, lin.out, dtype=x.dtype, device=dev)
+        ws = aq.workspace(aq.gemv_workspace_bytes(lin.layout, batch), dev)
+        nc = max(2, -(-3 * l2 // lin.planes.numel()))
+        copies = [lin.planes.clone() for _ in range(nc)]
+        rows = []
+        for m in ms:
+            with torch.cuda.stream(stream):
+                us = graph_us(lambda i, m=m: aq.aq_gemv(lin.layout, m, copies[i % nc], lin.books,
+                                                        lin.scales, x, xc, batch, y, xc, ws), 20, stream)
+            nb = layer_bytes(lin.out, lin.inp, m, B=lin.B, batch=batch)
+            e = {"m": m, "bits_per_weight": m * lin.B // 8, "us": round(us, 3),
+                 "GB_s": round(nb / us / 1e3, 1), "frac_hbm": round(nb / us / 1e3 / hbm_peak, 4)}
+            if batch > 1:
+                tf = 2.0 * batch * lin.out * lin.inp / (us * 1e-6) / 1e12
+                e["TFLOP_s"] = round(tf, 2)
+                e["frac_alu"] = round(tf / alu_peak, 4)
+            rows.append(e)
+        del copies
+        return rows
+
+    def cfg_layers(name):
+        return [(n, AQLinear.from_layer(l, device=dev)) for n, l in workloads.config_layers(name)]
+
+    (_, lin1), = cfg_layers("single_1024")
+    res["single_1024"] = {"b1": layer_entry(lin1, "f16", 1, (1, 2))}
+    (_, lina), = cfg_layers("attn_4096")
+    res["attn_4096"] = {"b%d" % b: layer_entry(lina, "f16", b, (1, 2, 3, 4)) for b in (4, 16)}
+    blk = cfg_layers("llama8b_block")
+    res["llama8b_block"] = {n: {"b%d" % b: layer_entry(lin, "bf16", b, (1, 2, 3, 4)) for b in (1, 8)}
+                            for n, lin in blk}
+    # the summed block: the seven calls back to back in one graph, three weight copies each
+    for b in (1, 8):
+        xs = {}
+        for _, lin in blk:
+            if lin.inp not in xs:
+                xs[lin.inp] = x_to_device(workloads.make_x(b, lin.inp, "bf16", seed=b), "bf16")
+        ys = [torch.empty(b, lin.out, dtype=torch.bfloat16, device=dev) for _, lin in blk]
+        wss = [aq.workspace(aq.gemv_workspace_bytes(lin.layout, b), dev) for _, lin in blk]
+        cps = [[lin.planes.clone() for _ in range(3)] for _, lin in blk]
+        rows = []
+        for m in (1, 2, 3, 4):
+            def step(i, m=m):
+                for j, (_, lin) in enumerate(blk):
+                    aq.aq_gemv(lin.layout, m, cps[j][i % 3], lin.books, lin.scales, xs[lin.inp],
+                               aq.AQ_BF16, b, ys[j], aq.AQ_BF16, wss[j])
+            with torch.cuda.stream(stream):
+                us = graph_us(step, 10, stream)
+            nb = sum(layer_bytes(lin.out, lin.inp, m, batch=b) for _, lin in blk)
+            e = {"m": m, "us": round(us, 3), "GB_s": round(nb / us / 1e3, 1),
+                 "frac_hbm": round(nb / us / 1e3 / hbm_peak, 4)}
+            if b > 1:
+                tf = 2.0 * b * sum(lin.out * lin.inp for _, lin in blk) / (us * 1e-6) / 1e12
+                e["TFLOP_s"] = round(tf, 2)
+                e["frac_alu"] = round(tf / alu_peak, 4)
+            rows.append(e)
+        res["llama8b_block"]["block_sum_b%d" % b] = rows
+        del cps
+    del blk
+    (_, linb), = cfg_layers("big_book_8192")
+    res["big_book_8192"] = {"b%d" % b: layer_entry(linb, "f16", b, (1, 2)) for b in (1, 16)}
+    res["big_book_8192"]["note"] = ("2^16-entry books (1 MiB each) are gathered through L2; "
+                                    "frac_hbm counts the algorithmic bytes of the call")
+    return res
+
+
 def own_arm(args):
     import numpy as np
     import torch
@@ -445,7 +571,12 @@ def own_arm(args):
         torch.cuda.synchronize(dev)
         return e0.elapsed_time(e1)
 
-    g_warm, g_timed = capture(step, args.warmup), capture(step, args.steps)
+    # The timed steps run as replays of one graph of at most 200 steps (and one graph for the
+    # remainder), so that a long timed region needs no long capture.
+    glen = min(args.steps, 200)
+    g_warm, g_timed = capture(step, args.warmup), capture(step, glen)
+    rest = args.steps % glen
+    g_rest = capture(step, rest) if rest else None
     torch.cuda.synchronize(dev)
 
     def barrier():
@@ -457,9 +588,20 @@ def own_arm(args):
     clocks = ClockSampler(local)
     clocks.start()
     barrier()
-    ms_total = time_graph(g_timed)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize(dev)
+    with torch.cuda.stream(stream):
+        e0.record()
+        for _ in range(args.steps // glen):
+            g_timed.replay()
+        if g_rest is not None:
+            g_rest.replay()
+        e1.record()
+    torch.cuda.synchronize(dev)
+    ms_total = e0.elapsed_time(e1)
     barrier()
     clk = clocks.stop()
+    del g_rest
     ms_total, value = whole_job(ms_total, world, bytes_step, args.steps, device=dev)
     ms_step = ms_total / args.steps
 
@@ -469,9 +611,9 @@ def own_arm(args):
     # events around it, median of 7.
     per_m_us, single_us = {}, {}
     for m in ms:
-        g = capture(lambda i, m=m: call(i, m), args.steps)
+        g = capture(lambda i, m=m: call(i, m), glen)
         g.replay()
-        per_m_us[m] = statistics.median(time_graph(g) for _ in range(5)) * 1e3 / args.steps
+        per_m_us[m] = statistics.median(time_graph(g) for _ in range(5)) * 1e3 / glen
         del g
         lat = []
         with torch.cuda.stream(stream):
@@ -494,9 +636,9 @@ def own_arm(args):
         prev = ys32[m - 1] if m > 1 else None
         g = capture(lambda i, m=m, prev=prev: aq.aq_gemv_refine(
             L, m, copies[i % ncopies], lin.books, lin.scales, x, aq.AQ_F16, 1, prev, ys32[m],
-            aq.AQ_F32, ws), args.steps)
+            aq.AQ_F32, ws), glen)
         g.replay()
-        refine_us[m] = time_graph(g) * 1e3 / args.steps
+        refine_us[m] = time_graph(g) * 1e3 / glen
         del g
     refine_bytes = layer_bytes(out, inp, 1, ysize=4) + 4 * out   # one plane; y_prev read too
 
@@ -520,7 +662,7 @@ def own_arm(args):
         x_dev = torch.empty_like(x_host, device=dev)
         y_dev = torch.empty(len(ms), out, dtype=torch.float16, device=dev)   # one row per m
         e_s, e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        n_e2e = max(20, args.steps // 2)
+        n_e2e = max(20, min(args.steps // 2, 2000))
         with torch.cuda.stream(stream):
             for i in range(args.warmup + n_e2e):
                 if i == args.warmup:
@@ -541,6 +683,9 @@ def own_arm(args):
                "api": "paper_2606_12876_gb300.aq_gemv (ctypes -> libaq.so), eager"}
 
     gemm = None if args.no_gemm else measure_gemm(dev, stream, peaks, tokens=args.gemm_tokens)
+    configs = None
+    if rank == 0 and not args.no_configs:
+        configs = measure_configs(dev, stream, hbm_peak, clk.get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0))
     loading = measure_loading(lin, dev, stream, ms) if rank == 0 and not args.no_loading else None
     wmse = None if args.no_wmse else measure_wmse(lin, dev, stream, peaks)
 
@@ -572,6 +717,7 @@ def own_arm(args):
                        "l2": "rotating %d weight copies (%d x %.1f MB >= 3x L2 %.0f MB)" % (
                            ncopies, ncopies, pbytes / 1e6, l2 / 1e6)},
             "per_m": per_m,
+            "configs": configs,
             "gemm": gemm,
             "dynamic_loading": loading,
             "wmse": wmse,
@@ -584,6 +730,8 @@ def own_arm(args):
             "cpu_baseline": cpu,
             "e2e": e2e,
             "gpu_launches": 2 * len(ms) * args.steps,   # product + split-K reduction per call
+            "timed_region": {"graph_steps": glen, "replays": args.steps // glen,
+                             "remainder_steps": rest, "ms": round(ms_total, 3)},
             "clocks": clk,
         }
         print(json.dumps(line), flush=True)
@@ -591,8 +739,29 @@ def own_arm(args):
         torch.distributed.destroy_process_group()
 
 
+def profile_gemv(args):
+    """Three aq_gemv calls of one layer of a named workload, nothing else (ncu captures)."""
+    import torch
+    from paper_2606_12876_gb300 import build as libbuild
+    from paper_2606_12876_gb300.linear import AQLinear, x_to_device
+    import workloads
+    libbuild.build()
+    name, _, lname = args.profile_gemv.partition(":")
+    (_, layer), = list(workloads.config_layers(name, only=[lname] if lname else None))
+    lin = AQLinear.from_layer(layer)
+    xdt = workloads.CONFIGS[name]["x_dtype"]
+    x = x_to_device(workloads.config_x(name, args.batch, layer["in"]), xdt)
+    for _ in range(3):
+        lin.gemv(x, args.m)
+    torch.cuda.synchronize()
+    print("profiled %s batch %d m %d" % (args.profile_gemv, args.batch, args.m))
+
+
 def main():
     args = parse()
+    if args.profile_gemv:
+        profile_gemv(args)
+        return
     if args.impl == "reference":
         reference_arm(args)
     else:
