@@ -287,12 +287,17 @@ aq_status aq_store_create(const aq_layout* layout, aq_store** store);
  * Each may be host memory (pinned, for a copy that runs asynchronously) or device memory, and
  * must stay valid until the copies have run. Work that reads the new prefix must be ordered
  * after them: enqueue it on stream, or make its stream wait for an event recorded there.
- * Lowering (m < m0) synchronises the device, so that no kernel can still be reading the
- * dropped planes, then unmaps the memory that only planes m..m0-1 use (the granule that plane
- * m-1 shares with plane m stays). The src pointers are not used and may be NULL. m = m0 does
- * nothing.
+ * Lowering (m < m0) is ordered on stream and does not wait: the memory that only planes
+ * m..m0-1 use (the granule that plane m-1 shares with plane m stays) is released once the
+ * work enqueued on stream before the call has finished. Work that reads the dropped planes
+ * must therefore be enqueued on stream before the call (or be ordered before it), and no
+ * later work may read them. The release itself happens in a later call on the store that
+ * finds that work finished (aq_store_set_prefix, aq_store_device_bytes, aq_store_destroy);
+ * a raise that needs the addresses again first takes the allocations back instead. No other
+ * stream of the process is made to wait. The src pointers are not used and may be NULL. m = m0
+ * does nothing.
  * Errors: AQ_ERR_INVALID_ARG (null store, m outside 0..M, a NULL src pointer that a raise
- * needs), AQ_ERR_CUDA (mapping or copy failed; the prefix then stays m0). */
+ * needs), AQ_ERR_CUDA (mapping, copy or event failed; the prefix then stays m0). */
 aq_status aq_store_set_prefix(aq_store* store, int m, const void* src_planes,
                               const void* src_books, const void* src_scales, void* stream);
 
@@ -304,8 +309,11 @@ int aq_store_prefix(const aq_store* store);
 void* aq_store_planes(const aq_store* store);
 void* aq_store_books(const aq_store* store);
 void* aq_store_scales(const aq_store* store);
-/* Bytes of device memory the store holds mapped (0 for a NULL store). */
-size_t aq_store_device_bytes(const aq_store* store);
+/* Bytes of device memory the store holds (0 for a NULL store): the scales, the codebooks, the
+ * resident planes and dropped planes whose release still waits for their stream. Dropped
+ * planes whose stream work has finished are released first, so after the caller's stream has
+ * been synchronised the count is that of the resident prefix. */
+size_t aq_store_device_bytes(aq_store* store);
 
 /* Synchronise the device, release the store's memory and address range, free the handle.
  * NULL: nothing (AQ_OK). Errors: AQ_ERR_CUDA if the synchronisation reported an error (the

@@ -3,16 +3,18 @@
 // One stored model serves every bit width, and a device holds as many codebooks as its memory
 // or latency budget allows (Sec. 1 and Sec. 5). Because the code planes are codebook-major,
 // the planes of a prefix m are one contiguous range, so growing the prefix appends planes and
-// shrinking it drops a tail.
+// shrinking it drops a tail. Dropping is ordered on the caller's stream: the dropped
+// allocations are released once that stream has passed the call (an event), checked at the
+// next call on the store, so no other stream of the process is made to wait.
 //
 // The store reserves device address space for the whole layer once and backs it with physical
 // memory through the CUDA virtual-memory calls (cuMemAddressReserve, cuMemCreate, cuMemMap):
 //   [head: scales | codebooks of all M books] [planes 0..M-1]
 // The head is mapped when the store is created (the codebooks are small: 2^B*16 bytes per
 // book); the plane range is mapped only as far as the resident prefix needs, in whole
-// allocation granules. Raising the prefix maps one more physical allocation behind the last
-// one and copies the new planes in; lowering it unmaps the allocations that lie wholly past
-// the new prefix. Addresses never move, so pointers into the store stay valid for its life
+// allocation granules. Raising the prefix maps one physical allocation per new plane (the
+// granules it does not share with the plane before) and copies the new planes in; lowering it
+// releases the allocations that lie wholly past the new prefix. Addresses never move, so pointers into the store stay valid for its life
 // (a plain allocation would have to be reallocated and copied to grow).
 //
 // The driver calls are looked up through the runtime (cudaGetDriverEntryPointByVersion), so
@@ -156,6 +158,12 @@ aq_status sync_device(int dev) {
 
 }  // namespace
 
+// A dropped plane allocation waiting for the work enqueued before its drop to finish.
+struct Pending {
+    Mapping mp;
+    cudaEvent_t done;
+};
+
 struct aq_store {
     Dims d;
     int dev;
@@ -168,6 +176,7 @@ struct aq_store {
     Mapping head;
     std::vector<Mapping> planes; // mappings of the plane range, in address order
     size_t planes_mapped;        // bytes of the plane range mapped (sum of `planes`)
+    std::vector<Pending> pending;  // dropped mappings above the resident ones, in address order
     int m;                       // resident prefix
 };
 
@@ -175,7 +184,7 @@ namespace {
 
 CUdeviceptr planes_base(const aq_store* s) { return s->base + s->head_bytes; }
 
-// Unmaps the plane mappings that lie wholly at or past `keep` bytes of the plane range.
+// Unmaps the plane mappings that lie wholly at or past `keep` bytes of the plane range, now.
 aq_status drop_planes(const Driver* drv, aq_store* s, size_t keep) {
     aq_status st = AQ_OK;
     while (!s->planes.empty() && s->planes.back().addr >= planes_base(s) + keep) {
@@ -187,7 +196,53 @@ aq_status drop_planes(const Driver* drv, aq_store* s, size_t keep) {
     return st;
 }
 
+// Releases the dropped mappings whose stream work has finished (all of them with wait).
+aq_status reap(const Driver* drv, aq_store* s, bool wait) {
+    aq_status st = AQ_OK;
+    for (size_t i = 0; i < s->pending.size();) {
+        Pending& p = s->pending[i];
+        const cudaError_t q = wait ? cudaEventSynchronize(p.done) : cudaEventQuery(p.done);
+        if (q == cudaErrorNotReady) {
+            ++i;
+            continue;
+        }
+        if (q != cudaSuccess && st == AQ_OK) st = aq::cuda_fail(q, "cudaEventQuery");
+        const aq_status e = unmap_one(drv, p.mp);
+        if (st == AQ_OK) st = e;
+        cudaEventDestroy(p.done);
+        s->pending.erase(s->pending.begin() + (long)i);
+    }
+    return st;
+}
+
+// Moves the mappings that lie wholly at or past `keep` bytes of the plane range to the pending
+// list, each with an event recorded on stream after the work enqueued so far.
+aq_status defer_drop(aq_store* s, size_t keep, cudaStream_t stream) {
+    std::vector<Pending> moved;
+    while (!s->planes.empty() && s->planes.back().addr >= planes_base(s) + keep) {
+        cudaEvent_t ev = nullptr;
+        if (cudaError_t e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming); e != cudaSuccess)
+            return aq::cuda_fail(e, "cudaEventCreateWithFlags");
+        if (cudaError_t e = cudaEventRecord(ev, stream); e != cudaSuccess) {
+            cudaEventDestroy(ev);
+            return aq::cuda_fail(e, "cudaEventRecord");
+        }
+        moved.push_back(Pending{s->planes.back(), ev});
+        s->planes_mapped -= s->planes.back().bytes;
+        s->planes.pop_back();
+    }
+    // keep the pending list in address order: the newly dropped mappings lie below the older
+    // pending ones
+    s->pending.insert(s->pending.begin(), moved.rbegin(), moved.rend());
+    return AQ_OK;
+}
+
 void release_all(const Driver* drv, aq_store* s) {
+    for (Pending& p : s->pending) {
+        unmap_one(drv, p.mp);
+        cudaEventDestroy(p.done);
+    }
+    s->pending.clear();
     drop_planes(drv, s, 0);
     if (s->head.bytes) unmap_one(drv, s->head);
     if (s->base) drv->addr_free(s->base, s->reserved);
@@ -244,30 +299,46 @@ extern "C" aq_status aq_store_set_prefix(aq_store* s, int m, const void* src_pla
     if (!s || m < 0 || m > s->d.M) return AQ_ERR_INVALID_ARG;
     const int m0 = s->m;
     if (m == m0) return AQ_OK;
+    if (m > m0 && (!src_planes || !src_books || (m0 == 0 && !src_scales))) return AQ_ERR_INVALID_ARG;
     const Driver* drv = nullptr;
     if (aq_status e = driver(&drv); e != AQ_OK) return e;
     const size_t pb = s->d.plane_bytes;
 
+    const cudaStream_t st = (cudaStream_t)stream;
+    // dropped allocations whose stream work has finished are released now
+    const aq_status reaped = reap(drv, s, false);
     if (m < m0) {
-        // No kernel may still be reading the planes that are about to lose their memory.
-        if (aq_status e = sync_device(s->dev); e != AQ_OK) return e;
-        const aq_status e = drop_planes(drv, s, aq::round_up((size_t)m * pb, s->gran));
+        // The memory of the dropped planes is released once `stream` has passed this point
+        // (work reading them must be ordered before the call on it); other streams run on.
+        const aq_status e = defer_drop(s, aq::round_up((size_t)m * pb, s->gran), st);
         s->m = m;
-        return e;
+        return e != AQ_OK ? e : reaped;
     }
 
-    if (!src_planes || !src_books || (m0 == 0 && !src_scales)) return AQ_ERR_INVALID_ARG;
     const size_t need = aq::round_up((size_t)m * pb, s->gran);
-    if (need > s->planes_mapped) {
+    // Dropped allocations still waiting for their release lie right where the planes grow:
+    // take them back (their addresses cannot be mapped twice; their contents are rewritten by
+    // the copies below).
+    while (need > s->planes_mapped && !s->pending.empty() &&
+           s->pending.front().mp.addr == planes_base(s) + s->planes_mapped) {
+        s->planes.push_back(s->pending.front().mp);
+        s->planes_mapped += s->pending.front().mp.bytes;
+        cudaEventDestroy(s->pending.front().done);
+        s->pending.erase(s->pending.begin());
+    }
+    // One allocation per plane (its granules not yet mapped), so that lowering later can give
+    // back every plane it drops.
+    for (int k = m0; k < m && need > s->planes_mapped; ++k) {
+        const size_t end = aq::round_up((size_t)(k + 1) * pb, s->gran);
+        if (end <= s->planes_mapped) continue;
         Mapping mp;
         if (aq_status e = map_new(drv, s->dev, planes_base(s) + s->planes_mapped,
-                                  need - s->planes_mapped, &mp);
+                                  end - s->planes_mapped, &mp);
             e != AQ_OK)
             return e;
         s->planes.push_back(mp);
-        s->planes_mapped = need;
+        s->planes_mapped = end;
     }
-    const cudaStream_t st = (cudaStream_t)stream;
     unsigned char* dst = (unsigned char*)s->base;
     const size_t off = (size_t)m0 * pb, n = (size_t)(m - m0) * pb;
     if (n)
@@ -306,8 +377,13 @@ extern "C" void* aq_store_books(const aq_store* s) {
 
 extern "C" void* aq_store_scales(const aq_store* s) { return s ? (void*)s->base : nullptr; }
 
-extern "C" size_t aq_store_device_bytes(const aq_store* s) {
-    return s ? s->head_bytes + s->planes_mapped : 0;
+extern "C" size_t aq_store_device_bytes(aq_store* s) {
+    if (!s) return 0;
+    const Driver* drv = nullptr;
+    if (driver(&drv) == AQ_OK) reap(drv, s, false);
+    size_t held = s->head_bytes + s->planes_mapped;
+    for (const Pending& p : s->pending) held += p.mp.bytes;
+    return held;
 }
 
 extern "C" aq_status aq_store_destroy(aq_store* s) {

@@ -107,7 +107,9 @@ class AQLinear:
     def set_prefix(self, m):
         """Raise or lower the resident prefix of a from_host layer to m (0..M). Raising copies
         planes and codebooks on the current stream, so later work on that stream sees them;
-        lowering synchronises the device and frees the dropped planes' memory."""
+        lowering releases the dropped planes' memory once the work enqueued on the current
+        stream so far has finished (nothing waits for it; work reading the dropped planes must
+        have been enqueued on this stream)."""
         if self.store is None:
             raise TypeError("set_prefix needs a layer made by from_host")
         h = self._host
@@ -116,7 +118,8 @@ class AQLinear:
         self.resident = m
 
     def device_bytes(self):
-        """Device memory held for the layer's weights (scales, codebooks, resident planes)."""
+        """Device memory held for the layer's weights (scales, codebooks, resident planes, and
+        for a from_host layer dropped planes whose release still waits for their stream)."""
         if self.store is not None:
             return aq_store_device_bytes(self.store)
         return sum(t.numel() * t.element_size() for t in (self.planes, self.books, self.scales))

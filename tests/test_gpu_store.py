@@ -8,6 +8,8 @@ store holds must follow the resident prefix in whole 2 MiB granules."""
 import ctypes
 
 import numpy as np
+import time
+
 import pytest
 import torch
 
@@ -71,12 +73,44 @@ def test_device_memory_follows_the_prefix():
         assert head == GRANULE
         for m in (2, 3, 4, 1, 0, 3):
             dyn.set_prefix(m)
+            torch.cuda.current_stream().synchronize()   # a lowering's release follows its stream
             assert dyn.device_bytes() == head + m * pb, m
         with pytest.raises(ValueError):
             dyn.gemv(x_to_device(workloads.make_x(1, 4096, "f16", seed=1), "f16"), 4)
     finally:
         dyn.close()
     assert dyn.resident == 0
+
+
+def test_lowering_does_not_wait_for_other_streams():
+    """Lowering the prefix is ordered on the caller's stream only: a long kernel running on
+    another stream does not hold the call up, and the dropped planes' memory is released once
+    the caller's stream has passed the call. A raise straight after a lowering takes the
+    dropped allocations back, and results stay those of the fully resident layer."""
+    layer, full, host = _setup(CASES[0])
+    pb = aq.plane_bytes(full.layout)
+    dyn = AQLinear.from_host(host, 4)
+    x = x_to_device(workloads.make_x(1, layer["in"], "f16", seed=5), "f16")
+    try:
+        head = dyn.device_bytes() - 4 * pb
+        side = torch.cuda.Stream()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(side):
+            torch.cuda._sleep(400_000_000)          # a few hundred ms of spinning on `side`
+        t0 = time.perf_counter()
+        dyn.set_prefix(2)
+        took = time.perf_counter() - t0
+        still_running = not side.query()
+        assert still_running and took < 0.05, (took, still_running)
+        dyn.set_prefix(3)                           # straight back up: plane 2 is taken back
+        torch.cuda.current_stream().synchronize()
+        assert torch.equal(dyn.gemv(x, 3), full.gemv(x, 3))
+        dyn.set_prefix(1)
+        torch.cuda.current_stream().synchronize()
+        assert dyn.device_bytes() == head + pb
+        side.synchronize()
+    finally:
+        dyn.close()
 
 
 def test_refinement_while_loading():
