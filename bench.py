@@ -58,6 +58,8 @@ def parse():
                          "prints no bench line), with --batch and --m")
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--m", type=int, default=1)
+    ap.add_argument("--bits", type=int, default=0,
+                    help="with --profile-gemv: code width other than the workload's (4, 8, 16)")
     return ap.parse_args()
 
 
@@ -748,6 +750,11 @@ def profile_gemv(args):
     libbuild.build()
     name, _, lname = args.profile_gemv.partition(":")
     (_, layer), = list(workloads.config_layers(name, only=[lname] if lname else None))
+    if args.bits:
+        cfg = workloads.CONFIGS[name]
+        layer = workloads.make_layer(layer["out"], layer["in"], cfg["G"], cfg["M"], args.bits,
+                                     cfg["book_dtype"], cfg["book_std"], cfg["scale_dtype"],
+                                     cfg["seed"])
     lin = AQLinear.from_layer(layer)
     xdt = workloads.CONFIGS[name]["x_dtype"]
     x = x_to_device(workloads.config_x(name, args.batch, layer["in"]), xdt)
