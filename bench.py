@@ -43,6 +43,8 @@ def parse():
     ap.add_argument("--no-gemm", action="store_true")
     ap.add_argument("--no-wmse", action="store_true",
                     help="skip the per-prefix distortion measurement")
+    ap.add_argument("--no-beam", action="store_true",
+                    help="skip the beam-search code update measurement")
     ap.add_argument("--wmse-only", action="store_true",
                     help="only the per-prefix distortion measurement (for profiling)")
     ap.add_argument("--no-loading", action="store_true",
@@ -376,6 +378,56 @@ def measure_wmse(lin, dev, stream, peaks, reps=10):
             "peak_source": "measured" if "bf16_tflops" in peaks else "fallback"}
 
 
+def measure_beam(lin, layer, dev, stream, sm_mhz, K=8, reps=3):
+    """aq_beam_search on the benchmark layer (the code update of Alg. 1, App. C): every group
+    of the 4096 x 4096 layer searches its four codes with a beam of width K = 8. W = the full
+    reconstruction plus N(0, 0.01^2) noise (book type), H = X X^T / n for Gaussian X (fp32),
+    lambda = 1, 1/2, 1/4, 1/8. CUDA events around `reps` back-to-back calls (each: residuals,
+    S, E_k S on the CUDA cores, the search)."""
+    import numpy as np
+    import torch
+    import paper_2606_12876_gb300 as aq
+    out, inp, M, B = lin.out, lin.inp, lin.M, layer["B"]
+    g = torch.Generator(device=dev).manual_seed(9)
+    W = (lin.decode(M).float() + 0.01 * torch.randn(out, inp, device=dev, generator=g)).half()
+    X = torch.randn(inp, 2 * inp, device=dev, generator=g)
+    H = (X @ X.t()) / X.shape[1]
+    del X
+    codes = torch.from_numpy(np.ascontiguousarray(layer["codes"])).to(dev)
+    new = torch.empty_like(codes)
+    books = torch.from_numpy(layer["books"].view(np.int16)).to(dev)
+    scales = torch.from_numpy(layer["scales"].view(np.int16)).to(dev)
+    ws = aq.workspace(aq.beam_workspace_bytes(lin.layout), dev)
+    lam = [1.0 / (1 << k) for k in range(M)]
+    call = lambda: aq.aq_beam_search(lin.layout, W, codes, books, scales, H, aq.AQ_F32, lam, K,
+                                     new, ws, stream=stream)
+    with torch.cuda.stream(stream):
+        call()
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            call()
+        e1.record()
+    torch.cuda.synchronize(dev)
+    ms = e0.elapsed_time(e1) / reps
+    groups = out * (inp // 8)
+    nb = 1 << B
+    cands = nb + (M - 1) * K * nb                      # candidates scored per group
+    # per candidate: d (8 FMA), S_gg d (64 FMA), d.(S_gg d) and d.h (16 FMA), score (2)
+    cand_flops = 2 * (8 + 64 + 16) + 2
+    gemm_flops = 2.0 * M * out * inp * inp             # E_k S for every prefix
+    flops = groups * cands * cand_flops + gemm_flops
+    changed = float((new != codes).any(dim=2).float().mean())
+    peak = fp32_alu_peak_tflops(sm_mhz)
+    tf = flops / (ms * 1e-3) / 1e12
+    return {"workload": "attn_4096", "out": out, "in": inp, "M": M, "B": B, "K": K,
+            "ms": round(ms, 3), "groups_per_s": round(groups / (ms * 1e-3), 1),
+            "candidates_per_group": cands, "flops": flops, "fp32_TFLOP_s": round(tf, 2),
+            "alu_peak_TFLOP_s": round(peak, 1), "frac_alu_peak": round(tf / peak, 4),
+            "groups_changed": round(changed, 4)}
+
+
 def graph_us(calls, n, stream, reps=5):
     """us per call of a CUDA graph of n calls (calls(i) enqueues call i; weight copies rotate
     inside it): median over reps replays, events around the graph only, so back-to-back calls
@@ -690,6 +742,10 @@ def own_arm(args):
         configs = measure_configs(dev, stream, hbm_peak, clk.get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0))
     loading = measure_loading(lin, dev, stream, ms) if rank == 0 and not args.no_loading else None
     wmse = None if args.no_wmse else measure_wmse(lin, dev, stream, peaks)
+    beam = None
+    if rank == 0 and not args.no_beam:
+        beam = measure_beam(lin, layer, dev, stream,
+                            clk.get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0))
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -723,6 +779,7 @@ def own_arm(args):
             "gemm": gemm,
             "dynamic_loading": loading,
             "wmse": wmse,
+            "beam_search": beam,
             "roofline": {
                 "bound": "hbm", "kernel": "gemv_lut_kernel m=%d" % dom["m"],
                 "achieved": dom["GB_s"], "peak": hbm_peak, "unit": "GB/s",

@@ -253,6 +253,44 @@ aq_status aq_wmse(const aq_layout* layout, const void* w, const void* planes, co
                   const void* scales, const void* h, int h_dtype, const double* lambda, double* d,
                   void* workspace, size_t workspace_bytes, void* stream);
 
+/* ---------------------------------------------------------------- code update (beam search)
+ * The code update of Alg. 1 (Sec. 5, "update assignments b using beam search"; App. C calls it
+ * a search for the codeword combinations that minimise the error of the layer's outputs). The
+ * paper gives no further detail; this is the reading implemented: every (row o, group g), with
+ * the row's other groups held at their current codes, chooses its M codes by a beam search of
+ * width K over the books in order k = 0..M-1, minimising the row's Drop-by-Drop objective
+ *     sum_k lambda[k-1] * e^(k) S e^(k)^T,  e^(k) = W[o] - W^(k)[o],  S = (H + H^T)/2
+ * (the trace form of aq_wmse above, restricted to the row). Every group is updated from the
+ * same current codes (a Jacobi step: the groups' new codes are not combined while searching).
+ * With delta_k the group's block of e^(k) and h_k = (S e^(k))_g - S_gg e^(k)_g its cross term
+ * with the rest of the row, the group's terms are delta_k^T S_gg delta_k + 2 delta_k^T h_k;
+ * book t extends each kept state (P = sum of its chosen codewords) by every codeword c of
+ * C_t, scoring the parent's score + lambda[t] * (d^T S_gg d + 2 d^T h_{t+1}) with
+ * d = w_g - s[o] (P + C_t[c]), and the K best extensions are kept, ordered by score, then the
+ * parent's rank, then c. The result is the best state after book M-1. K = 2^(B(M-1)) makes the
+ * search exhaustive (the exact minimiser per group).
+ *   w        : device, [d_out][d_in] of book_dtype (the original weight)
+ *   codes    : device, the current codes, natural layout [d_out][d_in/8][M], uint8 (B = 4 or
+ *              8; B = 16 returns AQ_ERR_UNSUPPORTED: the 2^16-entry books do not fit on chip)
+ *   books, scales : as aq_decode
+ *   h        : device, [d_in][d_in] of h_dtype (AQ_F32 or AQ_BF16), row-major; any square H
+ *   lambda   : HOST, M non-negative doubles (the weight of prefix k at index k-1), or NULL for
+ *              all ones
+ *   beam     : K, 1..16
+ *   codes_out: device, same layout as codes, 16-byte aligned; may be codes (in place: codes
+ *              are read only before any is written)
+ *   workspace: device, aq_beam_workspace_bytes(layout) bytes, 16-byte aligned: a status word,
+ *              S (d_in^2 floats), the residuals E_k and the products E_k S of every prefix
+ *              (2 * M * d_out * d_in floats). No initialisation needed.
+ * Arithmetic: fp32 throughout (residuals, E_k S on the CUDA cores, scores); with inputs whose
+ * sums are exact in fp32 the codes equal the fp64 search's exactly. Stream-ordered; errors:
+ * as aq_gemv. */
+size_t aq_beam_workspace_bytes(const aq_layout* layout);
+aq_status aq_beam_search(const aq_layout* layout, const void* w, const void* codes,
+                         const void* books, const void* scales, const void* h, int h_dtype,
+                         const double* lambda, int beam, void* codes_out, void* workspace,
+                         size_t workspace_bytes, void* stream);
+
 /* ---------------------------------------------------------------- dynamic loading
  * Device storage for one layer that holds only a prefix of its codebooks. One stored model
  * serves every bit width, and each deployment keeps as many codebooks on the device as its

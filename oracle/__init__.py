@@ -250,3 +250,74 @@ def widen(bits, dtype):
     if dtype == "f16":
         return bits.view(np.float16).astype(np.float64)
     return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def beam_update(layer, W, H, lam, K, only=None):
+    """One code update of Alg. 1 ("update assignments b using beam search"; App. C describes
+    it as a search for the codeword combinations that minimise the error of the layer's
+    outputs), in this reading: for every row o and group g, with the codes of the row's other
+    groups held at their current values, the group's M codes are chosen by a beam search of
+    width K over the books in order 0..M-1 that minimises the Drop-by-Drop objective of Sec. 5
+    restricted to the row, sum_k lam[k-1] * e^(k) S e^(k)^T with e^(k) = W[o] - W^(k)[o] and
+    S = (H + H^T)/2 (only the symmetric part of H enters a trace form). Every group is updated
+    from the same current codes. Changing group g moves only its block of e^(k), by
+    delta_k = w_g - s_o * (sum_{j<k} C_j[b_j]), so the terms that depend on the group's codes
+    are delta_k^T S_gg delta_k + 2 delta_k^T h_k with h_k the cross term of the block with the
+    rest of the row, h_k = (S e^(k))_g - S_gg e^(k)_g.
+
+    Beam: states (codes chosen so far, their codeword sum P, score); from the single empty
+    state, book t extends every state by every codeword c of C_t, scoring
+    score + lam[t] * (d^T S_gg d + 2 d^T h_{t+1}) with d = w_g - s_o (P + C_t[c]); the K best
+    extensions are kept, ordered by (score, rank of the parent state, c). The result is the
+    first state after book M-1. Scores in fp64.
+
+    W: [out][in] float64, H: [in][in] float64, lam: M weights, K >= 1. only: optional
+    iterable of (o, g) pairs; the other groups keep their codes. Returns new codes with the
+    shape and dtype of layer["codes"]."""
+    out, inp, G, M, B = layer["out"], layer["in"], layer["G"], layer["M"], layer["B"]
+    codes = np.asarray(layer["codes"])
+    books = widen(layer["books"], layer["book_dtype"]).reshape(M, 1 << B, G)
+    s = widen(layer["scales"], layer["scale_dtype"])
+    W = np.asarray(W, dtype=np.float64)
+    H = np.asarray(H, dtype=np.float64)
+    S = (H + H.T) / 2
+    lam = np.asarray(lam, dtype=np.float64)
+    E = [W - reconstruct_exact(layer, k) for k in range(1, M + 1)]   # e^(k), k = 1..M
+    V = [e @ S for e in E]                                          # rows of S e^(k)
+    new = codes.copy()
+    nb = 1 << B
+    pairs = [(o, g) for o in range(out) for g in range(inp // G)] if only is None else only
+    for o, g in pairs:
+        blk = slice(g * G, (g + 1) * G)
+        Sgg = S[blk, blk]
+        wg = W[o, blk]
+        h = [V[k][o, blk] - Sgg @ E[k][o, blk] for k in range(M)]
+        states = [((), np.zeros(G), 0.0)]
+        for t in range(M):
+            score, rank, cw = [], [], []
+            for r, (cs, P, sc) in enumerate(states):
+                D = wg - s[o] * (P + books[t])          # row c: d for codeword c of C_t
+                q = np.einsum("ce,ef,cf->c", D, Sgg, D)
+                score.append(sc + lam[t] * (q + 2.0 * (D @ h[t])))
+                rank.append(np.full(nb, r))
+                cw.append(np.arange(nb))
+            score, rank, cw = np.concatenate(score), np.concatenate(rank), np.concatenate(cw)
+            keep = np.lexsort((cw, rank, score))[:K]    # by score, then parent rank, then c
+            states = [(states[rank[i]][0] + (int(cw[i]),), states[rank[i]][1] + books[t, cw[i]],
+                       float(score[i])) for i in keep]
+        new[o, g, :] = states[0][0]
+    return new
+
+
+def row_objective(layer, W, H, lam, o):
+    """sum_k lam[k-1] * e^(k) S e^(k)^T for row o (S = (H + H^T)/2, e^(k) = W[o] - W^(k)[o],
+    exact reconstruction): the quantity the code update minimises, evaluated directly."""
+    M = layer["M"]
+    W = np.asarray(W, dtype=np.float64)
+    H = np.asarray(H, dtype=np.float64)
+    S = (H + H.T) / 2
+    tot = 0.0
+    for k in range(1, M + 1):
+        e = W[o] - reconstruct_exact(layer, k)[o]
+        tot += lam[k - 1] * float(e @ S @ e)
+    return tot

@@ -27,7 +27,8 @@ EXPORTS = ["aq_abi_version", "aq_status_string", "aq_last_error", "aq_plane_byte
            "aq_gemv_static_scratch_status",
            "aq_gemv_refine", "aq_store_create", "aq_store_set_prefix", "aq_store_prefix",
            "aq_store_planes", "aq_store_books", "aq_store_scales", "aq_store_device_bytes",
-           "aq_store_destroy", "aq_wmse_workspace_bytes", "aq_wmse", "aq_selftest_wait"]
+           "aq_store_destroy", "aq_wmse_workspace_bytes", "aq_wmse", "aq_beam_workspace_bytes",
+           "aq_beam_search", "aq_selftest_wait"]
 
 
 class AQError(RuntimeError):
@@ -90,6 +91,9 @@ def lib():
             "aq_store_device_bytes": (sz, [vp]),
             "aq_store_destroy": (i32, [vp]),
             "aq_wmse_workspace_bytes": (sz, [lp]),
+            "aq_beam_workspace_bytes": (sz, [lp]),
+            "aq_beam_search": (i32, [lp, vp, vp, vp, vp, vp, i32, ctypes.POINTER(ctypes.c_double),
+                                     i32, vp, vp, sz, vp]),
             "aq_selftest_wait": (i32, [vp, sz, vp]),
             "aq_wmse": (i32, [lp, vp, vp, vp, vp, vp, i32, ctypes.POINTER(ctypes.c_double), vp,
                               vp, sz, vp]),
@@ -260,6 +264,26 @@ def aq_wmse(layout, w, planes, books, scales, h, h_dtype, lam, d, workspace,
     _check(lib().aq_wmse(ctypes.byref(layout), _ptr(w), _ptr(planes), _ptr(books), _ptr(scales),
                          _ptr(h), h_dtype, lam_arr, _ptr(d), _ptr(workspace), workspace_bytes,
                          _stream(stream)), "aq_wmse")
+
+
+def beam_workspace_bytes(layout):
+    return lib().aq_beam_workspace_bytes(ctypes.byref(layout))
+
+
+def aq_beam_search(layout, w, codes, books, scales, h, h_dtype, lam, beam, codes_out, workspace,
+                   workspace_bytes=None, stream=None):
+    """New codes [d_out][d_in/8][M] (into codes_out) from a beam search of width `beam` per
+    group over the books, minimising sum_k lam[k-1] e^(k) S e^(k)^T of the group's row with the
+    other groups at their current codes (lam: M host floats, or None for all ones)."""
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    lam_arr = None
+    if lam is not None:
+        lam_arr = (ctypes.c_double * len(lam))(*[float(v) for v in lam])
+    _check(lib().aq_beam_search(ctypes.byref(layout), _ptr(w), _ptr(codes), _ptr(books),
+                                _ptr(scales), _ptr(h), h_dtype, lam_arr, int(beam),
+                                _ptr(codes_out), _ptr(workspace), workspace_bytes,
+                                _stream(stream)), "aq_beam_search")
 
 
 def aq_workspace_init(workspace, nbytes=None, stream=None):

@@ -240,6 +240,33 @@ aq_status aq_wmse(const aq_layout* layout, const void* w, const void* planes, co
                            as_stream(stream));
 }
 
+size_t aq_beam_workspace_bytes(const aq_layout* layout) {
+    Dims d;
+    if (aq::make_dims(layout, &d) != AQ_OK) return 0;
+    return aq::beam_ws_bytes(d);
+}
+
+aq_status aq_beam_search(const aq_layout* layout, const void* w, const void* codes,
+                         const void* books, const void* scales, const void* h, int h_dtype,
+                         const double* lambda, int beam, void* codes_out, void* workspace,
+                         size_t workspace_bytes, void* stream) {
+    Dims d;
+    aq_status st = aq::make_dims(layout, &d);
+    if (st != AQ_OK) return st;
+    if (d.B == 16) return AQ_ERR_UNSUPPORTED;          // 2^16-entry books do not fit on chip
+    if (h_dtype != AQ_F32 && h_dtype != AQ_BF16) return AQ_ERR_INVALID_ARG;
+    if (beam < 1 || beam > 16) return AQ_ERR_INVALID_ARG;
+    if (lambda)
+        for (int k = 0; k < d.M; ++k)
+            if (!(lambda[k] >= 0.0)) return AQ_ERR_INVALID_ARG;
+    if (d.out == 0) return AQ_OK;
+    if ((st = check_ptrs({w, codes, books, scales, h, codes_out})) != AQ_OK) return st;
+    if (!workspace || workspace_bytes < aq::beam_ws_bytes(d)) return AQ_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;
+    return aq::launch_beam(d, w, codes, books, scales, h, h_dtype, lambda, beam, codes_out,
+                           workspace, as_stream(stream));
+}
+
 size_t aq_gemm_workspace_bytes(const aq_layout* layout, int tokens) {
     Dims d;
     if (aq::make_dims(layout, &d) != AQ_OK || tokens < 0) return 0;

@@ -94,6 +94,12 @@ aq_status launch_gemm(const Dims& d, int m, const void* planes, const void* book
                       void* ws, cudaStream_t st);
 // aq_selftest_wait: one bounded wait that nothing completes (records AQ_ERR_TIMEOUT).
 aq_status launch_selftest_wait(unsigned int* status, cudaStream_t st);
+// Beam-search code update (aq_beam_search): workspace bytes, and the launch (validated
+// arguments; codes natural [out][in/8][M], uint8 for B <= 8).
+size_t beam_ws_bytes(const Dims& d);
+aq_status launch_beam(const Dims& d, const void* w, const void* codes, const void* books,
+                      const void* scales, const void* h, int h_dt, const double* lambda, int K,
+                      void* codes_out, void* ws, cudaStream_t st);
 // Per-prefix distortion (aq_wmse): workspace bytes, and the launch (validated arguments).
 size_t wmse_ws_bytes(const Dims& d);
 aq_status launch_wmse(const Dims& d, const void* w, const void* planes, const void* books,

@@ -379,6 +379,59 @@ def pin_wmse_abs_equals_wmse_for_nonnegative_terms():
     assert np.all(np.abs(D2) <= A2 * (1 + 1e-12)) and np.any(np.abs(D2) < 0.9 * A2), (D2, A2)
 
 
+def _beam_case(out, inp, M, B, seed):
+    layer = workloads.make_layer(out, inp, G=8, M=M, B=B, book_std=0.3, seed=seed)
+    rng = _rng(seed + 1)
+    W = _onehot_reconstruction(layer, M) + 0.1 * rng.standard_normal((out, inp))
+    X = rng.standard_normal((inp, 3 * inp))
+    H = X @ X.T / X.shape[1] + 0.2 * rng.standard_normal((inp, inp))   # not symmetric
+    return layer, W, H
+
+
+def pin_beam_exhaustive_matches_bruteforce():
+    """A beam wide enough to keep every partial state (K = (2^B)^(M-1)) returns, for every
+    group, the code combination that minimises the row's Drop-by-Drop objective with the row's
+    other groups held fixed; the objective is evaluated directly (full-row trace form, exact
+    reconstruction) for all (2^B)^M combinations. Two weight matrices: one near a codeword
+    combination, and one far from every combination, where a one-state (greedy) search picks a
+    worse combination for some groups, so that the width of the beam is pinned too."""
+    layer, W, H = _beam_case(6, 16, 2, 4, seed=41)
+    W_far = _rng(45).standard_normal(W.shape) * 0.6
+    lam = np.array([0.7, 0.3])
+    greedy_differs = False
+    for Wt in (W, W_far):
+        got = oracle.beam_update(layer, Wt, H, lam, 16)
+        greedy = oracle.beam_update(layer, Wt, H, lam, 1)
+        for o in range(6):
+            for g in range(2):
+                best, arg = None, None
+                for c0 in range(16):
+                    for c1 in range(16):
+                        trial = dict(layer)
+                        trial["codes"] = layer["codes"].copy()
+                        trial["codes"][o, g] = (c0, c1)
+                        f = oracle.row_objective(trial, Wt, H, lam, o)
+                        if best is None or f < best - 1e-12:
+                            best, arg = f, (c0, c1)
+                assert tuple(got[o, g]) == arg, (o, g, tuple(got[o, g]), arg)
+                greedy_differs |= tuple(greedy[o, g]) != arg
+    assert greedy_differs, "the case does not tell a beam from a greedy search"
+
+
+def pin_beam_single_book_nearest_codeword():
+    """One book, H = I, lambda = 1: the update is the nearest scaled codeword of each group,
+    argmin_c ||w_g - s_o C[c]||^2, for any beam width."""
+    layer, W, _ = _beam_case(4, 24, 1, 8, seed=43)
+    books = workloads_values(layer["books"], "f16").reshape(256, 8)
+    s = workloads_values(layer["scales"], "f16")
+    for K in (1, 3):
+        got = oracle.beam_update(layer, W, np.eye(24), [1.0], K)
+        for o in range(4):
+            for g in range(3):
+                d = W[o, g * 8:(g + 1) * 8] - s[o] * books
+                assert got[o, g, 0] == int(np.argmin(np.sum(d * d, axis=1))), (K, o, g)
+
+
 def pin_wmse_vanishes_at_the_exact_weight():
     """W = W^(M): the full prefix has zero distortion; a shorter prefix leaves the dropped
     codebooks' contribution, which is positive for a positive definite H."""

@@ -165,6 +165,33 @@ def test_wmse_sizes_and_argument_errors_on_the_host():
     assert call(_lay(), ws=FAKE + 8) == aq.AQ_ERR_ALIGNMENT
 
 
+def test_beam_sizes_and_argument_errors_on_the_host():
+    L = aq.Layout.make(4096, 4096, 4)
+    # status block, S in fp32, then E_k and E_k S of the four prefixes in fp32
+    assert aq.beam_workspace_bytes(L) == 256 + 4096 * 4096 * 4 + 2 * 4 * 4096 * 4096 * 4
+    lib = aq.lib()
+
+    def call(L, hdt=aq.AQ_F32, lam=None, K=4, out=FAKE, ws=FAKE, wsb=None):
+        lam_arr = None if lam is None else (ctypes.c_double * len(lam))(*lam)
+        return lib.aq_beam_search(
+            ctypes.byref(L) if L is not None else None, FAKE, FAKE, FAKE, FAKE, FAKE, hdt,
+            lam_arr, K, out, ws,
+            aq.beam_workspace_bytes(L) if wsb is None and L is not None else (wsb or 0), None)
+    assert call(None, wsb=0) == aq.AQ_ERR_INVALID_ARG
+    assert call(_lay(), hdt=aq.AQ_F16) == aq.AQ_ERR_INVALID_ARG
+    assert call(_lay(), K=0) == aq.AQ_ERR_INVALID_ARG
+    assert call(_lay(), K=17) == aq.AQ_ERR_INVALID_ARG
+    assert call(_lay(), lam=[1.0, -0.5, 1.0, 1.0]) == aq.AQ_ERR_INVALID_ARG
+    assert call(_lay(), lam=[1.0, float("nan"), 1.0, 1.0]) == aq.AQ_ERR_INVALID_ARG
+    assert call(_lay(B=16)) == aq.AQ_ERR_UNSUPPORTED
+    assert call(_lay(), out=None) == aq.AQ_ERR_INVALID_ARG
+    assert call(_lay(), out=FAKE + 1) == aq.AQ_ERR_ALIGNMENT
+    assert call(_lay(), ws=None) == aq.AQ_ERR_WORKSPACE
+    assert call(_lay(), wsb=aq.beam_workspace_bytes(_lay()) - 4) == aq.AQ_ERR_WORKSPACE
+    assert call(_lay(), ws=FAKE + 8) == aq.AQ_ERR_ALIGNMENT
+    assert call(_lay(out=0), ws=None) == aq.AQ_OK      # nothing to update
+
+
 def _x16(tokens):
     """Offset of the fp16 activation copy: status block, then one float per token."""
     return 256 + (tokens * 4 + 255) // 256 * 256

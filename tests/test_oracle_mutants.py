@@ -48,6 +48,14 @@ PY_MUTANTS = [
     ("wmse_abs_keeps_sign_of_H", "A = np.abs(np.asarray(H, dtype=np.float64))",
      "A = np.asarray(H, dtype=np.float64)"),
     ("wmse_abs_drops_normalisation", "np.sum((E @ A) * E)) / out", "np.sum((E @ A) * E))"),
+    ("beam_drops_cross_term", "h = [V[k][o, blk] - Sgg @ E[k][o, blk] for k in range(M)]",
+     "h = [0.0 * V[k][o, blk] for k in range(M)]"),
+    ("beam_uses_unsymmetrised_H", "    S = (H + H.T) / 2\n    lam = np.asarray(lam, dtype=np.float64)\n    E = [W - reconstruct_exact",
+     "    S = H\n    lam = np.asarray(lam, dtype=np.float64)\n    E = [W - reconstruct_exact"),
+    ("beam_weights_shifted", "score.append(sc + lam[t] * (q", "score.append(sc + lam[M - 1 - t] * (q"),
+    ("beam_scale_dropped", "D = wg - s[o] * (P + books[t])", "D = wg - (P + books[t])"),
+    ("beam_keeps_one_state", "keep = np.lexsort((cw, rank, score))[:K]",
+     "keep = np.lexsort((cw, rank, score))[:1]"),
     ("wmse_abs_prefix_off_by_one", "E = np.abs(np.asarray(W, dtype=np.float64) - reconstruct_exact(layer, k))",
      "E = np.abs(np.asarray(W, dtype=np.float64) - reconstruct_exact(layer, max(1, k - 1)))"),
 ]
