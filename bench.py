@@ -482,6 +482,7 @@ def measure_configs(dev, stream, hbm_peak, sm_mhz):
         x = x_to_device(workloads.make_x(batch, lin.inp, xdt, seed=batch), xdt)
         y = torch.empty(batch, lin.out, dtype=x.dtype, device=dev)
         ws = aq.workspace(aq.gemv_workspace_bytes(lin.layout, batch), dev)
+        sink = torch.zeros(4, dtype=torch.int32, device=dev)
         nc = max(2, -(-3 * l2 // lin.planes.numel()))
         copies = [lin.planes.clone() for _ in range(nc)]
         rows = []
@@ -492,6 +493,14 @@ def measure_configs(dev, stream, hbm_peak, sm_mhz):
             nb = layer_bytes(lin.out, lin.inp, m, B=lin.B, batch=batch)
             e = {"m": m, "bits_per_weight": m * lin.B // 8, "us": round(us, 3),
                  "GB_s": round(nb / us / 1e3, 1), "frac_hbm": round(nb / us / 1e3 / hbm_peak, 4)}
+            if batch == 1:
+                # the read probe over the same code bytes: the per-call floor of this size
+                pb = aq.packed_bytes(lin.layout, m)
+                with torch.cuda.stream(stream):
+                    fl = graph_us(lambda i, pb=pb: aq.aq_selftest_read(copies[i % nc], pb, sink),
+                                  20, stream)
+                e["read_floor_us"] = round(fl, 3)
+                e["frac_of_read_floor"] = round(fl / us, 4)
             if batch > 1:
                 tf = 2.0 * batch * lin.out * lin.inp / (us * 1e-6) / 1e12
                 e["TFLOP_s"] = round(tf, 2)
@@ -519,6 +528,7 @@ def measure_configs(dev, stream, hbm_peak, sm_mhz):
         ys = [torch.empty(b, lin.out, dtype=torch.bfloat16, device=dev) for _, lin in blk]
         wss = [aq.workspace(aq.gemv_workspace_bytes(lin.layout, b), dev) for _, lin in blk]
         cps = [[lin.planes.clone() for _ in range(3)] for _, lin in blk]
+        sink = torch.zeros(4, dtype=torch.int32, device=dev)
         rows = []
         for m in (1, 2, 3, 4):
             def step(i, m=m):
@@ -530,6 +540,14 @@ def measure_configs(dev, stream, hbm_peak, sm_mhz):
             nb = sum(layer_bytes(lin.out, lin.inp, m, batch=b) for _, lin in blk)
             e = {"m": m, "us": round(us, 3), "GB_s": round(nb / us / 1e3, 1),
                  "frac_hbm": round(nb / us / 1e3 / hbm_peak, 4)}
+            if b == 1:
+                def floor_step(i, m=m):
+                    for j, (_, lin) in enumerate(blk):
+                        aq.aq_selftest_read(cps[j][i % 3], aq.packed_bytes(lin.layout, m), sink)
+                with torch.cuda.stream(stream):
+                    fl = graph_us(floor_step, 10, stream)
+                e["read_floor_us"] = round(fl, 3)
+                e["frac_of_read_floor"] = round(fl / us, 4)
             if b > 1:
                 tf = 2.0 * b * sum(lin.out * lin.inp for _, lin in blk) / (us * 1e-6) / 1e12
                 e["TFLOP_s"] = round(tf, 2)
@@ -682,6 +700,17 @@ def own_arm(args):
         single_us[m] = statistics.median(lat)
 
 
+    # Read floor: the read probe (aq_selftest_read, the GEMV's launch shape doing nothing but
+    # reading) over the same m planes of the same rotating copies; same graph timing.
+    sink = torch.zeros(4, dtype=torch.int32, device=dev)
+    floor_us = {}
+    for m in ms:
+        nb = aq.packed_bytes(L, m)
+        g = capture(lambda i, nb=nb: aq.aq_selftest_read(copies[i % ncopies], nb, sink), glen)
+        g.replay()
+        floor_us[m] = statistics.median(time_graph(g) for _ in range(5)) * 1e3 / glen
+        del g
+
     # Refinement step (aq_gemv_refine): the increment from prefix m-1 to m, reading plane m-1
     # only, fp32 output added to the previous fp32 result; same graph timing.
     ys32 = {m: torch.zeros(1, out, dtype=torch.float32, device=dev) for m in (0,) + ms}
@@ -704,6 +733,8 @@ def own_arm(args):
                       "frac_hbm": round(gbs / hbm_peak, 4),
                       "frac_hbm_spec_8TBs": round(gbs / 8000.0, 4),
                       "single_call_us": round(single_us[m], 3), "bytes": bytes_m[m],
+                      "read_floor_us": round(floor_us[m], 3),
+                      "frac_of_read_floor": round(floor_us[m] / us, 4),
                       "refine_from_m_minus_1_us": round(refine_us[m], 3),
                       "refine_GB_s": round(refine_bytes / (refine_us[m] * 1e-6) / 1e9, 1)})
     dom = per_m[-1]       # the full prefix: the most bytes per call

@@ -369,6 +369,17 @@ aq_status aq_store_destroy(aq_store* store);
  * aq_workspace_status: SYNCHRONISES stream, then returns the device-side status a kernel
  * recorded in the workspace (AQ_OK if none) and clears it. */
 aq_status aq_selftest_wait(void* workspace, size_t workspace_bytes, void* stream);
+
+/* aq_selftest_read: a read probe for measurement (no counterpart in the paper). Enqueues one
+ * kernel with the launch shape of the one-token GEMV (one CTA per SM, programmatic dependent
+ * launch, the source requested before waiting for the preceding kernel) that only reads:
+ * the XOR of all 32-bit words of src[0, bytes) is XORed into *sink. Timed back to back, it
+ * gives the per-call cost of reading the same bytes with nothing computed, the floor that a
+ * GEMV call of the same size is compared with.
+ *   src   : device, 16-byte aligned, bytes a multiple of 16 (read only)
+ *   sink  : device, one 32-bit word, 4-byte aligned (the caller zeroes it to check the fold)
+ * Errors: AQ_ERR_INVALID_ARG (sink NULL, or src NULL with bytes > 0), AQ_ERR_ALIGNMENT. */
+aq_status aq_selftest_read(const void* src, size_t bytes, void* sink, void* stream);
 aq_status aq_workspace_init(void* workspace, size_t bytes, void* stream);
 aq_status aq_workspace_status(void* workspace, void* stream);
 

@@ -28,7 +28,7 @@ EXPORTS = ["aq_abi_version", "aq_status_string", "aq_last_error", "aq_plane_byte
            "aq_gemv_refine", "aq_store_create", "aq_store_set_prefix", "aq_store_prefix",
            "aq_store_planes", "aq_store_books", "aq_store_scales", "aq_store_device_bytes",
            "aq_store_destroy", "aq_wmse_workspace_bytes", "aq_wmse", "aq_beam_workspace_bytes",
-           "aq_beam_search", "aq_selftest_wait"]
+           "aq_beam_search", "aq_selftest_wait", "aq_selftest_read"]
 
 
 class AQError(RuntimeError):
@@ -95,6 +95,7 @@ def lib():
             "aq_beam_search": (i32, [lp, vp, vp, vp, vp, vp, i32, ctypes.POINTER(ctypes.c_double),
                                      i32, vp, vp, sz, vp]),
             "aq_selftest_wait": (i32, [vp, sz, vp]),
+            "aq_selftest_read": (i32, [vp, sz, vp, vp]),
             "aq_wmse": (i32, [lp, vp, vp, vp, vp, vp, i32, ctypes.POINTER(ctypes.c_double), vp,
                               vp, sz, vp]),
         }
@@ -290,6 +291,12 @@ def aq_workspace_init(workspace, nbytes=None, stream=None):
     if nbytes is None:
         nbytes = workspace.numel() * workspace.element_size()
     _check(lib().aq_workspace_init(_ptr(workspace), nbytes, _stream(stream)), "aq_workspace_init")
+
+
+def aq_selftest_read(src, nbytes, sink, stream=None):
+    """Read probe: XOR of the 32-bit words of the first nbytes of src folded into sink[0]."""
+    _check(lib().aq_selftest_read(_ptr(src), nbytes, _ptr(sink), _stream(stream)),
+           "aq_selftest_read")
 
 
 def aq_workspace_status(workspace, stream=None):

@@ -298,6 +298,12 @@ aq_status aq_selftest_wait(void* workspace, size_t workspace_bytes, void* stream
     return aq::launch_selftest_wait((unsigned int*)workspace, as_stream(stream));
 }
 
+aq_status aq_selftest_read(const void* src, size_t bytes, void* sink, void* stream) {
+    if (!sink || (!src && bytes > 0)) return AQ_ERR_INVALID_ARG;
+    if (!aligned16(src) || ((uintptr_t)sink & 3u) || bytes % 16) return AQ_ERR_ALIGNMENT;
+    return aq::launch_selftest_read(src, bytes, (unsigned int*)sink, as_stream(stream));
+}
+
 aq_status aq_workspace_init(void* workspace, size_t bytes, void* stream) {
     if (!workspace) return AQ_ERR_INVALID_ARG;
     if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;

@@ -94,6 +94,8 @@ aq_status launch_gemm(const Dims& d, int m, const void* planes, const void* book
                       void* ws, cudaStream_t st);
 // aq_selftest_wait: one bounded wait that nothing completes (records AQ_ERR_TIMEOUT).
 aq_status launch_selftest_wait(unsigned int* status, cudaStream_t st);
+// Read probe (aq_selftest_read): reads bytes at src with the GEMV's launch shape.
+aq_status launch_selftest_read(const void* src, size_t bytes, unsigned int* sink, cudaStream_t st);
 // Beam-search code update (aq_beam_search): workspace bytes, and the launch (validated
 // arguments; codes natural [out][in/8][M], uint8 for B <= 8).
 size_t beam_ws_bytes(const Dims& d);

@@ -182,11 +182,12 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
     };
     if (static_weights) {
         // The weights are read-only while calls run (AQ_LAYOUT_STATIC_WEIGHTS): request the
-        // codebooks and fill the code ring before waiting for the preceding kernel, so they
-        // overlap its tail.
+        // codebooks and the first code stage before waiting for the preceding kernel, so they
+        // overlap its tail. Only one stage: the activations are requested right after the
+        // wait and queue behind whatever code copies are still in flight (measured on the
+        // 14336 x 4096 layer: one stage 4-7 % faster per call than a full ring).
         load_books();
-        if (warp == kCons && lane == 0)
-            while (p_q < nslots && p_w.it < i1) issue_next();
+        if (warp == kCons && lane == 0 && p_w.it < i1) issue_next();
     }
     pdl_wait();                 // inputs may come from the preceding kernel in the stream
     pdl_launch_dependents();    // the split-K reduction may become resident (it waits for us)

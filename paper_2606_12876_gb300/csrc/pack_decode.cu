@@ -162,6 +162,88 @@ aq_status launch_selftest_wait(unsigned int* status, cudaStream_t st) {
     return cuda_ok(cudaGetLastError(), "kernel launch");
 }
 
+namespace {
+
+// Read probe: the launch shape of the one-token GEMV (one CTA per SM, sixteen warps,
+// programmatic dependent launch, source requested before the grid wait) doing nothing but
+// reading. CTA b takes 1 KiB chunks [c0, c1); warp w takes chunks c0 + w, c0 + w + 16, ...,
+// four in flight; lane L reads bytes 16 L and 512 + 16 L of a chunk (each load instruction
+// covers 512 contiguous bytes). The 32-bit words are XOR-folded, and each CTA XORs its fold
+// into *sink once. A tail of bytes % 1024 is read by CTA 0, 16 bytes per thread.
+constexpr int kReadWarps = 16, kReadDepth = 4;
+
+__global__ void __launch_bounds__(kReadWarps * 32, 1)
+selftest_read_kernel(const uint8_t* __restrict__ src, size_t chunks, size_t tail, int q, int r,
+                     unsigned int* sink) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, b = blockIdx.x;
+    const size_t c0 = (size_t)b * q + min(b, r), c1 = c0 + q + (b < r ? 1 : 0);
+    uint4 v[kReadDepth][2];
+    size_t c = c0 + warp;
+#pragma unroll
+    for (int d = 0; d < kReadDepth; ++d) {
+        const size_t cd = c + (size_t)d * kReadWarps;
+        v[d][0] = v[d][1] = make_uint4(0u, 0u, 0u, 0u);
+        if (cd < c1) {
+            v[d][0] = ld_stream_v4(src + cd * 1024 + lane * 16);
+            v[d][1] = ld_stream_v4(src + cd * 1024 + 512 + lane * 16);
+        }
+    }
+    pdl_wait();
+    pdl_launch_dependents();
+    uint32_t acc = 0;
+    for (; c < c1; c += (size_t)kReadDepth * kReadWarps) {
+#pragma unroll
+        for (int d = 0; d < kReadDepth; ++d) {
+            acc ^= v[d][0].x ^ v[d][0].y ^ v[d][0].z ^ v[d][0].w ^ v[d][1].x ^ v[d][1].y ^
+                   v[d][1].z ^ v[d][1].w;
+            v[d][0] = v[d][1] = make_uint4(0u, 0u, 0u, 0u);
+            const size_t cn = c + (size_t)(d + kReadDepth) * kReadWarps;
+            if (cn < c1) {
+                v[d][0] = ld_stream_v4(src + cn * 1024 + lane * 16);
+                v[d][1] = ld_stream_v4(src + cn * 1024 + 512 + lane * 16);
+            }
+        }
+    }
+    if (b == 0)
+        for (size_t i = (size_t)threadIdx.x * 16; i < tail; i += (size_t)kReadWarps * 32 * 16) {
+            const uint4 t = ld_stream_v4(src + chunks * 1024 + i);
+            acc ^= t.x ^ t.y ^ t.z ^ t.w;
+        }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc ^= __shfl_xor_sync(0xffffffffu, acc, o);
+    __shared__ uint32_t red[kReadWarps];
+    if (lane == 0) red[warp] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint32_t f = 0;
+        for (int w = 0; w < kReadWarps; ++w) f ^= red[w];
+        atomicXor(sink, f);
+    }
+}
+
+}  // namespace
+
+aq_status launch_selftest_read(const void* src, size_t bytes, unsigned int* sink, cudaStream_t st) {
+    DeviceInfo di;
+    if (aq_status e = device_info(&di); e != AQ_OK) return e;
+    const size_t chunks = bytes / 1024, tail = bytes % 1024;
+    const size_t grid = chunks < (size_t)di.sms ? (chunks > 0 ? chunks : 1) : (size_t)di.sms;
+    const int q = (int)(chunks / grid), r = (int)(chunks % grid);
+    if (chunks / grid > 0x7fffffffULL) return AQ_ERR_UNSUPPORTED;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kReadWarps * 32);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cuda_ok(cudaLaunchKernelEx(&cfg, selftest_read_kernel, (const uint8_t*)src, chunks, tail,
+                                      q, r, sink),
+                   "cudaLaunchKernelEx");
+}
+
 aq_status launch_pack(const Dims& d, const void* codes, void* planes, cudaStream_t st) {
     const size_t total = (size_t)d.M * d.plane_elems;
     if (total == 0) return AQ_OK;

@@ -221,3 +221,12 @@ def test_selftest_wait_argument_errors_on_the_host():
     assert lib.aq_selftest_wait(None, 256, None) == aq.AQ_ERR_INVALID_ARG
     assert lib.aq_selftest_wait(FAKE, 16, None) == aq.AQ_ERR_WORKSPACE
     assert lib.aq_selftest_wait(FAKE + 8, 256, None) == aq.AQ_ERR_ALIGNMENT
+
+
+def test_selftest_read_argument_errors_on_the_host():
+    lib = aq.lib()
+    assert lib.aq_selftest_read(FAKE, 1024, None, None) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_selftest_read(None, 1024, FAKE, None) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_selftest_read(FAKE + 8, 1024, FAKE, None) == aq.AQ_ERR_ALIGNMENT
+    assert lib.aq_selftest_read(FAKE, 1000, FAKE, None) == aq.AQ_ERR_ALIGNMENT
+    assert lib.aq_selftest_read(FAKE, 1024, FAKE + 2, None) == aq.AQ_ERR_ALIGNMENT
