@@ -184,7 +184,7 @@ aq_status aq_gemv_refine(const aq_layout* layout, int m, const void* planes, con
  *   - Every call on a device shares the one buffer, which keeps the last call's contents:
  *     calls that may overlap on the GPU (other streams, other host threads) race on it and
  *     must be ordered by the caller. */
-#define AQ_STATIC_SCRATCH_BYTES ((size_t)4 << 20)
+#define AQ_STATIC_SCRATCH_BYTES ((size_t)16 << 20)
 aq_status aq_gemv_static_scratch(const aq_layout* layout, int m, const void* planes,
                                  const void* books, const void* scales, const void* x,
                                  int x_dtype, int batch, void* y, int y_dtype, void* stream);

@@ -42,11 +42,19 @@ inline size_t ws_partial_offset(const Dims&) { return kWsStatusBytes; }
 
 // The table-lookup GEMV (2^8-entry books; batch 1 and 2 with prefixes up to kLutMaxM, batch
 // 3..4 with prefixes up to kLutMultiM: their two 64 KiB tables and five or more codebooks
-// leave room for a single code stage) writes one partial plane per (slice, book, token); every
-// other GEMV one per (slice, token).
-constexpr int kLutMaxM = 8, kLutMultiM = 4;
-inline int lut_max_m(int batch) { return batch <= 2 ? kLutMaxM : batch <= 4 ? kLutMultiM : 0; }
-inline bool uses_lut(const Dims& d, int m, int batch) { return d.B == 8 && m <= lut_max_m(batch); }
+// leave room for a single code stage; batch 5..8 with prefixes up to kLut8M and fp16 tables,
+// when the layer has at least kLut8MinItems (slice, book, 32-row block) items, about 30 per SM:
+// below that an eight-token table build costs more than the tensor-core kernel's decode)
+// writes one partial plane per (slice, book, token); every other GEMV one per (slice, token).
+constexpr int kLutMaxM = 8, kLutMultiM = 4, kLut8M = 6;
+constexpr long long kLut8MinItems = 4560;
+inline int lut_max_m(int batch) {
+    return batch <= 2 ? kLutMaxM : batch <= 4 ? kLutMultiM : batch <= 8 ? kLut8M : 0;
+}
+inline bool uses_lut(const Dims& d, int m, int batch) {
+    if (d.B != 8 || m > lut_max_m(batch)) return false;
+    return batch <= 4 || (long long)d.S * m * d.RBc >= kLut8MinItems;
+}
 
 // Prefill GEMM workspace: [status block, 256 B: status word at 0, the dense form's weight
 // factor (float) at kWsWfacOffset][per-token activation factors, float][fp16 copy of bf16

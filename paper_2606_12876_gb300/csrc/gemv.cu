@@ -409,6 +409,327 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
     }
 }
 
+// ------------------------------------------------------------------ 8-token LUT kernel (B = 8)
+//
+// gemv_lut8 (a pass of up to 8 tokens, B = 8, m <= kLut8MaxM; 9..16 tokens take two passes):
+// the table form for several tokens with fp16 table entries. The table of a (slice s, book k)
+// unit holds, for every codeword j and group g, the eight tokens' products x_t,g . C_k[j],
+// four tokens to an 8-byte entry: sub-table h (tokens 4h..4h+3) at byte h*65536 + j*256 + 8g.
+// A code byte then costs one prmt (offset j*256 + 8g), two 8-byte shared loads and eight
+// mixed-type adds into fp32 sums; the 32 lanes of a warp hit 32 different groups (the row
+// rotation), i.e. 32 different 8-byte words: two wavefronts per load, conflict-free.
+// Range: the entries of token t in unit (s, k) are scaled by 2^f with
+// f = 12 - floor(log2(8 max|x_t over slice s| max|C_k|)), so every entry is below 2^13 in
+// magnitude and the largest ones use fp16's full precision; the item's sum is multiplied by
+// 2^-f when it is stored. Both scalings are exact. The entries of two consecutive code bytes
+// are first added in fp16 (packed adds; a sum of two stays below 2^14), then widened once
+// into the fp32 sums: one extra fp16 rounding per pair of entries (a longer window measured
+// per-element errors beyond the product tolerance on long rows), half the widening work.
+// Work split, code ring, producer warp, bounded waits and partial planes as gemv_lut (one
+// partial plane per (slice, book, token)); the tables are rebuilt in place behind a barrier.
+constexpr int kLut8MaxM = 6;       // 128 KiB of tables, m codebooks and two 32 KiB code stages
+
+// Packed fp16 pair add, each half rounded to nearest.
+__device__ __forceinline__ uint32_t hadd2(uint32_t a, uint32_t b) {
+    uint32_t d;
+    asm("add.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
+
+inline size_t lut8_smem_bytes(int m, int slots) {
+    return 131072 + (size_t)m * 4096 + (size_t)slots * kSlot + 2 * kSlots * 8;
+}
+
+template <int BDT, int XDT>
+__global__ void __launch_bounds__(kLutThreads, 1)
+gemv_lut8_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
+                 const uint16_t* __restrict__ x, float* __restrict__ partials,
+                 unsigned int* __restrict__ status, int m, int in, int ng, int rows_pad, int RBc,
+                 size_t plane_bytes, int nslots, int cpu, int q, int r, int static_weights,
+                 int batch, int t_base) {
+    extern __shared__ __align__(128) unsigned char smem[];
+    unsigned char* T = smem;                                       // two 64 KiB sub-tables
+    uint4* Cb = (uint4*)(smem + 131072);                           // [m][256] codewords
+    unsigned char* ring = smem + 131072 + (size_t)m * 4096;        // nslots x 32 KiB
+    uint64_t* full = (uint64_t*)(ring + (size_t)nslots * kSlot);
+    uint64_t* empty = full + kSlots;
+    __shared__ volatile int s_abort;
+    __shared__ unsigned int s_cmax[kLut8MaxM];   // bits of max |C_k| (non-negative floats order as ints)
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    int i0, i1;
+    {
+        int b = blockIdx.x, base = 0;
+        if (cpu > 0) {
+            const int u = b / cpu;
+            b -= u * cpu;
+            base = u * RBc;
+        }
+        i0 = base + b * q + min(b, r);
+        i1 = i0 + q + (b < r ? 1 : 0);
+    }
+    const int u_first = i0 / RBc, s_first = u_first / m;
+    struct Walk {
+        int it, s, k, rb, n;
+    };
+    auto walk_start = [&]() {
+        Walk w{i0, s_first, u_first - s_first * m, i0 - u_first * RBc, 0};
+        w.n = min(min(kStageRb, RBc - w.rb), i1 - w.it);
+        return w;
+    };
+    auto walk_next = [&](Walk& w) {
+        w.it += w.n;
+        w.rb += w.n;
+        if (w.rb == RBc) {
+            w.rb = 0;
+            if (++w.k == m) {
+                w.k = 0;
+                ++w.s;
+            }
+        }
+        w.n = min(min(kStageRb, RBc - w.rb), i1 - w.it);
+    };
+
+    int p_q = 0, p_slot = 0;
+    uint32_t p_phase = 0;
+    Walk p_w = walk_start();
+    auto issue_next = [&]() {
+        const size_t src = ((size_t)p_w.s * rows_pad + (size_t)p_w.rb * 32) * 32;
+        mbar_arrive_expect_tx(&full[p_slot], (uint32_t)(p_w.n * 1024));
+        bulk_g2s(ring + (size_t)p_slot * kSlot, planes + (size_t)p_w.k * plane_bytes + src,
+                 (uint32_t)(p_w.n * 1024), &full[p_slot]);
+        ++p_q;
+        if (++p_slot == nslots) {
+            p_slot = 0;
+            p_phase ^= 1u;
+        }
+        walk_next(p_w);
+    };
+    if (tid == 0) {
+        for (int d = 0; d < nslots; ++d) {
+            mbar_init(&full[d], 1);
+            mbar_init(&empty[d], kCons);
+        }
+        mbar_fence_init();
+        s_abort = 0;
+    }
+    if (tid < kLut8MaxM) s_cmax[tid] = 0u;
+    __syncthreads();
+    uint4 cb_r[3];
+    auto load_books = [&]() {
+#pragma unroll
+        for (int i = 0; i < 3; ++i) {
+            const int c = tid + i * kCons * 32;
+            cb_r[i] = (tid < kCons * 32 && c < m * 256) ? __ldg((const uint4*)books + c)
+                                                         : make_uint4(0u, 0u, 0u, 0u);
+        }
+    };
+    if (static_weights) {
+        // read-only weights (AQ_LAYOUT_STATIC_WEIGHTS): codebooks and the first code stage
+        // are requested before waiting for the preceding kernel
+        load_books();
+        if (warp == kCons && lane == 0 && p_w.it < i1) issue_next();
+    }
+    pdl_wait();
+    pdl_launch_dependents();
+    if (!static_weights) load_books();
+
+    if (warp == kCons) {
+        // ---- producer
+        if (lane == 0) {
+            while (p_w.it < i1) {
+                if (s_abort) break;
+                if (p_q >= nslots && !mbar_wait(&empty[p_slot], p_phase ^ 1u)) {
+                    record_status(status, AQ_ERR_TIMEOUT);
+                    s_abort = 1;
+                    break;
+                }
+                issue_next();
+            }
+            for (int j = max(0, p_q - nslots); j < p_q; ++j) mbar_wait(&full[j % nslots], (j / nslots) & 1);
+        }
+        __syncwarp();
+        return;
+    }
+
+    // ---- consumers: stage the codebooks and each book's largest magnitude
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+        const int c = tid + i * kCons * 32;
+        float mx = 0.0f;
+        if (c < m * 256) {
+            Cb[c] = cb_r[i];
+            float f[8];
+            unpack8<BDT>(cb_r[i], f);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) mx = fmaxf(mx, fabsf(f[e]));
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        // the 32 codewords of a warp belong to one book (256 per book)
+        if (lane == 0 && c < m * 256) atomicMax(&s_cmax[c >> 8], __float_as_uint(mx));
+    }
+    named_barrier(1, kCons * 32);
+
+    // Code bytes: each lane reads its row's 32 bytes as two 16-byte halves, lanes 4-7 of every
+    // eight the second half first (conflict-free ring reads). Read position r (0..31) is row
+    // position p = (r + 16 c0) mod 32, group (p + lane) mod 32. gz[v] bytes 0..2 = 8 * group of
+    // read positions 3v..3v+2, byte 3 = 0 (the zero that fills the offset's upper half).
+    const int c0 = (lane >> 2) & 1;
+    uint32_t gz[11];
+#pragma unroll
+    for (int v = 0; v < 11; ++v) {
+        uint32_t z = 0;
+#pragma unroll
+        for (int i = 0; i < 3; ++i) {
+            const int rr = 3 * v + i;
+            if (rr < 32) z |= (uint32_t)((((rr + (c0 ? 16 : 0)) + lane) & 31) * 8) << (8 * i);
+        }
+        gz[v] = z;
+    }
+
+    // Table of unit (s, k) for this pass's tokens: lane g (group g of slice s) computes, for
+    // codewords j = 16*warp .. 16*warp + 15, the entries of all eight tokens from its group's
+    // activations, pre-multiplied by 2^f (exact: f is also limited so that no scaled
+    // activation exceeds 2^100).
+    float sinv[8];      // 2^-f of each token for the current unit
+    auto build = [&](int s, int k) {
+        const int g = s * 32 + lane;
+        const float cmax = __uint_as_float(s_cmax[k]);
+        float xv[8][8];
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+            uint4 xr = make_uint4(0u, 0u, 0u, 0u);
+            if (t_base + t < batch && g < ng) xr = __ldg((const uint4*)(x + (size_t)(t_base + t) * in) + g);
+            unpack8<XDT>(xr, xv[t]);
+        }
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+            float mx = 0.0f;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) mx = fmaxf(mx, fabsf(xv[t][e]));
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            const float bound = 8.0f * mx * cmax;
+            int f = 0;
+            if (bound > 0.0f) f = min(min(126, 100 - exponent_of(mx)), max(-126, 12 - exponent_of(bound)));
+            const float sc = pow2f(f);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) xv[t][e] *= sc;
+            sinv[t] = pow2f(-f);
+        }
+        unsigned char* Tl = T + lane * 8;
+#pragma unroll 2
+        for (int i = 0; i < 16; ++i) {
+            const int j = warp * 16 + i;
+            float c[8];
+            unpack8<BDT>(Cb[k * 256 + j], c);
+            float v[8];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                float2 a = make_float2(xv[t][0] * c[0], xv[t][1] * c[1]);
+                a = ffma2(make_float2(xv[t][2], xv[t][3]), make_float2(c[2], c[3]), a);
+                a = ffma2(make_float2(xv[t][4], xv[t][5]), make_float2(c[4], c[5]), a);
+                a = ffma2(make_float2(xv[t][6], xv[t][7]), make_float2(c[6], c[7]), a);
+                v[t] = a.x + a.y;
+            }
+            uint32_t h[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(h[u]) : "f"(v[2 * u + 1]), "f"(v[2 * u]));
+            *(uint2*)(Tl + j * 256) = make_uint2(h[0], h[1]);
+            *(uint2*)(Tl + 65536 + j * 256) = make_uint2(h[2], h[3]);
+        }
+    };
+
+    int slot = 0;
+    uint32_t phase = 0;
+    int cur_s = -1, cur_k = -1;
+    for (Walk w = walk_start(); w.it < i1; walk_next(w)) {
+        const int n = w.n, s = w.s, rb = w.rb;
+        if (s != cur_s || w.k != cur_k) {
+            if (cur_k >= 0) named_barrier(1, kCons * 32);   // the previous unit looked up
+            build(s, w.k);
+            cur_s = s;
+            cur_k = w.k;
+            named_barrier(1, kCons * 32);                    // the unit's table built
+        }
+        float acc0[8], acc1[8];
+#pragma unroll
+        for (int t = 0; t < 8; ++t) acc0[t] = acc1[t] = 0.0f;
+        bool ok = !s_abort;
+        if (ok && !mbar_wait(&full[slot], phase)) {
+            record_status(status, AQ_ERR_TIMEOUT);
+            s_abort = 1;
+            ok = false;
+        }
+        const bool two = warp + kCons < n;
+        if (ok && warp < n) {
+            const unsigned char* row0 = ring + (size_t)slot * kSlot + warp * 1024 + lane * 32;
+            const uint4 a0 = *(const uint4*)(row0 + c0 * 16);
+            const uint4 b0 = *(const uint4*)(row0 + (c0 ^ 1) * 16);
+            const uint32_t w0[8] = {a0.x, a0.y, a0.z, a0.w, b0.x, b0.y, b0.z, b0.w};
+            uint32_t w1[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+            if (two) {
+                const unsigned char* row1 = row0 + kCons * 1024;
+                const uint4 a1 = *(const uint4*)(row1 + c0 * 16);
+                const uint4 b1 = *(const uint4*)(row1 + (c0 ^ 1) * 16);
+                w1[0] = a1.x; w1[1] = a1.y; w1[2] = a1.z; w1[3] = a1.w;
+                w1[4] = b1.x; w1[5] = b1.y; w1[6] = b1.z; w1[7] = b1.w;
+            }
+            // The four code bytes of word qq: offsets j*256 + 8g; the entries (fp16 pairs of
+            // tokens 0-1, 2-3, 4-5, 6-7) of bytes 0+1 and of bytes 2+3 are added in fp16, then
+            // widened into the fp32 sums.
+            auto look4 = [&](uint32_t code_word, int qq, float (&acc)[8]) {
+#pragma unroll
+                for (int i = 0; i < 4; i += 2) {
+                    uint32_t sum[4];
+#pragma unroll
+                    for (int ii = 0; ii < 2; ++ii) {
+                        const int rr = 4 * qq + i + ii;
+                        const uint32_t sel =
+                            0x7700u | ((uint32_t)(i + ii) << 4) | (uint32_t)(4 + rr % 3);
+                        const uint32_t o = prmt(code_word, gz[rr / 3], sel);
+                        const uint2 lo = *(const uint2*)(T + o);
+                        const uint2 hi = *(const uint2*)(T + 65536 + o);
+                        if (ii == 0) {
+                            sum[0] = lo.x; sum[1] = lo.y; sum[2] = hi.x; sum[3] = hi.y;
+                        } else {
+                            sum[0] = hadd2(sum[0], lo.x);
+                            sum[1] = hadd2(sum[1], lo.y);
+                            sum[2] = hadd2(sum[2], hi.x);
+                            sum[3] = hadd2(sum[3], hi.y);
+                        }
+                    }
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) add_widen2<AQ_F16>(sum[u], acc[2 * u], acc[2 * u + 1]);
+                }
+            };
+#pragma unroll
+            for (int qq = 0; qq < 8; ++qq) {
+                look4(w0[qq], qq, acc0);
+                if (two) look4(w1[qq], qq, acc1);
+            }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[slot]);
+        if (++slot == nslots) {
+            slot = 0;
+            phase ^= 1u;
+        }
+        if (ok && warp < n) {
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                if (t_base + t >= batch) break;
+                float* dst = partials + (((size_t)s * m + cur_k) * batch + t_base + t) * rows_pad +
+                             (size_t)(rb + warp) * 32 + lane;
+                dst[0] = acc0[t] * sinv[t];
+                if (two) dst[kCons * 32] = acc1[t] * sinv[t];
+            }
+        }
+    }
+}
+
 // ------------------------------------------------------------------ direct kernel (any B, b <= 16)
 
 template <int NB, int B, int BDT, int SDT>
@@ -911,6 +1232,61 @@ aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
                       (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0, a.batch);
 }
 
+// One pass of gemv_lut8 over tokens [t_base, t_base + 8): the work split of run_lut.
+template <int BDT, int XDT>
+aq_status run_lut8(const Dims& d, int m, const GemvArgs& a, int t_base, cudaStream_t st) {
+    DeviceInfo di;
+    if (aq_status e = device_info(&di); e != AQ_OK) return e;
+    auto kern = gemv_lut8_kernel<BDT, XDT>;
+    const size_t fixed = lut8_smem_bytes(m, 0) + 8192;
+    int nslots = di.smem_optin > (int)fixed ? (int)((di.smem_optin - fixed) / kSlot) : 0;
+    if (nslots > kSlots) nslots = kSlots;
+    if (nslots < 2) return AQ_ERR_UNSUPPORTED;
+    const size_t smem = lut8_smem_bytes(m, nslots);
+    int occ = 0;
+    if (aq_status e = prepare(kern, smem, kLutThreads, m, &occ); e != AQ_OK) return e;
+    const long long units = (long long)d.S * m;
+    const long long items = units * d.RBc;
+    if (items > 0x7fffffffLL) return AQ_ERR_UNSUPPORTED;
+    // An 8-token table build costs about eight times a one-token build.
+    constexpr long long kTableItems = 280;
+    long long cpu = di.sms / units;
+    if (cpu > d.RBc) cpu = d.RBc;
+    long long cost_cpu = -1;
+    if (cpu >= 1) cost_cpu = kTableItems + (d.RBc + cpu - 1) / cpu;
+    const long long grid_b = items < di.sms ? items : di.sms;
+    const long long qb = items / grid_b, rb = items % grid_b;
+    long long cost_b = 0;
+    for (long long b = 0; b < grid_b; ++b) {
+        const long long i0 = b * qb + (b < rb ? b : rb), i1 = i0 + qb + (b < rb ? 1 : 0);
+        const long long tables = (i1 - 1) / d.RBc - i0 / d.RBc + 1;
+        const long long c = tables * kTableItems + (i1 - i0);
+        if (c > cost_b) cost_b = c;
+    }
+    int grid, q, r;
+    if (cost_cpu >= 0 && cost_cpu <= cost_b) {
+        grid = (int)(cpu * units);
+        q = d.RBc / (int)cpu;
+        r = d.RBc % (int)cpu;
+    } else {
+        cpu = 0;
+        grid = (int)grid_b;
+        q = (int)qb;
+        r = (int)rb;
+    }
+    return launch_pdl(kern, dim3(grid), dim3(kLutThreads), smem, st, (const uint8_t*)a.planes,
+                      (const uint16_t*)a.books, (const uint16_t*)a.x, a.partials, a.status, m,
+                      d.in, d.ng, d.rows_pad, d.RBc, d.plane_bytes, nslots, (int)cpu, q, r,
+                      (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0, a.batch, t_base);
+}
+
+template <int BDT, int XDT>
+aq_status run_lut8_all(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
+    for (int t = 0; t < a.batch; t += 8)
+        if (aq_status e = run_lut8<BDT, XDT>(d, m, a, t, st); e != AQ_OK) return e;
+    return AQ_OK;
+}
+
 template <int NB, int B, int BDT, int SDT>
 aq_status run_direct(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
     DeviceInfo di;
@@ -1032,6 +1408,14 @@ static aq_status launch_product(const Dims& d, int m, const void* planes, const 
                 case 1: return run_lut<AQ_F16, AQ_BF16, 2>(d, m, a, st);
                 case 2: return run_lut<AQ_BF16, AQ_F16, 2>(d, m, a, st);
                 default: return run_lut<AQ_BF16, AQ_BF16, 2>(d, m, a, st);
+            }
+        }
+        if (batch > 4) {
+            switch (bb * 2 + xb) {
+                case 0: return run_lut8_all<AQ_F16, AQ_F16>(d, m, a, st);
+                case 1: return run_lut8_all<AQ_F16, AQ_BF16>(d, m, a, st);
+                case 2: return run_lut8_all<AQ_BF16, AQ_F16>(d, m, a, st);
+                default: return run_lut8_all<AQ_BF16, AQ_BF16>(d, m, a, st);
             }
         }
         switch (bb * 2 + xb) {

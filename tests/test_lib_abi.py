@@ -230,3 +230,14 @@ def test_selftest_read_argument_errors_on_the_host():
     assert lib.aq_selftest_read(FAKE + 8, 1024, FAKE, None) == aq.AQ_ERR_ALIGNMENT
     assert lib.aq_selftest_read(FAKE, 1000, FAKE, None) == aq.AQ_ERR_ALIGNMENT
     assert lib.aq_selftest_read(FAKE, 1024, FAKE + 2, None) == aq.AQ_ERR_ALIGNMENT
+
+
+def test_gemv_workspace_follows_the_kernel_choice():
+    """Batch 5..8: one partial plane per (slice, book, token) when the eight-token table kernel
+    serves the layer (at least 4560 (slice, book, row block) items at the largest prefix it
+    takes, six books), else one per (slice, token)."""
+    big = aq.Layout.make(1000, 8200, 6)            # 33 slices x 6 books x 32 row blocks
+    assert aq.gemv_workspace_bytes(big, 8) == 256 + 33 * 8 * 6 * 1024 * 4
+    small = aq.Layout.make(300, 1032, 4)           # 5 slices x 4 books x 10 row blocks
+    assert aq.gemv_workspace_bytes(small, 8) == 256 + 5 * 8 * 320 * 4
+    assert aq.gemv_workspace_bytes(big, 16) == 256 + 33 * 16 * 1024 * 4
