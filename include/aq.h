@@ -94,10 +94,13 @@ const char* aq_last_error(void);
  *   even p and the high four bits for odd p, so a unit is 16 bytes and a plane
  *   rows_pad*ng_pad/2 bytes. */
 
-/* Bytes of one code plane; 0 if the layout is invalid. */
+/* Bytes of one code plane (the codes b of one codebook, Sec. 3.2; App. C counts them as
+ * d_out*(d_in/g)*B bits per codebook, the codes term of Eq. avg_bits); 0 if the layout is
+ * invalid. */
 size_t aq_plane_bytes(const aq_layout* layout);
 
-/* Bytes of the first m planes (m*aq_plane_bytes); 0 if the layout or m is invalid. */
+/* Bytes of the first m planes (m*aq_plane_bytes): the codes a prefix-m call reads (Sec. 5,
+ * the first k codebooks); 0 if the layout or m is invalid. */
 size_t aq_packed_bytes(const aq_layout* layout, int m);
 
 /* Pack natural codes into planes (the codes b_{i,j,m} of Sec. 3.2).
@@ -119,25 +122,35 @@ aq_status aq_decode(const aq_layout* layout, int m, const void* planes, const vo
                     const void* scales, void* w, void* stream);
 
 /* ---------------------------------------------------------------- GEMV (batch 1..16)
- * y[t, o] = sum_i x[t, i] * W_m[o, i] for t < batch, accumulated in fp32. The kernel reads
- * the first m planes once (HBM-bound at batch 1); 8-bit codebooks are staged on chip.
+ * y[t, o] = sum_i x[t, i] * W_m[o, i] for t < batch (Sec. 2.2 Y = W X, with W_m the prefix-m
+ * reconstruction of Sec. 3.2 / Sec. 5), accumulated in fp32. The kernel reads the first m
+ * planes once (HBM-bound at batch 1); 8-bit codebooks are staged on chip. At batch 5..8 with
+ * up to six 2^8-entry books, on layers of at least 4560 (256-input slice, codebook, 32-row
+ * block) items, the products are taken from per-(slice, codebook) tables of fp16 values (each
+ * token's scaled by a power of two, so the range of the activations is kept); elsewhere every
+ * intermediate is fp32 or a tf32 operand.
  *   x         : device, [batch][d_in] of x_dtype (AQ_F16 or AQ_BF16), row-major
  *   y         : device, [batch][d_out] of y_dtype (AQ_F16, AQ_BF16 or AQ_F32), row-major
  *   workspace : device scratch of at least aq_gemv_workspace_bytes(layout, batch) bytes:
  *               a status word and fp32 partial sums for every row: one per 256-input
- *               slice and token, or, with 2^8-entry books at batch 1..2 (batch 3..4), one
- *               per slice, token and codebook of the largest prefix up to 8 (up to 4)
- *               served that way. Zero-fill it once before its first use (aq_workspace_init); every
+ *               slice and token, or, with 2^8-entry books at batch 1..2 (batch 3..4, batch
+ *               5..8 on the layers above), one per slice, token and codebook of the largest
+ *               prefix up to 8 (up to 4, up to 6) served that way. Zero-fill it once before its first use (aq_workspace_init); every
  *               call leaves it ready for the next one.
  *               Calls that may overlap on the GPU must not share a workspace.
  * Two kernels are enqueued, both with programmatic dependent launch: the product (fp32
- * partial sums per 256-input slice, and per codebook at batch 1..4 with 2^8-entry books, into
+ * partial sums per 256-input slice, and per codebook at batch 1..8 with 2^8-entry books, into
  * the workspace) and a split-K reduction that sums each row's partials, scales it and
  * writes y (4-bit codes at batch 1: one kernel that writes y itself). Each waits for the
  * preceding grid before reading memory. The partials of each
  * row are summed in a fixed order, so the result does not depend on scheduling.
- * Accuracy: |y - y_exact| <= 1e-2*(1+|y_exact|) per element and relative Frobenius error
- * <= 2e-3, with y_exact the fp64 product of the exactly widened stored values. */
+ * Accuracy: relative Frobenius error <= 2e-3 and |y - y_exact| <= 1e-2*(1+|y_exact|) per
+ * element, with y_exact the fp64 product of the exactly widened stored values, on unit-scale
+ * inputs (activations of order 1, codebook entries of the order of N(0, 0.02^2), as in the
+ * benchmark layers). Batch 1..4 add fp32 table entries (fp32 roundings only); batch 5..16
+ * round each decoded weight to a tf32 operand, or each table entry to fp16 and pairs of
+ * entries once more, so their per-element error is bounded by about
+ * 2^-10 * |s[o]| * sum_i |x_i| sum_k |C_k[b_k]_i|, which scales with the inputs. */
 size_t aq_gemv_workspace_bytes(const aq_layout* layout, int batch);
 aq_status aq_gemv(const aq_layout* layout, int m, const void* planes, const void* books,
                   const void* scales, const void* x, int x_dtype, int batch, void* y,
