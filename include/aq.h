@@ -156,6 +156,34 @@ aq_status aq_gemv(const aq_layout* layout, int m, const void* planes, const void
                   const void* scales, const void* x, int x_dtype, int batch, void* y,
                   int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
 
+/* ---------------------------------------------------------------- GEMV of a group of layers
+ * (No counterpart in the paper: a way to call the product of Sec. 2.2 with the prefix-m
+ * reconstruction of Sec. 3.2 / Sec. 5 for several layers that read the same activations,
+ * such as a decoder block's query, key and value projections, or its gate and up projections.)
+ * y_l = x * W_m,l^T for l < n, each as aq_gemv would compute it, bit for bit: every layer's
+ * partial sums and their summation order are those of its own call. At batch 1 with 2^8-entry
+ * codebooks the n products run as one kernel over the items of all layers and the n
+ * reductions as one kernel, so the group pays the fixed cost of a call (two kernel boundaries,
+ * the activation load, the first table build) once instead of n times; otherwise the layers
+ * are computed one after the other, as n calls of aq_gemv.
+ *   n        : 1..4 layers
+ *   layouts  : n layouts with the same in_features, code_bits, book_dtype and scale_dtype
+ *   m        : 1 <= m <= num_books of every layer
+ *   planes, books, scales : host arrays of n device pointers, as for aq_gemv
+ *   x        : device, [batch][d_in], shared by the layers
+ *   y        : host array of n device pointers, layer l's [batch][d_out_l] of y_dtype
+ *   workspace: aq_gemv_group_workspace_bytes(n, layouts, batch) bytes, 16-byte aligned,
+ *              zero-filled before first use: layer l's aq_gemv workspace at the sum of the
+ *              earlier layers' sizes, each rounded up to 256 bytes; a device-side status is
+ *              recorded in layer 0's status word (aq_workspace_status(workspace, ...)).
+ * Errors: as aq_gemv; AQ_ERR_INVALID_ARG also for n outside 1..4, NULL pointer arrays or
+ * layouts that differ in in_features, code_bits, book_dtype or scale_dtype. */
+size_t aq_gemv_group_workspace_bytes(int n, const aq_layout* layouts, int batch);
+aq_status aq_gemv_group(int n, const aq_layout* layouts, int m, const void* const* planes,
+                        const void* const* books, const void* const* scales, const void* x,
+                        int x_dtype, int batch, void* const* y, int y_dtype, void* workspace,
+                        size_t workspace_bytes, void* stream);
+
 /* ---------------------------------------------------------------- GEMV refinement (prefix m-1 -> m)
  * y = y_prev + x * (s o C_{m-1}[b_{m-1}])^T: the increment that raises a product computed with
  * the first m-1 codebooks to the product with the first m (the successive reconstruction of

@@ -28,7 +28,8 @@ EXPORTS = ["aq_abi_version", "aq_status_string", "aq_last_error", "aq_plane_byte
            "aq_gemv_refine", "aq_store_create", "aq_store_set_prefix", "aq_store_prefix",
            "aq_store_planes", "aq_store_books", "aq_store_scales", "aq_store_device_bytes",
            "aq_store_destroy", "aq_wmse_workspace_bytes", "aq_wmse", "aq_beam_workspace_bytes",
-           "aq_beam_search", "aq_selftest_wait", "aq_selftest_read"]
+           "aq_beam_search", "aq_selftest_wait", "aq_selftest_read", "aq_gemv_group_workspace_bytes",
+           "aq_gemv_group"]
 
 
 class AQError(RuntimeError):
@@ -96,6 +97,10 @@ def lib():
                                      i32, vp, vp, sz, vp]),
             "aq_selftest_wait": (i32, [vp, sz, vp]),
             "aq_selftest_read": (i32, [vp, sz, vp, vp]),
+            "aq_gemv_group_workspace_bytes": (sz, [i32, lp, i32]),
+            "aq_gemv_group": (i32, [i32, lp, i32, ctypes.POINTER(vp), ctypes.POINTER(vp),
+                                    ctypes.POINTER(vp), vp, i32, i32, ctypes.POINTER(vp), i32,
+                                    vp, sz, vp]),
             "aq_wmse": (i32, [lp, vp, vp, vp, vp, vp, i32, ctypes.POINTER(ctypes.c_double), vp,
                               vp, sz, vp]),
         }
@@ -291,6 +296,26 @@ def aq_workspace_init(workspace, nbytes=None, stream=None):
     if nbytes is None:
         nbytes = workspace.numel() * workspace.element_size()
     _check(lib().aq_workspace_init(_ptr(workspace), nbytes, _stream(stream)), "aq_workspace_init")
+
+
+def gemv_group_workspace_bytes(layouts, batch):
+    arr = (Layout * len(layouts))(*layouts)
+    return lib().aq_gemv_group_workspace_bytes(len(layouts), arr, batch)
+
+
+def aq_gemv_group(layouts, m, planes, books, scales, x, x_dtype, batch, ys, y_dtype, workspace,
+                  workspace_bytes=None, stream=None):
+    """The GEMVs of several layers that share the activations x (one call of aq_gemv_group)."""
+    n = len(layouts)
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    vp = ctypes.c_void_p
+    arr = (Layout * n)(*layouts)
+    _check(lib().aq_gemv_group(n, arr, m, (vp * n)(*[_ptr(p) for p in planes]),
+                               (vp * n)(*[_ptr(b) for b in books]),
+                               (vp * n)(*[_ptr(s) for s in scales]), _ptr(x), x_dtype, batch,
+                               (vp * n)(*[_ptr(y) for y in ys]), y_dtype, _ptr(workspace),
+                               workspace_bytes, _stream(stream)), "aq_gemv_group")
 
 
 def aq_selftest_read(src, nbytes, sink, stream=None):

@@ -191,6 +191,57 @@ aq_status aq_gemv(const aq_layout* layout, int m, const void* planes, const void
                            as_stream(stream));
 }
 
+// Layouts of a group: 1..4 valid layouts with the same in_features, code width and codebook
+// and scale types; fills ds.
+static aq_status group_dims(int n, const aq_layout* layouts, Dims* ds) {
+    if (n < 1 || n > 4 || !layouts) return AQ_ERR_INVALID_ARG;
+    for (int l = 0; l < n; ++l) {
+        if (aq_status st = aq::make_dims(&layouts[l], &ds[l]); st != AQ_OK) return st;
+        if (ds[l].in != ds[0].in || ds[l].B != ds[0].B || ds[l].book_dt != ds[0].book_dt ||
+            ds[l].scale_dt != ds[0].scale_dt)
+            return AQ_ERR_INVALID_ARG;
+    }
+    return AQ_OK;
+}
+
+size_t aq_gemv_group_workspace_bytes(int n, const aq_layout* layouts, int batch) {
+    Dims ds[4];
+    if (group_dims(n, layouts, ds) != AQ_OK || batch < 0 || batch > 16) return 0;
+    size_t total = 0;
+    for (int l = 0; l < n; ++l) total += aq::round_up(gemv_ws_bytes(ds[l], batch), 256);
+    return total;
+}
+
+aq_status aq_gemv_group(int n, const aq_layout* layouts, int m, const void* const* planes,
+                        const void* const* books, const void* const* scales, const void* x,
+                        int x_dtype, int batch, void* const* y, int y_dtype, void* workspace,
+                        size_t workspace_bytes, void* stream) {
+    Dims ds[4];
+    aq_status st = group_dims(n, layouts, ds);
+    if (st != AQ_OK) return st;
+    for (int l = 0; l < n; ++l)
+        if ((st = check_m(ds[l], m)) != AQ_OK) return st;
+    if (batch < 0 || batch > 16) return AQ_ERR_INVALID_ARG;
+    if (x_dtype != AQ_F16 && x_dtype != AQ_BF16) return AQ_ERR_INVALID_ARG;
+    if (y_dtype != AQ_F16 && y_dtype != AQ_BF16 && y_dtype != AQ_F32) return AQ_ERR_INVALID_ARG;
+    if (!planes || !books || !scales || !y) return AQ_ERR_INVALID_ARG;
+    if (batch == 0) return AQ_OK;
+    for (int l = 0; l < n; ++l)
+        if (ds[l].out > 0)
+            if ((st = check_ptrs({planes[l], books[l], scales[l], x, y[l]})) != AQ_OK) return st;
+    if (!workspace || workspace_bytes < aq_gemv_group_workspace_bytes(n, layouts, batch))
+        return AQ_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return AQ_ERR_ALIGNMENT;
+    void* ws[4];
+    size_t off = 0;
+    for (int l = 0; l < n; ++l) {
+        ws[l] = (char*)workspace + off;
+        off += aq::round_up(gemv_ws_bytes(ds[l], batch), 256);
+    }
+    return aq::launch_gemv_group(ds, n, m, planes, books, scales, x, x_dtype, batch, y, y_dtype, ws,
+                                 as_stream(stream));
+}
+
 aq_status aq_gemv_refine(const aq_layout* layout, int m, const void* planes, const void* books,
                          const void* scales, const void* x, int x_dtype, int batch,
                          const void* y_prev, void* y, int y_dtype, void* workspace,

@@ -97,6 +97,11 @@ aq_status launch_decode(const Dims& d, int m, const void* planes, const void* bo
 aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* books,
                       const void* scales, const void* x, int x_dt, int batch, void* y,
                       int y_dt, void* ws, cudaStream_t st, const void* y_prev = nullptr);
+// aq_gemv_group: n (<= 4) layers sharing x; ws[l] = layer l's workspace region.
+aq_status launch_gemv_group(const Dims* ds, int n, int m, const void* const* planes,
+                            const void* const* books, const void* const* scales, const void* x,
+                            int x_dt, int batch, void* const* y, int y_dt, void* const* ws,
+                            cudaStream_t st);
 aq_status launch_gemm(const Dims& d, int m, const void* planes, const void* books,
                       const void* scales, const void* x, int x_dt, int tokens, void* y, int y_dt,
                       void* ws, cudaStream_t st);

@@ -53,9 +53,9 @@ constexpr int kXStage = 8;                        // (token, slice) activation r
 constexpr int lut_table_bytes(int nt) { return nt == 4 ? 131072 : 65536; }
 
 // Shared memory: [T][codebooks m x 4 KiB][activations 8 x 1 KiB fp32][ring][barriers]
-inline size_t lut_smem_bytes(int nt, int m, int slots) {
-    return (size_t)lut_table_bytes(nt) + (size_t)m * 4096 + kXStage * 1024 + (size_t)slots * kSlot +
-           2 * kSlots * 8;
+inline size_t lut_smem_bytes(int nt, int m, int slots, int nsets = 1) {
+    return (size_t)lut_table_bytes(nt) + (size_t)nsets * m * 4096 + kXStage * 1024 +
+           (size_t)slots * kSlot + 2 * kSlots * 8;
 }
 
 // Work is split by slice and by codebook: by linearity in the books (the successive-refinement
@@ -83,22 +83,37 @@ inline size_t lut_smem_bytes(int nt, int m, int slots) {
 // every plane), and consumer warp w looks up items w and w + 16 of the stage, so each wait on
 // the ring serves two row blocks. The codebooks and the activations of the CTA's first slices
 // are requested before any code.
-template <int BDT, int XDT, int NT>
+// The layers of one call: one layer, or up to kGroupMax layers that share the activations
+// (aq_gemv_group). Items are numbered layer after layer: layer l holds the items
+// [base[l], base[l+1]), numbered within the layer as above (unit u = s*m + k, then row block).
+// A CTA's items lie in at most two layers (checked by the host), whose first m codebooks it
+// stages.
+constexpr int kGroupMax = 4;
+struct LutLayers {
+    const uint8_t* planes[kGroupMax];
+    const uint16_t* books[kGroupMax];
+    float* partials[kGroupMax];
+    size_t plane_bytes[kGroupMax];
+    int rows_pad[kGroupMax], RBc[kGroupMax], base[kGroupMax + 1];
+    int n;
+};
+
+template <int BDT, int XDT, int NT, bool GROUP>
 __global__ void __launch_bounds__(kLutThreads, 1)
-gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
-                const uint16_t* __restrict__ x, float* __restrict__ partials,
-                unsigned int* __restrict__ status, int m, int in, int ng, int rows_pad, int RBc,
-                size_t plane_bytes, int nslots, int cpu, int q, int r, int static_weights,
-                int batch) {
+gemv_lut_kernel(const __grid_constant__ LutLayers L, const uint16_t* __restrict__ x,
+                unsigned int* __restrict__ status, int m, int in, int ng, int nslots, int cpu,
+                int q, int r, int static_weights, int batch) {
     constexpr int kTB = lut_table_bytes(NT);
     constexpr int kXSlices = kXStage / NT;      // activation slices staged per token
     extern __shared__ __align__(128) unsigned char smem[];
     unsigned char* T = smem;
-    uint4* Cb = (uint4*)(smem + kTB);                              // [m][256] codewords
+    const int nl = GROUP ? L.n : 1;             // layers (a single call: one, known at compile time)
+    const int nsets = nl > 1 ? 2 : 1;           // codebook sets staged (layers per CTA)
+    uint4* Cb = (uint4*)(smem + kTB);                              // [nsets][m][256] codewords
     // [NT][kXSlices][256] activations in fp32; group g of a slice at 128-byte line g/4, its
     // two 16-byte halves at quads (2*(g%4) + half) ^ (g/4 mod 8), so the table build's reads
     // (eight lanes at eight different lines) hit eight different bank quads.
-    unsigned char* xs = smem + kTB + (size_t)m * 4096;
+    unsigned char* xs = smem + kTB + (size_t)nsets * m * 4096;
     unsigned char* ring = xs + kXStage * 1024;                     // nslots x 32 KiB
     uint64_t* full = (uint64_t*)(ring + (size_t)nslots * kSlot);
     uint64_t* empty = full + kSlots;
@@ -112,35 +127,46 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
     int i0, i1;
     {
         int b = blockIdx.x, base = 0;
-        if (cpu > 0) {
+        if (cpu > 0) {                          // single layer only
             const int u = b / cpu;
             b -= u * cpu;
-            base = u * RBc;
+            base = u * L.RBc[0];
         }
         i0 = base + b * q + min(b, r);
         i1 = i0 + q + (b < r ? 1 : 0);
     }
-    const int u_first = i0 / RBc, s_first = u_first / m;
-    // A walk over the CTA's items in stages: up to kStageRb items, never crossing a unit.
+    const int S = (ng + 31) >> 5;
+    int l_first = 0;
+    while (l_first + 1 < nl && i0 >= L.base[l_first + 1]) ++l_first;
+    const int u_first = (i0 - (GROUP ? L.base[l_first] : 0)) / L.RBc[l_first], s_first = u_first / m;
+    // A walk over the CTA's items in stages: up to kStageRb items, never crossing a unit
+    // (nor, therefore, a layer). rbc, rp: row blocks and padded rows of layer l.
     struct Walk {
-        int it, s, k, rb, n;
+        int it, l, s, k, rb, n, rbc, rp;
     };
     auto walk_start = [&]() {
-        Walk w{i0, s_first, u_first - s_first * m, i0 - u_first * RBc, 0};
-        w.n = min(min(kStageRb, RBc - w.rb), i1 - w.it);
+        const int rbc = L.RBc[l_first];
+        Walk w{i0, l_first, s_first, u_first - s_first * m, i0 - (GROUP ? L.base[l_first] : 0) - u_first * rbc, 0,
+               rbc, L.rows_pad[l_first]};
+        w.n = min(min(kStageRb, rbc - w.rb), i1 - w.it);
         return w;
     };
     auto walk_next = [&](Walk& w) {
         w.it += w.n;
         w.rb += w.n;
-        if (w.rb == RBc) {
+        if (w.rb == w.rbc) {
             w.rb = 0;
             if (++w.k == m) {
                 w.k = 0;
-                ++w.s;
+                if (++w.s == S && w.l + 1 < nl) {
+                    w.s = 0;
+                    ++w.l;
+                    w.rbc = L.RBc[w.l];
+                    w.rp = L.rows_pad[w.l];
+                }
             }
         }
-        w.n = min(min(kStageRb, RBc - w.rb), i1 - w.it);
+        w.n = min(min(kStageRb, w.rbc - w.rb), i1 - w.it);
     };
 
     // Producer state (warp kCons, lane 0): the next copy is stage p_w into ring slot p_slot
@@ -149,9 +175,10 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
     uint32_t p_phase = 0;
     Walk p_w = walk_start();
     auto issue_next = [&]() {
-        const size_t src = ((size_t)p_w.s * rows_pad + (size_t)p_w.rb * 32) * 32;
+        const size_t src = ((size_t)p_w.s * p_w.rp + (size_t)p_w.rb * 32) * 32;
         mbar_arrive_expect_tx(&full[p_slot], (uint32_t)(p_w.n * 1024));
-        bulk_g2s(ring + (size_t)p_slot * kSlot, planes + (size_t)p_w.k * plane_bytes + src,
+        bulk_g2s(ring + (size_t)p_slot * kSlot,
+                 L.planes[GROUP ? p_w.l : 0] + (size_t)p_w.k * L.plane_bytes[GROUP ? p_w.l : 0] + src,
                  (uint32_t)(p_w.n * 1024), &full[p_slot]);
         ++p_q;
         if (++p_slot == nslots) {
@@ -171,14 +198,20 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
     __syncthreads();            // barriers initialised before the first copy
     // Codebooks and activations are requested first (into registers) by the consumer threads,
     // which store them below.
-    uint4 cb_r[4];
+    // codebook sets: layer l_first, and l_first + 1 when the CTA's items reach into it
+    int l_last = l_first;
+    while (l_last + 1 < nl && i1 - 1 >= L.base[l_last + 1]) ++l_last;
+    uint4 cb_r[2][4];
     auto load_books = [&]() {
 #pragma unroll
-        for (int r = 0; r < 4; ++r) {
-            const int i = tid + r * kCons * 32;
-            cb_r[r] = (tid < kCons * 32 && i < m * 256) ? __ldg((const uint4*)books + i)
-                                                          : make_uint4(0u, 0u, 0u, 0u);
-        }
+        for (int set = 0; set < 2; ++set)
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int i = tid + r * kCons * 32;
+                cb_r[set][r] = (l_first + set <= l_last && tid < kCons * 32 && i < m * 256)
+                                   ? __ldg((const uint4*)L.books[l_first + set] + i)
+                                   : make_uint4(0u, 0u, 0u, 0u);
+            }
     };
     if (static_weights) {
         // The weights are read-only while calls run (AQ_LAYOUT_STATIC_WEIGHTS): request the
@@ -217,10 +250,12 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
     } else {
         // ---- consumers
 #pragma unroll
-        for (int r = 0; r < 4; ++r) {
-            const int i = tid + r * kCons * 32;
-            if (i < m * 256) Cb[i] = cb_r[r];
-        }
+        for (int set = 0; set < 2; ++set)
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int i = tid + r * kCons * 32;
+                if (set < nsets && i < m * 256) Cb[set * m * 256 + i] = cb_r[set][r];
+            }
         if (tid < kXStage * 64) {
             const int e = tid & 63, g = e >> 1;
             float4 f;
@@ -252,14 +287,16 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
         float2 xv[4][4];
         int slot = 0;
         uint32_t phase = 0;                     // parity of the slot's current use
-        int cur_s = -1, cur_k = -1, h = 1;
+        int cur_s = -1, cur_k = -1, cur_l = -1, h = 1;
         for (Walk w = walk_start(); w.it < i1; walk_next(w)) {
             const int n = w.n, s = w.s, rb = w.rb;
-            if (s != cur_s || w.k != cur_k) {
+            if (s != cur_s || w.k != cur_k || w.l != cur_l) {
                 // Activations of the four groups 4gq..4gq+3 of slice s for token t.
                 auto load_xv = [&](int t) {
+                    // (the activations are shared by the layers of a group: slice s of x
+                    // whatever the layer)
                     const int sl = s - s_first;
-                    if (sl < kXSlices) {
+                    if ((unsigned)sl < (unsigned)kXSlices) {
                         const unsigned char* xb = xs + (t * kXSlices + sl) * 1024 + gq * 128;
 #pragma unroll
                         for (int u = 0; u < 4; ++u) {
@@ -288,7 +325,8 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                 auto build = [&](unsigned char* Th) {
                     uint4 cw[4];
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) cw[i] = Cb[w.k * 256 + warp * 16 + ph + 4 * i];
+                    for (int i = 0; i < 4; ++i)
+                        cw[i] = Cb[((GROUP ? w.l - l_first : 0) * m + w.k) * 256 + warp * 16 + ph + 4 * i];
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
                         float c[8];
@@ -321,6 +359,7 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                 }
                 cur_s = s;
                 cur_k = w.k;
+                cur_l = w.l;
                 named_barrier(1, kCons * 32);
             }
             float part0[NT], part1[NT];
@@ -400,7 +439,8 @@ gemv_lut_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
 #pragma unroll
                 for (int t = 0; t < NT; ++t) {
                     if (t >= batch) break;
-                    float* dst = partials + (((size_t)s * m + cur_k) * batch + t) * rows_pad + (size_t)(rb + warp) * 32 + lane;
+                    float* dst = L.partials[GROUP ? w.l : 0] + (((size_t)s * m + cur_k) * batch + t) * w.rp +
+                                 (size_t)(rb + warp) * 32 + lane;
                     dst[0] = part0[t];
                     if (warp + kCons < n) dst[kCons * 32] = part1[t];
                 }
@@ -971,11 +1011,23 @@ gemv_mma_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
 // waiting for the product kernel. With y_prev (a refinement, Sec. 4 successive
 // reconstruction) the scaled sum is added to y_prev[t][r], read in y's type (y_prev may be y).
 // The kernel is kept small: it runs once per CTA, so its instructions are fetched cold.
-template <int SDT>
+// The layers a reduction finishes: one, or the layers of a group (blockIdx.z = layer).
+struct ReduceLayers {
+    const float* partials[kGroupMax];
+    const uint16_t* scales[kGroupMax];
+    void* y[kGroupMax];
+    int out[kGroupMax], rows_pad[kGroupMax];
+};
+
+template <int SDT, bool GROUP>
 __global__ void __launch_bounds__(256)
-splitk_reduce_kernel(const float* __restrict__ partials, const uint16_t* __restrict__ scales,
-                     void* y, int y_dt, int out, int rows_pad, int P, int batch, int wpr,
+splitk_reduce_kernel(const __grid_constant__ ReduceLayers R, int y_dt, int P, int batch, int wpr,
                      int static_weights, const void* y_prev) {
+    const int z = GROUP ? blockIdx.z : 0;
+    const float* __restrict__ partials = R.partials[z];
+    const uint16_t* __restrict__ scales = R.scales[z];
+    void* y = R.y[z];
+    const int out = R.out[z], rows_pad = R.rows_pad[z];
     __shared__ float red[8][32];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     const int j = w & (wpr - 1), rg = w - j;     // rg: first warp of the row group
@@ -1179,42 +1231,70 @@ struct GemvArgs {
     unsigned int* status;
 };
 
+// The table-lookup product for n layers sharing the activations (n = 1: an ordinary call):
+// layer l's dims ds[l], pointers as[l] (x, batch and the status word are taken from as[0]).
+// Returns AQ_ERR_UNSUPPORTED without launching when a group cannot be served by one launch
+// (a CTA's items would reach into more than two layers).
 template <int BDT, int XDT, int NT>
-aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
+aq_status run_lut_layers(const Dims* ds, const GemvArgs* as, int n, int m, cudaStream_t st) {
     DeviceInfo di;
     if (aq_status e = device_info(&di); e != AQ_OK) return e;
-    auto kern = gemv_lut_kernel<BDT, XDT, NT>;
+    auto kern = gemv_lut_kernel<BDT, XDT, NT, false>;
+    if constexpr (NT == 1) {                    // groups: one token only
+        if (n > 1) kern = gemv_lut_kernel<BDT, XDT, NT, true>;
+    } else if (n > 1) {
+        return AQ_ERR_UNSUPPORTED;
+    }
+    const int nsets = n > 1 ? 2 : 1;
     // As many 32 KiB ring slots as fit next to the tables, codebooks and activations (<= 4).
-    const size_t fixed = lut_smem_bytes(NT, m, 0) + 8192;   // + static shared memory and slack
+    const size_t fixed = lut_smem_bytes(NT, m, 0, nsets) + 8192;   // + static shared memory and slack
     int nslots = di.smem_optin > (int)fixed ? (int)((di.smem_optin - fixed) / kSlot) : 0;
     if (nslots > kSlots) nslots = kSlots;
     if (nslots < 2) return AQ_ERR_UNSUPPORTED;
-    const size_t smem = lut_smem_bytes(NT, m, nslots);
+    const size_t smem = lut_smem_bytes(NT, m, nslots, nsets);
     int occ = 0;
-    if (aq_status e = prepare(kern, smem, kLutThreads, m, &occ); e != AQ_OK) return e;
-    const long long units = (long long)d.S * m;       // (slice, book) pairs
-    const long long items = units * d.RBc;
-    if (items > 0x7fffffffLL) return AQ_ERR_UNSUPPORTED;   // item indices are 32-bit
-    // One CTA per SM at most. Two ways to share the items: whole shares of single units
-    // (cpu CTAs per unit, one table build each), or an even split of all items over the SMs,
-    // where a CTA may straddle units and build two or more tables. Every call waits for its
-    // slowest CTA, so the choice takes the smaller worst-CTA cost, one table build being worth
-    // kTableItems row blocks of streaming (about 0.8 us against 23 ns per 1 KiB block at the
-    // per-SM share of HBM bandwidth).
+    if (aq_status e = prepare(kern, smem, kLutThreads, m * nsets, &occ); e != AQ_OK) return e;
+    LutLayers L = {};
+    L.n = n;
+    long long items = 0;
+    for (int l = 0; l < n; ++l) {
+        L.planes[l] = (const uint8_t*)as[l].planes;
+        L.books[l] = (const uint16_t*)as[l].books;
+        L.partials[l] = as[l].partials;
+        L.plane_bytes[l] = ds[l].plane_bytes;
+        L.rows_pad[l] = ds[l].rows_pad;
+        L.RBc[l] = ds[l].RBc;
+        L.base[l] = (int)items;
+        items += (long long)ds[l].S * m * ds[l].RBc;
+        if (items > 0x7fffffffLL) return AQ_ERR_UNSUPPORTED;   // item indices are 32-bit
+    }
+    L.base[n] = (int)items;
+    const Dims& d = ds[0];
+    const long long units = (long long)d.S * m;       // (slice, book) pairs of one layer
+    // One CTA per SM at most. Two ways to share the items of a single layer: whole shares of
+    // single units (cpu CTAs per unit, one table build each), or an even split of all items
+    // over the SMs, where a CTA may straddle units and build two or more tables. Every call
+    // waits for its slowest CTA, so the choice takes the smaller worst-CTA cost, one table
+    // build being worth kTableItems row blocks of streaming (about 0.8 us against 23 ns per
+    // 1 KiB block at the per-SM share of HBM bandwidth). A group always takes the even split.
     constexpr long long kTableItems = 35;
-    long long cpu = di.sms / units;
+    long long cpu = n == 1 ? di.sms / units : 0;
     if (cpu > d.RBc) cpu = d.RBc;
     long long cost_cpu = -1;
     if (cpu >= 1) cost_cpu = kTableItems + (d.RBc + cpu - 1) / cpu;
     const long long grid_b = items < di.sms ? items : di.sms;
     const long long qb = items / grid_b, rb = items % grid_b;
     long long cost_b = 0;
-    for (long long b = 0; b < grid_b; ++b) {
-        const long long i0 = b * qb + (b < rb ? b : rb), i1 = i0 + qb + (b < rb ? 1 : 0);
-        const long long tables = (i1 - 1) / d.RBc - i0 / d.RBc + 1;
-        const long long c = tables * kTableItems + (i1 - i0);
-        if (c > cost_b) cost_b = c;
-    }
+    if (n == 1)
+        for (long long b = 0; b < grid_b; ++b) {
+            const long long i0 = b * qb + (b < rb ? b : rb), i1 = i0 + qb + (b < rb ? 1 : 0);
+            const long long tables = (i1 - 1) / d.RBc - i0 / d.RBc + 1;
+            const long long c = tables * kTableItems + (i1 - i0);
+            if (c > cost_b) cost_b = c;
+        }
+    else
+        for (int l = 0; l < n; ++l)   // a CTA (at most qb + 1 items) then meets at most two layers
+            if ((long long)ds[l].S * m * ds[l].RBc < qb + 1) return AQ_ERR_UNSUPPORTED;
     int grid, q, r;   // a CTA's share: q items, one more for the first r shares
     if (cost_cpu >= 0 && cost_cpu <= cost_b) {
         grid = (int)(cpu * units);
@@ -1226,10 +1306,14 @@ aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
         q = (int)qb;
         r = (int)rb;
     }
-    return launch_pdl(kern, dim3(grid), dim3(kLutThreads), smem, st, (const uint8_t*)a.planes,
-                      (const uint16_t*)a.books, (const uint16_t*)a.x, a.partials, a.status, m,
-                      d.in, d.ng, d.rows_pad, d.RBc, d.plane_bytes, nslots, (int)cpu, q, r,
-                      (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0, a.batch);
+    return launch_pdl(kern, dim3(grid), dim3(kLutThreads), smem, st, L, (const uint16_t*)as[0].x,
+                      as[0].status, m, d.in, d.ng, nslots, (int)cpu, q, r,
+                      (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0, as[0].batch);
+}
+
+template <int BDT, int XDT, int NT>
+aq_status run_lut(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
+    return run_lut_layers<BDT, XDT, NT>(&d, &a, 1, m, st);
 }
 
 // One pass of gemv_lut8 over tokens [t_base, t_base + 8): the work split of run_lut.
@@ -1449,20 +1533,37 @@ static aq_status launch_product(const Dims& d, int m, const void* planes, const 
 
 // P partial planes per token: one per (slice, book) for the LUT kernel, one per slice for the
 // direct kernel.
+// The reduction of n layers (P partial planes per row and token in each), one launch.
 template <int SDT>
-static aq_status launch_reduce(const Dims& d, int P, const GemvArgs& a, const void* y_prev,
-                               cudaStream_t st) {
+static aq_status launch_reduce_layers(const Dims* ds, const GemvArgs* as, int n, int P,
+                                      const void* y_prev, int static_weights, cudaStream_t st) {
     int occ = 0;
-    if (aq_status e = prepare(splitk_reduce_kernel<SDT>, 0, 256, 0, &occ); e != AQ_OK) return e;
+    auto kern = n > 1 ? splitk_reduce_kernel<SDT, true> : splitk_reduce_kernel<SDT, false>;
+    if (aq_status e = prepare(kern, 0, 256, 0, &occ); e != AQ_OK) return e;
     // Warps per 32-row group: one while a warp's sixteen loads cover the planes (no shared
     // memory step, a small grid), else eight (measured: 1 at P = 16, 8 at P >= 32 are the
     // fastest choices on the layer shapes of the benchmark).
     const int wpr = P <= 16 ? 1 : 8;
     const int rows_per_cta = 256 / wpr;
-    return launch_pdl(splitk_reduce_kernel<SDT>, dim3((d.out + rows_per_cta - 1) / rows_per_cta, a.batch),
-                      dim3(256), 0, st, (const float*)a.partials, (const uint16_t*)a.scales, a.y,
-                      a.y_dt, d.out, d.rows_pad, P, a.batch, wpr,
-                      (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0, y_prev);
+    ReduceLayers R = {};
+    int out_max = 0;
+    for (int l = 0; l < n; ++l) {
+        R.partials[l] = as[l].partials;
+        R.scales[l] = (const uint16_t*)as[l].scales;
+        R.y[l] = as[l].y;
+        R.out[l] = ds[l].out;
+        R.rows_pad[l] = ds[l].rows_pad;
+        if (ds[l].out > out_max) out_max = ds[l].out;
+    }
+    return launch_pdl(kern, dim3((out_max + rows_per_cta - 1) / rows_per_cta, as[0].batch, n), dim3(256), 0,
+                      st, R, as[0].y_dt, P, as[0].batch, wpr, static_weights, y_prev);
+}
+
+template <int SDT>
+static aq_status launch_reduce(const Dims& d, int P, const GemvArgs& a, const void* y_prev,
+                               cudaStream_t st) {
+    return launch_reduce_layers<SDT>(&d, &a, 1, P, y_prev,
+                                     (d.flags & AQ_LAYOUT_STATIC_WEIGHTS) ? 1 : 0, st);
 }
 
 aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* books,
@@ -1479,6 +1580,56 @@ aq_status launch_gemv(const Dims& d, int m, const void* planes, const void* book
     const int P = uses_lut(d, m, batch) ? d.S * m : d.S;
     return d.scale_dt == AQ_BF16 ? launch_reduce<AQ_BF16>(d, P, a, y_prev, st)
                                  : launch_reduce<AQ_F16>(d, P, a, y_prev, st);
+}
+
+// aq_gemv_group: n layers that share the activations x. ws[l] is layer l's workspace region
+// (status word and partial planes, laid out as for aq_gemv). At batch 1 with 2^8-entry books
+// the n products are one launch of the table-lookup kernel (the items of all layers in one
+// numbering) and the n reductions one launch; otherwise, or when a CTA's items would reach
+// into more than two layers, the layers run as n ordinary calls. Either way each layer's
+// partial sums and their order are those of its own call, so the results are identical.
+aq_status launch_gemv_group(const Dims* ds, int n, int m, const void* const* planes,
+                            const void* const* books, const void* const* scales, const void* x,
+                            int x_dt, int batch, void* const* y, int y_dt, void* const* ws,
+                            cudaStream_t st) {
+    if (batch == 0) return AQ_OK;
+    bool any_rows = false;
+    for (int l = 0; l < n; ++l) any_rows |= ds[l].out > 0;
+    if (!any_rows) return AQ_OK;
+    bool fused = n >= 2 && batch == 1 && uses_lut(ds[0], m, 1);
+    for (int l = 0; l < n && fused; ++l) fused = ds[l].out > 0;
+    if (fused) {
+        Dims dd[kGroupMax];
+        GemvArgs as[kGroupMax];
+        int flags = AQ_LAYOUT_STATIC_WEIGHTS;
+        for (int l = 0; l < n; ++l) {
+            dd[l] = ds[l];
+            flags &= ds[l].flags;
+            as[l] = GemvArgs{planes[l], books[l], scales[l], x, x_dt, batch, y[l], y_dt,
+                             (float*)((char*)ws[l] + ws_partial_offset(ds[l])), (unsigned int*)ws[0]};
+        }
+        dd[0].flags = flags;   // prefetch before the grid wait only if every layer's weights are static
+        const int bb = ds[0].book_dt == AQ_BF16, xb = x_dt == AQ_BF16;
+        aq_status e;
+        switch (bb * 2 + xb) {
+            case 0: e = run_lut_layers<AQ_F16, AQ_F16, 1>(dd, as, n, m, st); break;
+            case 1: e = run_lut_layers<AQ_F16, AQ_BF16, 1>(dd, as, n, m, st); break;
+            case 2: e = run_lut_layers<AQ_BF16, AQ_F16, 1>(dd, as, n, m, st); break;
+            default: e = run_lut_layers<AQ_BF16, AQ_BF16, 1>(dd, as, n, m, st); break;
+        }
+        if (e == AQ_OK) {
+            const int P = ds[0].S * m, sw = flags ? 1 : 0;
+            return ds[0].scale_dt == AQ_BF16 ? launch_reduce_layers<AQ_BF16>(dd, as, n, P, nullptr, sw, st)
+                                             : launch_reduce_layers<AQ_F16>(dd, as, n, P, nullptr, sw, st);
+        }
+        if (e != AQ_ERR_UNSUPPORTED) return e;   // nothing was launched for UNSUPPORTED
+    }
+    for (int l = 0; l < n; ++l)
+        if (aq_status e = launch_gemv(ds[l], m, planes[l], books[l], scales[l], x, x_dt, batch, y[l],
+                                      y_dt, ws[l], st, nullptr);
+            e != AQ_OK)
+            return e;
+    return AQ_OK;
 }
 
 }  // namespace aq

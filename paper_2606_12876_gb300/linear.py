@@ -12,7 +12,7 @@ import numpy as np
 import torch
 
 from . import (AQ_BF16, AQ_F16, AQ_F32, AQ_LAYOUT_STATIC_WEIGHTS, DTYPES, TORCH_DTYPES, Layout,
-               aq_decode, aq_gemm,
+               aq_decode, aq_gemm, aq_gemv_group, gemv_group_workspace_bytes,
                aq_gemv, aq_gemv_refine, aq_pack, aq_store_books, aq_store_create, aq_wmse,
                wmse_workspace_bytes, aq_workspace_init,
                aq_store_device_bytes, aq_store_planes, aq_store_scales, aq_store_set_prefix,
@@ -228,6 +228,31 @@ class AQLinear:
 
     def __call__(self, x, m):
         return self.gemv(x, m) if x.shape[0] <= 16 else self.gemm(x, m)
+
+
+_group_ws = {}
+
+
+def gemv_group(layers, x, m, ys=None, y_dtype=None):
+    """y_l = x W_m,l^T for AQLinear layers that share the input x (aq_gemv_group: one product
+    and one reduction launch at batch 1); returns the list of outputs."""
+    xd = _dtype_code(x.dtype)
+    yd = xd if y_dtype is None else y_dtype
+    batch = x.shape[0]
+    dev = layers[0].device
+    for lin in layers:
+        lin._check_m(m)
+    if ys is None:
+        ys = [torch.empty(batch, lin.out, dtype=TORCH_DTYPES[yd], device=dev) for lin in layers]
+    layouts = [lin.layout for lin in layers]
+    key = (tuple((lin.out, lin.inp, lin.M, lin.B) for lin in layers), batch, _stream(None), str(dev))
+    ws = _group_ws.get(key)
+    if ws is None:
+        ws = workspace(gemv_group_workspace_bytes(layouts, batch), dev)
+        _group_ws[key] = ws
+    aq_gemv_group(layouts, m, [lin.planes for lin in layers], [lin.books for lin in layers],
+                  [lin.scales for lin in layers], x, xd, batch, ys, yd, ws)
+    return ys
 
 
 def _dtype_code(dt):

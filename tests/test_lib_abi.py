@@ -241,3 +241,27 @@ def test_gemv_workspace_follows_the_kernel_choice():
     small = aq.Layout.make(300, 1032, 4)           # 5 slices x 4 books x 10 row blocks
     assert aq.gemv_workspace_bytes(small, 8) == 256 + 5 * 8 * 320 * 4
     assert aq.gemv_workspace_bytes(big, 16) == 256 + 33 * 16 * 1024 * 4
+
+
+def test_gemv_group_workspace_and_argument_errors_on_the_host():
+    """aq_gemv_group: the workspace is the layers' aq_gemv workspaces one after the other, each
+    rounded up to 256 bytes; host-side argument errors launch nothing."""
+    Ls = [aq.Layout.make(4096, 4096, 4), aq.Layout.make(1024, 4096, 4), aq.Layout.make(1000, 4096, 2)]
+    want = sum((aq.gemv_workspace_bytes(L, 1) + 255) // 256 * 256 for L in Ls)
+    assert aq.gemv_group_workspace_bytes(Ls, 1) == want
+    lib = aq.lib()
+    vp = ctypes.c_void_p
+    arr3 = (aq.Layout * 3)(*Ls)
+    ptrs = (vp * 3)(FAKE, FAKE, FAKE)
+    args = lambda n, layouts, m=1: (n, layouts, m, ptrs, ptrs, ptrs, FAKE, aq.AQ_F16, 1, ptrs,
+                                    aq.AQ_F16, FAKE, 1 << 30, None)
+    assert lib.aq_gemv_group(*args(0, arr3)) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_gemv_group(*args(5, (aq.Layout * 5)(*(Ls + Ls[:2])))) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_gemv_group(*args(3, arr3, m=3)) == aq.AQ_ERR_INVALID_ARG      # m > M of layer 2
+    other = (aq.Layout * 2)(Ls[0], aq.Layout.make(1024, 2048, 4))               # in differs
+    assert lib.aq_gemv_group(*args(2, other)) == aq.AQ_ERR_INVALID_ARG
+    bf = (aq.Layout * 2)(Ls[0], aq.Layout.make(1024, 4096, 4, book_dtype="bf16"))
+    assert lib.aq_gemv_group(*args(2, bf)) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_gemv_group(3, arr3, 1, None, ptrs, ptrs, FAKE, aq.AQ_F16, 1, ptrs, aq.AQ_F16,
+                             FAKE, 1 << 30, None) == aq.AQ_ERR_INVALID_ARG
+    assert lib.aq_gemv_group(*(args(3, arr3)[:11] + (FAKE, 16, None))) == aq.AQ_ERR_WORKSPACE
