@@ -825,7 +825,7 @@ gemv_direct_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restric
                 const uint32_t code = unit_code<B>(codes_s + ((size_t)k * 32 + lane) * UNIT, p);
                 uint4 cwv;
                 if constexpr (B <= 8) cwv = ((const uint4*)books_s)[(k << B) + code];
-                else cwv = __ldg((const uint4*)books + ((size_t)k << 16) + code);
+                else cwv = ld_stream_v4((const uint4*)books + ((size_t)k << 16) + code);
                 float c[8];
                 unpack8<BDT>(cwv, c);
 #pragma unroll
@@ -997,6 +997,84 @@ gemv_mma_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__
                     p0[rows_pad + 8] = acc[mt][nt][3];
                 }
             }
+    }
+}
+
+// ------------------------------------------------------------------ 2^16-entry books, one token
+//
+// gemv_gather16 (B = 16, 1 token, m <= 2): the codewords come from 1 MiB books read through L2,
+// so the kernel is bound by the number of random 16-byte gathers in flight. Lane L owns row
+// 32*rb + L of a slice; its 32 codes per book (64 bytes, position p holding group
+// (p + L) mod 32) are loaded into registers, then for every eight positions the lane issues all
+// 8*m codeword gathers (not allocated in L1: the hit rate there is nil) before it adds and
+// multiplies any of them. Activations are staged per slice in shared memory as fp32 and read
+// per lane (group (p + L) mod 32). Partials per (slice, row) as gemv_direct.
+constexpr int kG16Warps = 8;
+
+template <int BDT, int XDT, int MB>
+__global__ void __launch_bounds__(kG16Warps * 32)
+gemv_gather16_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
+                     const uint16_t* __restrict__ x, float* __restrict__ partials, int in,
+                     int rows_pad, int RBc, int rb_per_chunk, size_t plane_bytes) {
+    __shared__ __align__(16) float xs[256];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int s = blockIdx.y, chunk = blockIdx.x;
+    const int rb0 = chunk * rb_per_chunk, rb1 = min(rb0 + rb_per_chunk, RBc);
+    pdl_wait();
+    pdl_launch_dependents();
+    for (int i = tid; i < 256; i += kG16Warps * 32) {
+        const int col = s * 256 + i;
+        xs[i] = col < in ? bits_to_f32<XDT>(x[col]) : 0.0f;
+    }
+    __syncthreads();
+    for (int rb = rb0 + warp; rb < rb1; rb += kG16Warps) {
+        const int o = rb * 32 + lane;
+        uint4 cr[MB][4];                          // 32 codes per book, 8 per uint4
+#pragma unroll
+        for (int k = 0; k < MB; ++k) {
+            const uint4* src = (const uint4*)(planes + (size_t)k * plane_bytes + ((size_t)s * rows_pad + o) * 64);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) cr[k][q] = ld_stream_v4(src + q);
+        }
+        float acc = 0.0f;
+#pragma unroll
+        for (int p0 = 0; p0 < 32; p0 += 8) {
+            uint4 cw[MB][8];
+#pragma unroll
+            for (int k = 0; k < MB; ++k) {
+                const uint4 w4 = cr[k][p0 >> 3];
+                const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const uint32_t code = (wv[i >> 1] >> (16 * (i & 1))) & 0xffffu;
+                    cw[k][i] = ld_stream_v4((const uint4*)books + ((size_t)k << 16) + code);
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int g = (p0 + i + lane) & 31;
+                const float4 x0 = *(const float4*)(xs + g * 8);
+                const float4 x1 = *(const float4*)(xs + g * 8 + 4);
+                float w[8];
+                unpack8<BDT>(cw[0][i], w);
+#pragma unroll
+                for (int k = 1; k < MB; ++k) {
+                    float c[8];
+                    unpack8<BDT>(cw[k][i], c);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) w[e] += c[e];
+                }
+                acc = fmaf(x0.x, w[0], acc);
+                acc = fmaf(x0.y, w[1], acc);
+                acc = fmaf(x0.z, w[2], acc);
+                acc = fmaf(x0.w, w[3], acc);
+                acc = fmaf(x1.x, w[4], acc);
+                acc = fmaf(x1.y, w[5], acc);
+                acc = fmaf(x1.z, w[6], acc);
+                acc = fmaf(x1.w, w[7], acc);
+            }
+        }
+        partials[(size_t)s * rows_pad + o] = acc;
     }
 }
 
@@ -1390,6 +1468,23 @@ aq_status run_direct(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
                       a.partials, m, a.batch, d.in, d.rows_pad, d.RBc, rbpc, d.plane_bytes);
 }
 
+template <int BDT, int XDT, int MB>
+aq_status run_gather16(const Dims& d, const GemvArgs& a, cudaStream_t st) {
+    DeviceInfo di;
+    if (aq_status e = device_info(&di); e != AQ_OK) return e;
+    auto kern = gemv_gather16_kernel<BDT, XDT, MB>;
+    int occ = 0;
+    if (aq_status e = prepare(kern, 0, kG16Warps * 32, MB, &occ); e != AQ_OK) return e;
+    const int target = di.sms * occ;
+    int chunks = (target + d.S - 1) / d.S;
+    chunks = chunks < 1 ? 1 : (chunks > d.RBc ? d.RBc : chunks);
+    const int rbpc = (d.RBc + chunks - 1) / chunks;
+    chunks = (d.RBc + rbpc - 1) / rbpc;
+    return launch_pdl(kern, dim3(chunks, d.S), dim3(kG16Warps * 32), 0, st,
+                      (const uint8_t*)a.planes, (const uint16_t*)a.books, (const uint16_t*)a.x,
+                      a.partials, d.in, d.rows_pad, d.RBc, rbpc, d.plane_bytes);
+}
+
 template <int NT, int BDT, int MB>
 aq_status run_mma(const Dims& d, const GemvArgs& a, cudaStream_t st) {
     DeviceInfo di;
@@ -1429,6 +1524,13 @@ aq_status dispatch_mma(const Dims& d, int m, const GemvArgs& a, cudaStream_t st)
 
 template <int B, int BDT, int SDT>
 aq_status dispatch_direct(const Dims& d, int m, const GemvArgs& a, cudaStream_t st) {
+    if constexpr (B == 16) {
+        if (a.batch == 1 && m <= 2) {   // 2^16-entry books, one token: gathers in flight
+            const bool xb = a.x_dt == AQ_BF16;
+            if (m == 1) return xb ? run_gather16<BDT, AQ_BF16, 1>(d, a, st) : run_gather16<BDT, AQ_F16, 1>(d, a, st);
+            return xb ? run_gather16<BDT, AQ_BF16, 2>(d, a, st) : run_gather16<BDT, AQ_F16, 2>(d, a, st);
+        }
+    }
     if (a.batch <= 1) return run_direct<1, B, BDT, SDT>(d, m, a, st);
     if (a.batch <= 2) return run_direct<2, B, BDT, SDT>(d, m, a, st);
     if (a.batch <= 4) return run_direct<4, B, BDT, SDT>(d, m, a, st);
