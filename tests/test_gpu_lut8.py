@@ -92,3 +92,17 @@ def test_lut8_exact():
         ref = oracle.product_exact(layer, x_bits, "bf16", m)
         for b in (5, 6, 7, 8):
             assert_exact(lin.gemv(x[:b], m, y_dtype=aq.AQ_F32), ref[:b], "m=%d batch=%d" % (m, b))
+
+
+def test_lut8_refinement_chain_exact():
+    """aq_gemv_refine at 8 tokens on a layer of 9216 rows x 4096 inputs: every step's one-book
+    view has 16 x 288 = 4608 items, so each refinement runs the eight-token table kernel; the
+    chain m = 1..4 (fp32, in place) equals each prefix product bit for bit."""
+    layer = exact_layer(9216, 4096, 4, 8, "f16", seed=13)
+    lin = AQLinear.from_layer(layer)
+    x_bits = exact_x(8, 4096, "f16", seed=14)
+    x = x_to_device(x_bits, "f16")
+    y = None
+    for m in range(1, 5):
+        y = lin.refine(x, m, y, y=y)
+        assert_exact(y, oracle.product_exact(layer, x_bits, "f16", m), "refine to m=%d" % m)
