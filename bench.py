@@ -554,41 +554,44 @@ def measure_configs(dev, stream, hbm_peak, sm_mhz):
                 e["frac_alu"] = round(tf / alu_peak, 4)
             rows.append(e)
         res["llama8b_block"]["block_sum_b%d" % b] = rows
-        if b == 1:
-            # the same seven layers as four calls: q/k/v and gate/up each as one group call
-            # (aq_gemv_group), o and down alone
-            from paper_2606_12876_gb300.linear import gemv_group
-            names = [n for n, _ in blk]
-            idx = {n: j for j, n in enumerate(names)}
-            groups = [("q_proj", "k_proj", "v_proj"), ("o_proj",), ("gate_proj", "up_proj"),
-                      ("down_proj",)]
-            gws = {}
-            for gr in groups:
-                if len(gr) > 1:
-                    gws[gr] = aq.workspace(aq.gemv_group_workspace_bytes(
-                        [blk[idx[n]][1].layout for n in gr], b), dev)
-            grows = []
-            for m in (1, 2, 3, 4):
-                def gstep(i, m=m):
-                    for gr in groups:
-                        js = [idx[n] for n in gr]
-                        lins = [blk[j][1] for j in js]
-                        if len(gr) == 1:
-                            j = js[0]
-                            aq.aq_gemv(lins[0].layout, m, cps[j][i % 3], lins[0].books,
-                                       lins[0].scales, xs[lins[0].inp], aq.AQ_BF16, b, ys[j],
-                                       aq.AQ_BF16, wss[j])
-                        else:
-                            aq.aq_gemv_group([l.layout for l in lins], m, [cps[j][i % 3] for j in js],
-                                             [l.books for l in lins], [l.scales for l in lins],
-                                             xs[lins[0].inp], aq.AQ_BF16, b, [ys[j] for j in js],
-                                             aq.AQ_BF16, gws[gr])
-                with torch.cuda.stream(stream):
-                    us = graph_us(gstep, 10, stream)
-                nb = sum(layer_bytes(lin.out, lin.inp, m, batch=b) for _, lin in blk)
-                grows.append({"m": m, "us": round(us, 3), "GB_s": round(nb / us / 1e3, 1),
-                              "frac_hbm": round(nb / us / 1e3 / hbm_peak, 4)})
-            res["llama8b_block"]["block_grouped_b1"] = grows
+        # the same seven layers as four calls: q/k/v and gate/up each as one group call
+        # (aq_gemv_group), o and down alone
+        names = [n for n, _ in blk]
+        idx = {n: j for j, n in enumerate(names)}
+        groups = [("q_proj", "k_proj", "v_proj"), ("o_proj",), ("gate_proj", "up_proj"),
+                  ("down_proj",)]
+        gws = {}
+        for gr in groups:
+            if len(gr) > 1:
+                gws[gr] = aq.workspace(aq.gemv_group_workspace_bytes(
+                    [blk[idx[n]][1].layout for n in gr], b), dev)
+        grows = []
+        for m in (1, 2, 3, 4):
+            def gstep(i, m=m):
+                for gr in groups:
+                    js = [idx[n] for n in gr]
+                    lins = [blk[j][1] for j in js]
+                    if len(gr) == 1:
+                        j = js[0]
+                        aq.aq_gemv(lins[0].layout, m, cps[j][i % 3], lins[0].books,
+                                   lins[0].scales, xs[lins[0].inp], aq.AQ_BF16, b, ys[j],
+                                   aq.AQ_BF16, wss[j])
+                    else:
+                        aq.aq_gemv_group([l.layout for l in lins], m, [cps[j][i % 3] for j in js],
+                                         [l.books for l in lins], [l.scales for l in lins],
+                                         xs[lins[0].inp], aq.AQ_BF16, b, [ys[j] for j in js],
+                                         aq.AQ_BF16, gws[gr])
+            with torch.cuda.stream(stream):
+                us = graph_us(gstep, 10, stream)
+            nb = sum(layer_bytes(lin.out, lin.inp, m, batch=b) for _, lin in blk)
+            ge = {"m": m, "us": round(us, 3), "GB_s": round(nb / us / 1e3, 1),
+                  "frac_hbm": round(nb / us / 1e3 / hbm_peak, 4)}
+            if b > 1:
+                tf = 2.0 * b * sum(lin.out * lin.inp for _, lin in blk) / (us * 1e-6) / 1e12
+                ge["TFLOP_s"] = round(tf, 2)
+                ge["frac_alu"] = round(tf / alu_peak, 4)
+            grows.append(ge)
+        res["llama8b_block"]["block_grouped_b%d" % b] = grows
         del cps
     del blk
     (_, linb), = cfg_layers("big_book_8192")
