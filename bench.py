@@ -273,9 +273,16 @@ def measure_gemm(dev, stream, peaks, reps=5, tokens=4096):
         tf = flops / (ms * 1e-3) / 1e12
         rows.append({"m": m, "ms": round(ms, 4), "TFLOP_s": round(tf, 1),
                      "frac_bf16_peak": round(tf / peak, 4)})
-    wd = torch.randn(out, inp, device=dev, dtype=torch.bfloat16)
+    wd = torch.empty(out, inp, device=dev, dtype=torch.bfloat16)
+    # the unfused yardstick: W_m decoded alone (aq_decode into a dense bf16 matrix), then a
+    # dense bf16 product of the same shape
+    for e in rows:
+        e["decode_ms"] = round(timed(lambda: lin.decode(e["m"], out=wd)), 4)
+    torch.nn.init.normal_(wd)
     dense_ms = timed(lambda: torch.matmul(x, wd.t()))
     del wd
+    for e in rows:
+        e["decode_plus_dense_ms"] = round(e["decode_ms"] + dense_ms, 4)
     return {"workload": name, "tokens": tokens, "out": out, "in": inp, "M": 4,
             "compute": "fp16 tcgen05 pair MMA, fp32 accumulation; weights decoded in shared memory (m = 1), or W_m decoded once in fp16 and loaded by TMA (m >= 2 at 2048+ tokens)",
             "per_m": rows, "dense_bf16_torch_ms": round(dense_ms, 4),

@@ -758,73 +758,131 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
 
 // W16[o][i] = fp16(sum_{k<m} C_k[b_k[o, i/8]][i mod 8]): the unscaled fp32 sum of the m
 // codewords in book order, rounded once to fp16 (the values the GEMM's decoders write; the
-// epilogue applies the row scale). Each warp owns one 32-row block of one 256-input slice:
-// lane L stages its row's codes of the m planes, then the warp walks the 32 rows with lane L
-// producing group s*32 + L, so every store is 512 contiguous bytes.
+// epilogue applies the row scale).
+// One CTA per SM walks the (32-row block, 256-input slice) items, a warp at a time
+// (grid-stride; row blocks fastest, so a warp's code loads are one contiguous 1 KiB per plane
+// and its stores 512 contiguous bytes per row). The CTA stages the first m codebooks once, in
+// 2^cshift interleaved copies: copy c of codeword j at 16-byte slot j * 2^cshift + c, read by
+// the lanes L with L mod 2^cshift = c. With eight copies the eight lanes of each quarter-warp
+// phase of a 16-byte load reach eight different bank groups whatever their codes, so the
+// gathers are free of bank conflicts (with one copy random codes cost about 2.4 times the
+// conflict-free wavefronts); fewer copies where m books would not fit eight times. Each lane
+// copies its row's codes of the m planes into the warp's staging buffer (cp.async, 16 bytes
+// at a time), the next item's while the current one is decoded; then lane L walks the 32 rows
+// producing group s*32 + L of each.
 constexpr int kDenseWarps = 8;
 
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// Interleaved copies of the staged codebooks (log2) for code width B and prefix m: as many as
+// fit the shared-memory map (eight at most).
+inline int dense_w_cshift(int B, int m) {
+    if (B <= 4) return 3;
+    return m <= 4 ? 3 : m <= 6 ? 2 : 1;
+}
+inline size_t dense_w_smem(int B, int m) {
+    return (size_t)m * ((size_t)16 << B << dense_w_cshift(B, m)) +
+           (size_t)kDenseWarps * 2 * m * 32 * unit_bytes(B);
+}
+
 template <int B, int BDT>
-__global__ void __launch_bounds__(kDenseWarps * 32)
+__global__ void __launch_bounds__(kDenseWarps * 32, 1)
 dense_w_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
-               uint16_t* __restrict__ w16, float* __restrict__ wfac_out, int m, int out, int in,
-               int ng, int rows_pad, int RBc, size_t plane_bytes) {
+               uint16_t* __restrict__ w16, float* __restrict__ wfac_out, int m, int cshift, int out,
+               int in, int ng, int rows_pad, int RBc, int S, size_t plane_bytes) {
     constexpr int UNIT = unit_bytes(B);
+    constexpr int NC = 1 << B;
     extern __shared__ __align__(16) unsigned char smem_d[];
-    uint4* books_s = (uint4*)smem_d;                 // [m][2^B] codewords
+    uint4* books_s = (uint4*)smem_d;                 // [m][NC][2^cshift] codewords
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    unsigned char* codes_s = smem_d + staged_books_bytes(B, m) + (size_t)warp * m * 32 * UNIT;
+    // this warp's code buffers: [2][m][32 rows][UNIT]
+    unsigned char* cbuf = smem_d + ((size_t)m * NC << cshift) * 16 + (size_t)warp * 2 * m * 32 * UNIT;
     __shared__ unsigned int wmax[8];
+    const long long items = (long long)RBc * S;
+    const long long stride = (long long)gridDim.x * kDenseWarps;
+    auto issue = [&](long long item, int buf) {   // the item's codes into buffer buf
+        if (item < items) {
+            const int s = (int)(item / RBc), rb = (int)(item - (long long)s * RBc);
+            const size_t src = ((size_t)s * rows_pad + (size_t)rb * 32 + lane) * UNIT;
+            unsigned char* dst = cbuf + ((size_t)buf * m * 32 + lane) * UNIT;
+            for (int k = 0; k < m; ++k)
+#pragma unroll
+                for (int q = 0; q < UNIT / 16; ++q)
+                    cp_async16(dst + (size_t)k * 32 * UNIT + q * 16, planes + k * plane_bytes + src + q * 16);
+        }
+        cp_async_commit();
+    };
     pdl_wait();
     pdl_launch_dependents();
+    long long item = (long long)blockIdx.x * kDenseWarps + warp;
+    issue(item, 0);   // the first codes travel while the books are staged
     // Books staged times 2^-f (fp16 range, as in the GEMM's decoders); 2^f goes to the
     // workspace for the GEMM's epilogue (every CTA finds the same f; CTA 0 writes it).
     if (threadIdx.x < 8) wmax[threadIdx.x] = 0u;
     __syncthreads();
-    for (int i = threadIdx.x; i < (m << B); i += blockDim.x) {
-        const uint4 c = __ldg((const uint4*)books + i);
-        atomicMax(&wmax[i >> B], codeword_max_bits<BDT>(c));
-        books_s[i] = c;
-    }
+    for (int i = threadIdx.x; i < m * NC; i += blockDim.x)
+        atomicMax(&wmax[i >> B], codeword_max_bits<BDT>(__ldg((const uint4*)books + i)));
     __syncthreads();
     const int f = book_exponent<BDT>(wmax, m);
-    if (f)
-        for (int i = threadIdx.x; i < (m << B); i += blockDim.x) books_s[i] = scale_codeword<BDT>(books_s[i], pow2f(-f));
-    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *wfac_out = pow2f(f);
-    const int s = blockIdx.y;
-    const int rb = blockIdx.x * kDenseWarps + warp;
-    const bool active = rb < RBc;
-    if (active) {
-        const int o = rb * 32 + lane;
-        for (int k = 0; k < m; ++k) {
-            const uint4* src = (const uint4*)(planes + k * plane_bytes + ((size_t)s * rows_pad + o) * UNIT);
-            uint4* dst = (uint4*)(codes_s + ((size_t)k * 32 + lane) * UNIT);
-#pragma unroll
-            for (int q = 0; q < UNIT / 16; ++q) dst[q] = ld_stream_v4(src + q);
-        }
+    for (int i = threadIdx.x; i < (m * NC) << cshift; i += blockDim.x) {
+        const uint4 c = __ldg((const uint4*)books + (i >> cshift));
+        books_s[i] = f ? scale_codeword<BDT>(c, pow2f(-f)) : c;
     }
+    if (blockIdx.x == 0 && threadIdx.x == 0) *wfac_out = pow2f(f);
     __syncthreads();
-    const int g = s * 32 + lane;
-    if (!active || g >= ng) return;
-    const uint32_t books_u = smem_u32(books_s);
-    for (int r = 0; r < 32; ++r) {
-        const int o = rb * 32 + r;
-        if (o >= out) break;
-        const int p = (lane - r) & 31;               // position of group `lane` in row o
-        float a[8];
+    const uint32_t books_u = smem_u32(books_s) + ((uint32_t)(lane & ((1 << cshift) - 1)) << 4);
+    int buf = 0;
+    for (; item < items; item += stride) {
+        issue(item + stride, buf ^ 1);
+        cp_async_wait<1>();      // this lane's copies of the current item landed
+        __syncwarp();            // ... and every lane's
+        const int s = (int)(item / RBc), rb = (int)(item - (long long)s * RBc);
+        const int g = s * 32 + lane;
+        const unsigned char* cb = cbuf + (size_t)buf * m * 32 * UNIT;
+        if (g < ng) {
+            // four rows at a time: four independent gathers per book in flight
+            for (int r0 = 0; r0 < 32 && rb * 32 + r0 < out; r0 += 4) {
+                float a[4][8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) a[e] = -0.0f;
-        for (int k = 0; k < m; ++k) {
-            const uint32_t code = unit_code<B>(codes_s + ((size_t)k * 32 + r) * UNIT, p);
-            const uint4 c = lds128(books_u + (((uint32_t)k << B) + code) * 16u);
-            add_widen2<BDT>(c.x, a[0], a[1]);
-            add_widen2<BDT>(c.y, a[2], a[3]);
-            add_widen2<BDT>(c.z, a[4], a[5]);
-            add_widen2<BDT>(c.w, a[6], a[7]);
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) a[i][e] = -0.0f;
+                for (int k = 0; k < m; ++k) {
+                    uint4 c[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const int r = r0 + i;
+                        // position of group `lane` in row rb*32 + r
+                        const uint32_t code = unit_code<B>(cb + ((size_t)k * 32 + r) * UNIT, (lane - r) & 31);
+                        c[i] = lds128(books_u + ((((uint32_t)k << B) + code) << (cshift + 4)));
+                    }
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        add_widen2<BDT>(c[i].x, a[i][0], a[i][1]);
+                        add_widen2<BDT>(c[i].y, a[i][2], a[i][3]);
+                        add_widen2<BDT>(c[i].z, a[i][4], a[i][5]);
+                        add_widen2<BDT>(c[i].w, a[i][6], a[i][7]);
+                    }
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int o = rb * 32 + r0 + i;
+                    if (o < out)
+                        *(uint4*)(w16 + (size_t)o * in + (size_t)g * 8) =
+                            make_uint4(f16x2(make_float2(a[i][0], a[i][1])), f16x2(make_float2(a[i][2], a[i][3])),
+                                       f16x2(make_float2(a[i][4], a[i][5])), f16x2(make_float2(a[i][6], a[i][7])));
+                }
+            }
         }
-        *(uint4*)(w16 + (size_t)o * in + (size_t)g * 8) =
-            make_uint4(f16x2(make_float2(a[0], a[1])), f16x2(make_float2(a[2], a[3])),
-                       f16x2(make_float2(a[4], a[5])), f16x2(make_float2(a[6], a[7])));
+        __syncwarp();            // every lane has read the buffer before it is refilled
+        buf ^= 1;
     }
+    cp_async_wait<0>();
 }
 
 template <int B, int BDT>
@@ -832,16 +890,43 @@ aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* b
                          const void* scales, const void* x, const float* xfac, int tokens, void* y,
                          int y_dt, void* ws, uint16_t* w16, cudaStream_t st) {   // x: fp16 [tokens][in]
     {   // decode W_m once
-        const size_t smem = staged_books_bytes(B, m) + (size_t)kDenseWarps * m * 32 * unit_bytes(B);
+        const size_t smem = dense_w_smem(B, m);
         auto kern = dense_w_kernel<B, BDT>;
-        // (the kernel also has a few bytes of static shared memory, so the default 48 KiB
-        // limit on the total is raised already from 32 KiB of dynamic memory)
-        if (smem > 32 * 1024)
-            if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-                e != cudaSuccess)
-                return cuda_fail(e, "cudaFuncSetAttribute");
+        DeviceInfo di;
+        if (aq_status e = device_info(&di); e != AQ_OK) return e;
+        // the kernel's shared-memory limit raised once per device, its occupancy per prefix
+        static std::mutex mu_w;
+        static int occ_cache[64][kGemmMaxM + 1] = {};
+        int dev = 0;
+        if (cudaError_t e = cudaGetDevice(&dev); e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+        if (dev < 0 || dev >= 64 || m < 1 || m > kGemmMaxM) return AQ_ERR_UNSUPPORTED;
+        int occ = 0;
+        {
+            std::lock_guard<std::mutex> lock(mu_w);
+            if (occ_cache[dev][m] == 0) {
+                cudaFuncAttributes fa;
+                if (cudaError_t e = cudaFuncGetAttributes(&fa, kern); e != cudaSuccess)
+                    return cuda_fail(e, "cudaFuncGetAttributes");
+                const int dyn_max = di.smem_optin - (int)fa.sharedSizeBytes;
+                if ((int)smem > dyn_max) return AQ_ERR_UNSUPPORTED;
+                if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn_max);
+                    e != cudaSuccess)
+                    return cuda_fail(e, "cudaFuncSetAttribute");
+                int o = 0;
+                if (cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, kern, kDenseWarps * 32, smem);
+                    e != cudaSuccess)
+                    return cuda_fail(e, "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
+                if (o < 1) return AQ_ERR_UNSUPPORTED;
+                occ_cache[dev][m] = o;
+            }
+            occ = occ_cache[dev][m];
+        }
+        const long long items = (long long)d.RBc * d.S;
+        long long grid = (long long)di.sms * (occ > 0 ? occ : 1);
+        const long long need = (items + kDenseWarps - 1) / kDenseWarps;
+        if (grid > need) grid = need;
         cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3((d.RBc + kDenseWarps - 1) / kDenseWarps, d.S);
+        cfg.gridDim = dim3((unsigned)grid);
         cfg.blockDim = dim3(kDenseWarps * 32);
         cfg.dynamicSmemBytes = smem;
         cfg.stream = st;
@@ -851,8 +936,9 @@ aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* b
         cfg.attrs = attr;
         cfg.numAttrs = 1;
         if (aq_status e = cuda_ok(cudaLaunchKernelEx(&cfg, kern, (const uint8_t*)planes, (const uint16_t*)books,
-                                                     w16, (float*)((char*)ws + kWsWfacOffset), m, d.out,
-                                                     d.in, d.ng, d.rows_pad, d.RBc, d.plane_bytes),
+                                                     w16, (float*)((char*)ws + kWsWfacOffset), m,
+                                                     dense_w_cshift(B, m), d.out, d.in, d.ng, d.rows_pad,
+                                                     d.RBc, d.S, d.plane_bytes),
                                   "cudaLaunchKernelEx (dense W_m)");
             e != AQ_OK)
             return e;
