@@ -68,12 +68,13 @@ constexpr int kBStage = kRows * 128;          // 16 KiB
 // offsets). Up to four books: four activation stages, three weight stages, room for four
 // planes of codes and four codebooks. Longer prefixes need more room for codes and codebooks
 // (MB planes of 128 rows per slice, MB codebooks of 4 KiB): the activation ring drops to three
-// stages, and from seven books the weight ring to two.
-template <int MB>
+// stages, and from seven books the weight ring to two. The dense form has no codes or books in
+// shared memory: four stages of each ring.
+template <int MB, bool DENSE = false>
 struct GemmLayout {
-    static constexpr int kBooks = MB <= 4 ? 4 : MB;
-    static constexpr int kStagesA = MB <= 4 ? 4 : 3;
-    static constexpr int kStagesB = MB <= 6 ? 3 : 2;
+    static constexpr int kBooks = DENSE ? 0 : MB <= 4 ? 4 : MB;
+    static constexpr int kStagesA = DENSE || MB <= 4 ? 4 : 3;
+    static constexpr int kStagesB = DENSE ? 4 : MB <= 6 ? 3 : 2;
     static constexpr int kCodeBuf = kBooks * kRows * 32;   // one slice of codes, all planes
     static constexpr int kOffA = 0;
     static constexpr int kOffB = kOffA + kStagesA * kAStage;
@@ -204,7 +205,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
             const float* __restrict__ xfac, int tokens, int out, int in, int ng, int rows_pad,
             size_t plane_bytes) {
     static_assert(!DENSE || (MB == 1 && NP == 1), "dense tiles: one instantiation");
-    using GL = GemmLayout<MB>;
+    using GL = GemmLayout<MB, DENSE>;
     constexpr int kStagesA = GL::kStagesA, kStagesB = GL::kStagesB, kCodeBuf = GL::kCodeBuf;
     constexpr int kOffA = GL::kOffA, kOffB = GL::kOffB, kOffCodes = GL::kOffCodes;
     extern __shared__ __align__(1024) unsigned char smem[];
@@ -967,7 +968,7 @@ aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* b
             return AQ_ERR_CUDA;
     }
     auto kern = gemm_kernel<BDT, 1, 1, true>;
-    constexpr int smem = GemmLayout<1>::kSmem;
+    constexpr int smem = GemmLayout<1, true>::kSmem;
     static std::mutex mu;
     static bool attr_done[64] = {};
     int dev = 0;
