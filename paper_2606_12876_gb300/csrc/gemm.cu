@@ -65,16 +65,17 @@ constexpr int kBStage = kRows * 128;          // 16 KiB
 
 // Shared-memory map for prefix length MB (offsets from a 1024-byte aligned base; identical in
 // both CTAs of a pair, which the pair MMA relies on: it reads the peer's operands at the same
-// offsets). Up to four books: four activation stages, three weight stages, room for four
-// planes of codes and four codebooks. Longer prefixes need more room for codes and codebooks
-// (MB planes of 128 rows per slice, MB codebooks of 4 KiB): the activation ring drops to three
-// stages, and from seven books the weight ring to two. The dense form has no codes or books in
-// shared memory: four stages of each ring.
+// offsets). One or two books: four activation and four weight stages, room for MB planes of
+// codes and MB codebooks; three or four books: three weight stages, room for four of each.
+// Longer prefixes need more room for codes and codebooks (MB planes of 128 rows per slice, MB
+// codebooks of 4 KiB): the activation ring drops to three stages, and from seven books the
+// weight ring to two. The dense form has no codes or books in shared memory: four stages of
+// each ring.
 template <int MB, bool DENSE = false>
 struct GemmLayout {
-    static constexpr int kBooks = DENSE ? 0 : MB <= 4 ? 4 : MB;
+    static constexpr int kBooks = DENSE ? 0 : MB <= 2 ? MB : MB <= 4 ? 4 : MB;
     static constexpr int kStagesA = DENSE || MB <= 4 ? 4 : 3;
-    static constexpr int kStagesB = DENSE ? 4 : MB <= 6 ? 3 : 2;
+    static constexpr int kStagesB = DENSE || MB <= 2 ? 4 : MB <= 6 ? 3 : 2;
     static constexpr int kCodeBuf = kBooks * kRows * 32;   // one slice of codes, all planes
     static constexpr int kOffA = 0;
     static constexpr int kOffB = kOffA + kStagesA * kAStage;
