@@ -283,6 +283,45 @@ __device__ __forceinline__ void unrotate_codes(const uint32_t (&w)[8], int o, ui
     for (int j = 0; j < 8; ++j) u[j] = rb ? __funnelshift_l(t[(j + 7) & 7], t[j], rb) : t[j];
 }
 
+// Shared-memory accesses through 32-bit shared-window addresses. lds128 is for data that no
+// thread writes while it may be read (codebooks): the compiler may reorder it freely.
+// lds128_ordered stays after the barrier wait that precedes it.
+__device__ __forceinline__ uint4 lds128(uint32_t a) {
+    uint4 v;
+    asm("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ uint4 lds128_ordered(uint32_t a) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a) : "memory");
+    return v;
+}
+__device__ __forceinline__ void sts128(uint32_t a, uint4 v) {
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z),
+                 "r"(v.w)
+                 : "memory");
+}
+
+// 16-byte asynchronous copy global -> shared (cp.async, L2 only), its group commit and wait.
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// Interleaved copies (log2) of staged codebooks for the decoders that write a dense W_m
+// (aq_decode, and the prefill GEMM's dense form): copy c of codeword j at 16-byte slot
+// j * 2^copies + c, read by the lanes L with L mod 2^copies = c. With eight copies the eight
+// lanes of a quarter-warp phase of a 16-byte load reach eight different bank groups whatever
+// their codes; fewer where m books of 2^8 entries would not fit eight times next to the
+// decoders' code buffers.
+inline int book_copies_log2(int B, int m) {
+    if (B <= 4) return 3;
+    return m <= 4 ? 3 : m <= 6 ? 2 : 1;
+}
+
 // Bytes of one (row, slice) unit of a code plane: 32 codes of B bits (B = 4, 8 or 16).
 constexpr int unit_bytes(int B) { return 32 * B / 8; }
 // Bytes of shared memory for the first m codebooks when they are staged there (B <= 8:
@@ -356,6 +395,16 @@ __device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
                        cr = *(unsigned long long*)&c, dr;
     asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(dr) : "l"(ar), "l"(br), "l"(cr));
     return *(float2*)&dr;
+}
+
+// Two fp32 values rounded to nearest-even into a packed pair of 16-bit floats of type DT (low
+// half first): the same per-value rounding as f32_to_bits.
+template <int DT>
+__device__ __forceinline__ uint32_t round_pack2(float lo, float hi) {
+    uint32_t d;
+    if constexpr (DT == AQ_F16) asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+    else asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+    return d;
 }
 
 }  // namespace aq

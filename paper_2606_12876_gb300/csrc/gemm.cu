@@ -764,36 +764,21 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
 // One CTA per SM walks the (32-row block, 256-input slice) items, a warp at a time
 // (grid-stride; row blocks fastest, so a warp's code loads are one contiguous 1 KiB per plane
 // and its stores 512 contiguous bytes per row). The CTA stages the first m codebooks once, in
-// 2^cshift interleaved copies: copy c of codeword j at 16-byte slot j * 2^cshift + c, read by
-// the lanes L with L mod 2^cshift = c. With eight copies the eight lanes of each quarter-warp
-// phase of a 16-byte load reach eight different bank groups whatever their codes, so the
-// gathers are free of bank conflicts (with one copy random codes cost about 2.4 times the
-// conflict-free wavefronts); fewer copies where m books would not fit eight times. Each lane
+// 2^cshift interleaved copies (book_copies_log2), so the gathers are free of bank conflicts
+// with eight copies (with one copy random codes cost about 2.4 times the conflict-free
+// wavefronts). Each lane
 // copies its row's codes of the m planes into the warp's staging buffer (cp.async, 16 bytes
 // at a time), the next item's while the current one is decoded; then lane L walks the 32 rows
 // producing group s*32 + L of each.
-constexpr int kDenseWarps = 8;
+constexpr int kDenseMaxWarps = 16;
 
-__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
-
-// Interleaved copies of the staged codebooks (log2) for code width B and prefix m: as many as
-// fit the shared-memory map (eight at most).
-inline int dense_w_cshift(int B, int m) {
-    if (B <= 4) return 3;
-    return m <= 4 ? 3 : m <= 6 ? 2 : 1;
-}
-inline size_t dense_w_smem(int B, int m) {
-    return (size_t)m * ((size_t)16 << B << dense_w_cshift(B, m)) +
-           (size_t)kDenseWarps * 2 * m * 32 * unit_bytes(B);
+// Shared memory of a writer CTA of nw warps: the staged books and each warp's two code buffers.
+inline size_t dense_w_smem(int B, int m, int nw) {
+    return (size_t)m * ((size_t)16 << B << book_copies_log2(B, m)) + (size_t)nw * 2 * m * 32 * unit_bytes(B);
 }
 
 template <int B, int BDT>
-__global__ void __launch_bounds__(kDenseWarps * 32, 1)
+__global__ void __launch_bounds__(kDenseMaxWarps * 32, 1)
 dense_w_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
                uint16_t* __restrict__ w16, float* __restrict__ wfac_out, int m, int cshift, int out,
                int in, int ng, int rows_pad, int RBc, int S, size_t plane_bytes) {
@@ -801,12 +786,12 @@ dense_w_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ 
     constexpr int NC = 1 << B;
     extern __shared__ __align__(16) unsigned char smem_d[];
     uint4* books_s = (uint4*)smem_d;                 // [m][NC][2^cshift] codewords
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (int)(blockDim.x >> 5);
     // this warp's code buffers: [2][m][32 rows][UNIT]
     unsigned char* cbuf = smem_d + ((size_t)m * NC << cshift) * 16 + (size_t)warp * 2 * m * 32 * UNIT;
     __shared__ unsigned int wmax[8];
     const long long items = (long long)RBc * S;
-    const long long stride = (long long)gridDim.x * kDenseWarps;
+    const long long stride = (long long)gridDim.x * nw;
     auto issue = [&](long long item, int buf) {   // the item's codes into buffer buf
         if (item < items) {
             const int s = (int)(item / RBc), rb = (int)(item - (long long)s * RBc);
@@ -821,7 +806,7 @@ dense_w_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ 
     };
     pdl_wait();
     pdl_launch_dependents();
-    long long item = (long long)blockIdx.x * kDenseWarps + warp;
+    long long item = (long long)blockIdx.x * nw + warp;
     issue(item, 0);   // the first codes travel while the books are staged
     // Books staged times 2^-f (fp16 range, as in the GEMM's decoders); 2^f goes to the
     // workspace for the GEMM's epilogue (every CTA finds the same f; CTA 0 writes it).
@@ -892,44 +877,58 @@ aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* b
                          const void* scales, const void* x, const float* xfac, int tokens, void* y,
                          int y_dt, void* ws, uint16_t* w16, cudaStream_t st) {   // x: fp16 [tokens][in]
     {   // decode W_m once
-        const size_t smem = dense_w_smem(B, m);
         auto kern = dense_w_kernel<B, BDT>;
         DeviceInfo di;
         if (aq_status e = device_info(&di); e != AQ_OK) return e;
-        // the kernel's shared-memory limit raised once per device, its occupancy per prefix
+        // the kernel's shared-memory limit raised once per device; per prefix the warps per CTA
+        // (16, 12, 8 or 4) with the most resident warps per SM
         static std::mutex mu_w;
-        static int occ_cache[64][kGemmMaxM + 1] = {};
+        static int dyn_max[64] = {};
+        static int choice[64][kGemmMaxM + 1][2] = {};   // [dev][m] -> {warps, CTAs per SM}
         int dev = 0;
         if (cudaError_t e = cudaGetDevice(&dev); e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
         if (dev < 0 || dev >= 64 || m < 1 || m > kGemmMaxM) return AQ_ERR_UNSUPPORTED;
-        int occ = 0;
+        int nw = 0, occ = 0;
         {
             std::lock_guard<std::mutex> lock(mu_w);
-            if (occ_cache[dev][m] == 0) {
+            if (dyn_max[dev] == 0) {
                 cudaFuncAttributes fa;
                 if (cudaError_t e = cudaFuncGetAttributes(&fa, kern); e != cudaSuccess)
                     return cuda_fail(e, "cudaFuncGetAttributes");
-                const int dyn_max = di.smem_optin - (int)fa.sharedSizeBytes;
-                if ((int)smem > dyn_max) return AQ_ERR_UNSUPPORTED;
-                if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn_max);
+                const int lim = di.smem_optin - (int)fa.sharedSizeBytes;
+                if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
                     e != cudaSuccess)
                     return cuda_fail(e, "cudaFuncSetAttribute");
-                int o = 0;
-                if (cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, kern, kDenseWarps * 32, smem);
-                    e != cudaSuccess)
-                    return cuda_fail(e, "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
-                if (o < 1) return AQ_ERR_UNSUPPORTED;
-                occ_cache[dev][m] = o;
+                dyn_max[dev] = lim;
             }
-            occ = occ_cache[dev][m];
+            if (choice[dev][m][0] == 0) {
+                int best_w = 0;
+                for (int w : {16, 12, 8, 4}) {
+                    const size_t sm_bytes = dense_w_smem(B, m, w);
+                    if (sm_bytes > (size_t)dyn_max[dev]) continue;
+                    int o = 0;
+                    if (cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, kern, w * 32, sm_bytes);
+                        e != cudaSuccess)
+                        return cuda_fail(e, "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
+                    if (o * w > best_w) {
+                        best_w = o * w;
+                        choice[dev][m][0] = w;
+                        choice[dev][m][1] = o;
+                    }
+                }
+                if (best_w == 0) return AQ_ERR_UNSUPPORTED;
+            }
+            nw = choice[dev][m][0];
+            occ = choice[dev][m][1];
         }
+        const size_t smem = dense_w_smem(B, m, nw);
         const long long items = (long long)d.RBc * d.S;
-        long long grid = (long long)di.sms * (occ > 0 ? occ : 1);
-        const long long need = (items + kDenseWarps - 1) / kDenseWarps;
+        long long grid = (long long)di.sms * occ;
+        const long long need = (items + nw - 1) / nw;
         if (grid > need) grid = need;
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3((unsigned)grid);
-        cfg.blockDim = dim3(kDenseWarps * 32);
+        cfg.blockDim = dim3(nw * 32);
         cfg.dynamicSmemBytes = smem;
         cfg.stream = st;
         cudaLaunchAttribute attr[1];
@@ -939,7 +938,7 @@ aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* b
         cfg.numAttrs = 1;
         if (aq_status e = cuda_ok(cudaLaunchKernelEx(&cfg, kern, (const uint8_t*)planes, (const uint16_t*)books,
                                                      w16, (float*)((char*)ws + kWsWfacOffset), m,
-                                                     dense_w_cshift(B, m), d.out, d.in, d.ng, d.rows_pad,
+                                                     book_copies_log2(B, m), d.out, d.in, d.ng, d.rows_pad,
                                                      d.RBc, d.S, d.plane_bytes),
                                   "cudaLaunchKernelEx (dense W_m)");
             e != AQ_OK)

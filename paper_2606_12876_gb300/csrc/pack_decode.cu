@@ -3,6 +3,8 @@
 // Packing turns the natural code tensor b (Sec. 3.2: one B-bit index per output row, group
 // of 8 inputs and codebook) into codebook-major planes so that a prefix of m codebooks
 // (Sec. 5) is a prefix of the buffer. Decoding writes the partial reconstruction W_m densely.
+#include <mutex>
+
 #include "aq_internal.cuh"
 
 namespace aq {
@@ -49,92 +51,185 @@ __global__ void pack4_kernel(const uint8_t* __restrict__ codes, uint8_t* __restr
     }
 }
 
-constexpr int kDecWarps = 8;
+constexpr int kDecMaxWarps = 16;
 
-// Decode: each warp owns one 32-row block of one slice. Lane L stages its own row's codes
-// for the m planes in shared memory, then the warp walks the 32 rows with lane L producing
-// group s*32+L of that row, so each output row segment is written as 512 contiguous bytes.
+// Decode: one CTA per SM (or as many as fit) walks the (32-row block, slice) items, a warp at a
+// time (grid-stride; row blocks fastest, so a warp's code loads are one contiguous 1 KiB per
+// plane for 8-bit codes and its stores 512 contiguous bytes per row). For B <= 8 the CTA stages
+// the first m codebooks once, in 2^cshift interleaved copies (book_copies_log2: with eight the
+// codeword gathers are free of bank conflicts); 16-bit codebooks are read through L2. Each
+// lane copies its row's codes of the m planes into the warp's staging buffer (cp.async), the
+// next item's while the current one is decoded; then lane L walks the rows, four at a time,
+// producing group s*32 + L of each.
 // Bit-exact contract (aq.h): fp32 adds in book order from +0.0f, one fp32 multiply by the
 // scale, one round-to-nearest-even to the book type.
 template <int B, int BDT, int SDT>
-__global__ void __launch_bounds__(kDecWarps * 32)
+__global__ void __launch_bounds__(kDecMaxWarps * 32, 1)
 decode_kernel(const uint8_t* __restrict__ planes, const uint16_t* __restrict__ books,
-              const uint16_t* __restrict__ scales, uint16_t* __restrict__ w, int m, int out,
-              int in, int ng, int rows_pad, int RBc, size_t plane_bytes) {
+              const uint16_t* __restrict__ scales, uint16_t* __restrict__ w, int m, int cshift,
+              int out, int in, int ng, int rows_pad, int RBc, int S, size_t plane_bytes) {
     constexpr int UNIT = unit_bytes(B);              // bytes of one (row, slice) unit
+    constexpr bool STAGED = B <= 8;
     extern __shared__ __align__(16) unsigned char smem[];
-    uint16_t* books_s = (uint16_t*)smem;             // B <= 8: [m][2^B][8]
-    const size_t books_bytes = staged_books_bytes(B, m);
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    unsigned char* codes_s = smem + books_bytes + (size_t)warp * m * 32 * UNIT;
-
-    if constexpr (B <= 8) {
-        const uint4* src = (const uint4*)books;
-        uint4* dst = (uint4*)books_s;
-        for (int i = threadIdx.x; i < (m << B); i += blockDim.x) dst[i] = src[i];
-    }
-    const int s = blockIdx.y;
-    const int rb = blockIdx.x * kDecWarps + warp;
-    const bool active = rb < RBc;
-    if (active) {
-        const int o = rb * 32 + lane;
-        for (int k = 0; k < m; ++k) {
-            const uint4* src =
-                (const uint4*)(planes + k * plane_bytes + ((size_t)s * rows_pad + o) * UNIT);
-            uint4* dst = (uint4*)(codes_s + ((size_t)k * 32 + lane) * UNIT);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (int)(blockDim.x >> 5);
+    const size_t books_bytes = STAGED ? ((size_t)m << B << cshift) * 16 : 0;   // [m][2^B][2^cshift]
+    unsigned char* cbuf = smem + books_bytes + (size_t)warp * 2 * m * 32 * UNIT;   // [2][m][32][UNIT]
+    const long long items = (long long)RBc * S;
+    const long long stride = (long long)gridDim.x * nw;
+    auto issue = [&](long long item, int buf) {   // the item's codes into buffer buf
+        if (item < items) {
+            const int s = (int)(item / RBc), rb = (int)(item - (long long)s * RBc);
+            const size_t src = ((size_t)s * rows_pad + (size_t)rb * 32 + lane) * UNIT;
+            unsigned char* dst = cbuf + ((size_t)buf * m * 32 + lane) * UNIT;
+            for (int k = 0; k < m; ++k)
 #pragma unroll
-            for (int q = 0; q < UNIT / 16; ++q) dst[q] = ld_stream_v4(src + q);
+                for (int q = 0; q < UNIT / 16; ++q)
+                    cp_async16(dst + (size_t)k * 32 * UNIT + q * 16, planes + k * plane_bytes + src + q * 16);
         }
+        cp_async_commit();
+    };
+    long long item = (long long)blockIdx.x * nw + warp;
+    issue(item, 0);   // the first codes travel while the books are staged
+    if constexpr (STAGED) {
+        uint4* dst = (uint4*)smem;
+        for (int i = threadIdx.x; i < (m << B) << cshift; i += blockDim.x)
+            dst[i] = __ldg((const uint4*)books + (i >> cshift));
     }
     __syncthreads();
-    if (!active) return;
-
-    const int g = s * 32 + lane;
-    for (int r = 0; r < 32; ++r) {
-        const int o = rb * 32 + r;
-        if (o >= out) break;
-        const float sc = bits_to_f32<SDT>(scales[o]);
-        const int p = (lane - r) & 31;               // position of group `lane` in row o
-        float acc[8];
+    const uint32_t books_u = smem_u32(smem) + ((uint32_t)(lane & ((1 << cshift) - 1)) << 4);
+    // lane L holds the scale of row 32 rb + L of an item; the next item's is requested one item
+    // ahead, with its codes
+    auto scale_of = [&](long long it) -> uint16_t {
+        if (it >= items) return 0;
+        const int row = (int)(it % RBc) * 32 + lane;
+        return row < out ? scales[row] : (uint16_t)0;
+    };
+    uint16_t sc_next = scale_of(item);
+    int buf = 0;
+    for (; item < items; item += stride) {
+        issue(item + stride, buf ^ 1);
+        const float sc_l = bits_to_f32<SDT>(sc_next);
+        sc_next = scale_of(item + stride);
+        const int s = (int)(item / RBc), rb = (int)(item - (long long)s * RBc);
+        const int g = s * 32 + lane;
+        cp_async_wait<1>();      // this lane's copies of the current item landed
+        __syncwarp();            // ... and every lane's
+        const unsigned char* cb = cbuf + (size_t)buf * m * 32 * UNIT;
+        {
+            // every lane computes (padding groups beyond ng have code 0); lanes g < ng store
+            for (int r0 = 0; r0 < 32 && rb * 32 + r0 < out; r0 += 4) {
+                float acc[4][8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) acc[e] = 0.0f;
-        for (int k = 0; k < m; ++k) {
-            const uint32_t code = unit_code<B>(codes_s + ((size_t)k * 32 + r) * UNIT, p);
-            uint4 cw;
-            if constexpr (B <= 8) cw = ((const uint4*)books_s)[(k << B) + code];
-            else cw = __ldg((const uint4*)books + ((size_t)k << 16) + code);
-            float c[8];
-            unpack8<BDT>(cw, c);
+                for (int i = 0; i < 4; ++i)
 #pragma unroll
-            for (int e = 0; e < 8; ++e) acc[e] = __fadd_rn(acc[e], c[e]);
-        }
-        if (g < ng) {
-            uint32_t pk[4];
+                    for (int e = 0; e < 8; ++e) acc[i][e] = 0.0f;
+                for (int k = 0; k < m; ++k) {
+                    uint4 cw[4];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const uint32_t lo = f32_to_bits<BDT>(__fmul_rn(acc[2 * i], sc));
-                const uint32_t hi = f32_to_bits<BDT>(__fmul_rn(acc[2 * i + 1], sc));
-                pk[i] = lo | (hi << 16);
+                    for (int i = 0; i < 4; ++i) {
+                        const int r = r0 + i;
+                        // position of group `lane` in row rb*32 + r
+                        const uint32_t code = unit_code<B>(cb + ((size_t)k * 32 + r) * UNIT, (lane - r) & 31);
+                        if constexpr (STAGED)
+                            cw[i] = lds128(books_u + ((((uint32_t)k << B) + code) << (cshift + 4)));
+                        else
+                            cw[i] = __ldg((const uint4*)books + ((size_t)k << 16) + code);
+                    }
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {   // exact widening, one fp32 rounding per add
+                        add_widen2<BDT>(cw[i].x, acc[i][0], acc[i][1]);
+                        add_widen2<BDT>(cw[i].y, acc[i][2], acc[i][3]);
+                        add_widen2<BDT>(cw[i].z, acc[i][4], acc[i][5]);
+                        add_widen2<BDT>(cw[i].w, acc[i][6], acc[i][7]);
+                    }
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int o = rb * 32 + r0 + i;
+                    const float sc = __shfl_sync(0xffffffffu, sc_l, r0 + i);
+                    if (o < out && g < ng) {
+                        // times the scale (a packed fma with -0.0 added: the rounded product,
+                        // signed zeros included), then one rounding to the book type per value
+                        uint32_t pk[4];
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const float2 v = ffma2(make_float2(acc[i][2 * j], acc[i][2 * j + 1]),
+                                                   make_float2(sc, sc), make_float2(-0.0f, -0.0f));
+                            pk[j] = round_pack2<BDT>(v.x, v.y);
+                        }
+                        *(uint4*)(w + (size_t)o * in + (size_t)g * 8) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                    }
+                }
             }
-            *(uint4*)(w + (size_t)o * in + (size_t)g * 8) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
         }
+        __syncwarp();            // every lane has read the buffer before it is refilled
+        buf ^= 1;
     }
+    cp_async_wait<0>();
 }
 
 template <int B, int BDT, int SDT>
 aq_status run_decode(const Dims& d, int m, const void* planes, const void* books,
                      const void* scales, void* w, cudaStream_t st) {
-    const size_t smem = staged_books_bytes(B, m) + (size_t)kDecWarps * m * 32 * unit_bytes(B);
     auto kern = decode_kernel<B, BDT, SDT>;
-    if (smem > 48 * 1024)
-        if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)smem);
-            e != cudaSuccess)
-            return cuda_fail(e, "cudaFuncSetAttribute");
-    dim3 grid((d.RBc + kDecWarps - 1) / kDecWarps, d.S);
-    kern<<<grid, kDecWarps * 32, smem, st>>>((const uint8_t*)planes, (const uint16_t*)books,
-                                             (const uint16_t*)scales, (uint16_t*)w, m, d.out,
-                                             d.in, d.ng, d.rows_pad, d.RBc, d.plane_bytes);
+    DeviceInfo di;
+    if (aq_status e = device_info(&di); e != AQ_OK) return e;
+    // the kernel's shared-memory limit raised once per device (the attribute is per kernel)
+    static std::mutex mu;
+    static int dyn_max[64] = {};
+    int dev = 0;
+    if (cudaError_t e = cudaGetDevice(&dev); e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= 64) return AQ_ERR_UNSUPPORTED;
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        if (dyn_max[dev] == 0) {
+            cudaFuncAttributes fa;
+            if (cudaError_t e = cudaFuncGetAttributes(&fa, kern); e != cudaSuccess)
+                return cuda_fail(e, "cudaFuncGetAttributes");
+            const int lim = di.smem_optin - (int)fa.sharedSizeBytes;
+            if (cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
+                e != cudaSuccess)
+                return cuda_fail(e, "cudaFuncSetAttribute");
+            dyn_max[dev] = lim;
+        }
+    }
+    const int cshift = B <= 8 ? book_copies_log2(B, m) : 0;
+    const size_t books_bytes = B <= 8 ? ((size_t)m << B << cshift) * 16 : 0;
+    const size_t per_warp = (size_t)2 * m * 32 * unit_bytes(B);
+    // warps per CTA: the choice (16, 12, 8 or 4) with the most resident warps per SM (the
+    // code buffers are per warp), found once per device and prefix
+    static int choice[64][9][2] = {};   // [dev][m] -> {warps, CTAs per SM}
+    int nw = 0, occ = 0;
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        if (choice[dev][m][0] == 0) {
+            int best_w = 0;
+            for (int w : {16, 12, 8, 4}) {
+                const size_t sm_bytes = books_bytes + w * per_warp;
+                if (sm_bytes > (size_t)dyn_max[dev]) continue;
+                int o = 0;
+                if (cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, kern, w * 32, sm_bytes);
+                    e != cudaSuccess)
+                    return cuda_fail(e, "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
+                if (o * w > best_w) {
+                    best_w = o * w;
+                    choice[dev][m][0] = w;
+                    choice[dev][m][1] = o;
+                }
+            }
+            if (best_w == 0) return AQ_ERR_UNSUPPORTED;
+        }
+        nw = choice[dev][m][0];
+        occ = choice[dev][m][1];
+    }
+    const size_t smem = books_bytes + nw * per_warp;
+    const long long items = (long long)d.RBc * d.S;
+    long long grid = (long long)di.sms * occ;
+    const long long need = (items + nw - 1) / nw;
+    if (grid > need) grid = need;
+    kern<<<(unsigned)grid, nw * 32, smem, st>>>((const uint8_t*)planes, (const uint16_t*)books,
+                                                (const uint16_t*)scales, (uint16_t*)w, m, cshift, d.out,
+                                                d.in, d.ng, d.rows_pad, d.RBc, d.S, d.plane_bytes);
     return cuda_ok(cudaGetLastError(), "kernel launch");
 }
 
