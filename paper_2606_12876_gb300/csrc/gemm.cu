@@ -93,6 +93,8 @@ struct GemmLayout {
     // 1024-byte boundary (checked at run time: the 128-byte swizzled tiles need it).
     static constexpr int kSmem = kOffWmax + 32;
     static_assert(kSmem <= 227 * 1024, "shared memory map exceeds the per-CTA limit");
+    // the epilogue's 16-bit staging (eight warps x 32 tokens x 256 rows) reuses the operand rings
+    static_assert(kOffCodes - kOffA >= kDecWarps * 32 * kBN * 2, "operand rings too small for y staging");
 };
 
 __device__ __forceinline__ uint32_t pack2(float lo, float hi, int dt) {
@@ -200,7 +202,7 @@ __device__ __forceinline__ uint4 decode_group(uint32_t books, const uint32_t (&c
 template <int BDT, int MB, int NP, bool DENSE = false>
 __global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
-            const uint8_t* __restrict__ planes,
+            const __grid_constant__ CUtensorMap ymap, int y_tma, const uint8_t* __restrict__ planes,
             const uint16_t* __restrict__ books, const uint16_t* __restrict__ scales, void* y,
             int y_dt, int scale_dt, unsigned int* __restrict__ status,
             const float* __restrict__ xfac, int tokens, int out, int in, int ng, int rows_pad,
@@ -559,7 +561,45 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
         // Vector stores need 16-byte aligned row segments: out a multiple of 8 (the output
         // pointer itself is 16-byte aligned by contract).
         const bool vec = (out & 7) == 0;
-        if (ready) {
+        if (ready && y_tma) {
+            // 16-bit y by TMA stores: every MMA has completed, so the operand rings are free;
+            // each warp stages its 32 tokens x 256 rows as eight 32 x 32 chunks (2 KiB each, a
+            // token's 64 bytes per row of the chunk, 16-byte pieces placed by the 64-byte
+            // swizzle of the store's tensor map: piece j of token row r at j ^ ((r >> 1) & 3),
+            // conflict-free) and stores each chunk with one bulk tensor store.
+            const int q = warp & 3;                       // tensor-memory lane quarter
+            const int i = (warp - kDecWarp0) >> 2;        // token block (accumulator)
+            const int tw = t0 + i * 2 * kBM + (int)rank * kBM + q * 32;   // the warp's first token
+            const int t = tw + lane;
+            const float xf = (xfac && t < tokens) ? xfac[t] : 1.0f;   // 2^e_t (bf16 activations)
+            const uint32_t stage = smem_u32(smem + kOffA) + (uint32_t)(warp - kDecWarp0) * (kBN / 32) * 2048u;
+            const uint32_t sw = (uint32_t)(lane >> 1) & 3u;
+            for (int nc = 0; nc < kBN; nc += 32) {
+                float v[32];
+                tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + i * kBN + nc, v);
+                if (xf != 1.0f)
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) v[e] *= xf;   // exact: a power of two
+                const uint32_t chunk = stage + (uint32_t)(nc / 32) * 2048u;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const int e = 8 * j;
+                    sts128(chunk + (uint32_t)lane * 64u + (((uint32_t)j ^ sw) << 4),
+                           make_uint4(pack2(v[e] * scale_s[nc + e], v[e + 1] * scale_s[nc + e + 1], y_dt),
+                                      pack2(v[e + 2] * scale_s[nc + e + 2], v[e + 3] * scale_s[nc + e + 3], y_dt),
+                                      pack2(v[e + 4] * scale_s[nc + e + 4], v[e + 5] * scale_s[nc + e + 5], y_dt),
+                                      pack2(v[e + 6] * scale_s[nc + e + 6], v[e + 7] * scale_s[nc + e + 7], y_dt)));
+                }
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                __syncwarp();
+                if (lane == 0 && tw < tokens && n0 + nc < out) tma_store_2d(&ymap, n0 + nc, tw, chunk);
+            }
+            if (lane == 0) {   // the staged chunks are read before the CTA leaves
+                bulk_commit();
+                bulk_wait_read_all();
+            }
+            __syncwarp();
+        } else if (ready) {
             const int q = warp & 3;                       // tensor-memory lane quarter
             const int i = (warp - kDecWarp0) >> 2;        // token block (accumulator)
             const int t = t0 + i * 2 * kBM + (int)rank * kBM + q * 32 + lane;
@@ -679,6 +719,27 @@ int gemm_pairs_per_cluster(int m, int tokens) {
     return m >= 2 && tokens > kPairTokens ? 2 : 1;
 }
 
+// Tensor map of a 16-bit y [tokens][out] for the epilogue's bulk stores: 32 x 32 boxes, 64-byte
+// swizzle. *use = 0 (the per-thread stores) for fp32 y or rows that are not a multiple of 16
+// bytes long.
+aq_status make_y_map(CUtensorMap* map, int* use, void* y, int y_dt, int out, int tokens) {
+    std::memset(map, 0, sizeof(*map));
+    *use = 0;
+    if (y_dt == AQ_F32 || (out & 7) != 0 || ((uintptr_t)y & 15u) != 0) return AQ_OK;
+    EncodeTiledFn encode;
+    if (aq_status e = get_encode_fn(&encode); e != AQ_OK) return e;
+    const cuuint64_t dims[2] = {(cuuint64_t)out, (cuuint64_t)tokens};
+    const cuuint64_t strides[1] = {(cuuint64_t)out * 2};
+    const cuuint32_t box[2] = {32, 32};
+    const cuuint32_t estr[2] = {1, 1};
+    if (encode(map, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, y, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return AQ_ERR_CUDA;
+    *use = 1;
+    return AQ_OK;
+}
+
 template <int BDT>
 aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
                    const void* scales, const void* x, const float* xfac, int tokens, void* y,
@@ -699,7 +760,8 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
     // Pairs per cluster sharing the decode: sharing pays where the gathers bound the kernel
     // (m >= 2) and every pair of a cluster has tokens (one 512-token tile per pair).
     const int np = gemm_pairs_per_cluster(m, tokens);
-    using Kern = void (*)(const CUtensorMap, const CUtensorMap, const uint8_t*, const uint16_t*, const uint16_t*,
+    using Kern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, int, const uint8_t*,
+                          const uint16_t*, const uint16_t*,
                           void*, int, int, unsigned int*, const float*, int, int, int, int, int, size_t);
     const Kern k1[kGemmMaxM] = {gemm_kernel<BDT, 1, 1>, gemm_kernel<BDT, 2, 1>, gemm_kernel<BDT, 3, 1>,
                                 gemm_kernel<BDT, 4, 1>, gemm_kernel<BDT, 5, 1>, gemm_kernel<BDT, 6, 1>,
@@ -749,7 +811,10 @@ aq_status run_gemm(const Dims& d, int m, const void* planes, const void* books,
     cfg.numAttrs = 2;
     CUtensorMap unused;                 // the weight map is read only by the dense variant
     std::memset(&unused, 0, sizeof(unused));
-    return cuda_ok(cudaLaunchKernelEx(&cfg, kern, map, unused, (const uint8_t*)planes,
+    CUtensorMap ym;
+    int y_tma = 0;
+    if (aq_status e = make_y_map(&ym, &y_tma, y, y_dt, d.out, tokens); e != AQ_OK) return e;
+    return cuda_ok(cudaLaunchKernelEx(&cfg, kern, map, unused, ym, y_tma, (const uint8_t*)planes,
                                       (const uint16_t*)books, (const uint16_t*)scales, y, y_dt,
                                       d.scale_dt, (unsigned int*)ws, xfac, tokens, d.out, d.in, d.ng,
                                       d.rows_pad, d.plane_bytes),
@@ -996,7 +1061,10 @@ aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* b
     attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    return cuda_ok(cudaLaunchKernelEx(&cfg, kern, xm, wm, (const uint8_t*)planes, (const uint16_t*)books,
+    CUtensorMap ym;
+    int y_tma = 0;
+    if (aq_status e = make_y_map(&ym, &y_tma, y, y_dt, d.out, tokens); e != AQ_OK) return e;
+    return cuda_ok(cudaLaunchKernelEx(&cfg, kern, xm, wm, ym, y_tma, (const uint8_t*)planes, (const uint16_t*)books,
                                       (const uint16_t*)scales, y, y_dt, d.scale_dt, (unsigned int*)ws,
                                       xfac, tokens, d.out, d.in, d.ng, d.rows_pad, d.plane_bytes),
                    "cudaLaunchKernelEx (dense GEMM)");
