@@ -946,7 +946,7 @@ aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* b
         DeviceInfo di;
         if (aq_status e = device_info(&di); e != AQ_OK) return e;
         // the kernel's shared-memory limit raised once per device; per prefix the warps per CTA
-        // (16, 12, 8 or 4) with the most resident warps per SM
+        // (16, 12, 8, 6 or 4) with the most resident warps per SM
         static std::mutex mu_w;
         static int dyn_max[64] = {};
         static int choice[64][kGemmMaxM + 1][2] = {};   // [dev][m] -> {warps, CTAs per SM}
@@ -968,7 +968,7 @@ aq_status run_gemm_dense(const Dims& d, int m, const void* planes, const void* b
             }
             if (choice[dev][m][0] == 0) {
                 int best_w = 0;
-                for (int w : {16, 12, 8, 4}) {
+                for (int w : {16, 12, 8, 6, 4}) {
                     const size_t sm_bytes = dense_w_smem(B, m, w);
                     if (sm_bytes > (size_t)dyn_max[dev]) continue;
                     int o = 0;

@@ -196,7 +196,7 @@ aq_status run_decode(const Dims& d, int m, const void* planes, const void* books
     const int cshift = B <= 8 ? book_copies_log2(B, m) : 0;
     const size_t books_bytes = B <= 8 ? ((size_t)m << B << cshift) * 16 : 0;
     const size_t per_warp = (size_t)2 * m * 32 * unit_bytes(B);
-    // warps per CTA: the choice (16, 12, 8 or 4) with the most resident warps per SM (the
+    // warps per CTA: the choice (16, 12, 8, 6 or 4) with the most resident warps per SM (the
     // code buffers are per warp), found once per device and prefix
     static int choice[64][9][2] = {};   // [dev][m] -> {warps, CTAs per SM}
     int nw = 0, occ = 0;
@@ -204,7 +204,7 @@ aq_status run_decode(const Dims& d, int m, const void* planes, const void* books
         std::lock_guard<std::mutex> lock(mu);
         if (choice[dev][m][0] == 0) {
             int best_w = 0;
-            for (int w : {16, 12, 8, 4}) {
+            for (int w : {16, 12, 8, 6, 4}) {
                 const size_t sm_bytes = books_bytes + w * per_warp;
                 if (sm_bytes > (size_t)dyn_max[dev]) continue;
                 int o = 0;

@@ -28,6 +28,7 @@ RAGGED = [  # out, in, M, B, book dtype
     (33, 2056, 2, 8, "f16"), (50, 136, 2, 16, "f16"), (70, 520, 3, 16, "bf16"),
     (257, 1032, 4, 8, "f16"), (60, 1032, 8, 8, "f16"), (45, 264, 5, 8, "bf16"),
     (37, 560, 3, 4, "f16"), (100, 264, 4, 4, "bf16"),
+    (40, 264, 8, 16, "f16"), (33, 520, 8, 4, "bf16"),
 ]
 
 
