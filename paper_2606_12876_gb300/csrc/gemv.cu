@@ -1355,11 +1355,24 @@ aq_status run_lut_layers(const Dims* ds, const GemvArgs* as, int n, int m, cudaS
     // waits for its slowest CTA, so the choice takes the smaller worst-CTA cost, one table
     // build being worth kTableItems row blocks of streaming (about 0.8 us against 23 ns per
     // 1 KiB block at the per-SM share of HBM bandwidth). A group always takes the even split.
+    // In the whole-share form a grid of more than kLutCpuMaxCtas CTAs costs about 0.6 us more
+    // (kGridItems / NT row blocks of NT-token lookups): one CTA on each of 144 SMs measured
+    // slower than 128 or 96 CTAs with larger shares (4096 x 4096 at m = 3: 6.60 against
+    // 5.85 us with two CTAs per unit; 14336 x 4096 at m = 1: 6.33 against 5.55 us with
+    // eight), unless the larger shares cost more (14336 x 4096 at m = 3: 10.17 against
+    // 11.19 us; four tokens, 4096 x 4096 at m = 3: 10.7 against 12.2 us).
     constexpr long long kTableItems = 35;
-    long long cpu = n == 1 ? di.sms / units : 0;
-    if (cpu > d.RBc) cpu = d.RBc;
-    long long cost_cpu = -1;
-    if (cpu >= 1) cost_cpu = kTableItems + (d.RBc + cpu - 1) / cpu;
+    constexpr long long kLutCpuMaxCtas = 128, kGridItems = 25;
+    long long cpu = 0, cost_cpu = -1;
+    if (n == 1)
+        for (long long c = 1; c * units <= di.sms && c <= d.RBc; ++c) {
+            const long long cost = kTableItems + (d.RBc + c - 1) / c +
+                                   (c * units > kLutCpuMaxCtas ? kGridItems / NT : 0);
+            if (cost_cpu < 0 || cost < cost_cpu) {
+                cost_cpu = cost;
+                cpu = c;
+            }
+        }
     const long long grid_b = items < di.sms ? items : di.sms;
     const long long qb = items / grid_b, rb = items % grid_b;
     long long cost_b = 0;
