@@ -49,11 +49,16 @@ def test_gemm_matches_oracle(case, y_dtype):
         U.assert_product_close(U.to_f64(y), oracle.product_exact(layer, xb, dt, m), "m=%d" % m)
 
 
-@pytest.mark.parametrize("case", [(2100, 300, 520, 5, "bf16"), (2048, 256, 1032, 3, "f16")],
+@pytest.mark.parametrize("case", [(2100, 300, 520, 5, "bf16"), (2048, 256, 1032, 3, "f16"),
+                                  (2090, 1288, 520, 2, "bf16")],
                          ids=lambda c: "x".join(map(str, c)))
-def test_gemm_dense_path_long_inputs(case):
+@pytest.mark.parametrize("y_dtype", [aq.AQ_F32, aq.AQ_BF16, aq.AQ_F16])
+def test_gemm_dense_path_long_inputs(case, y_dtype):
     """From 2048 tokens, prefixes of two or more books decode W_m once into the workspace
-    (fp16) and run TMA-fed pair MMAs on it: every prefix within the product tolerance."""
+    (fp16) and run TMA-fed pair MMAs on it: every prefix within the product tolerance. A
+    16-bit y whose rows are a multiple of 16 bytes is written by bulk tensor stores from the
+    operand rings (partial 32 x 32 chunks at a ragged row or token edge: 1288 rows, 2090
+    tokens); 300 rows take the per-thread stores."""
     tok, out, inp, M, dt = case
     layer = workloads.make_layer(out, inp, G=8, M=M, B=8, book_dtype=dt, book_std=0.05,
                                  scale_dtype=dt, seed=tok + M)
@@ -62,21 +67,23 @@ def test_gemm_dense_path_long_inputs(case):
     x = x_to_device(xb, dt)
     rows = np.r_[0:64, tok // 2:tok // 2 + 64, tok - 64:tok]
     for m in range(1, M + 1):
-        y = lin.gemm(x, m, y_dtype=aq.AQ_F32)
+        y = lin.gemm(x, m, y_dtype=y_dtype)
         ys = U.to_f64(y[torch.as_tensor(rows, device="cuda")])
         U.assert_product_close(ys, oracle.product_exact(layer, xb[rows], dt, m), "m=%d" % m)
 
 
-@pytest.mark.parametrize("tok", [40, 700])
-def test_gemm_4bit_codes(tok):
-    """4-bit codes (16-entry codebooks): W_m decoded into the workspace, then the pair MMAs."""
-    layer = workloads.make_layer(300, 520, G=8, M=4, B=4, book_dtype="bf16", book_std=0.05,
+@pytest.mark.parametrize("tok,out,y_dtype", [(40, 300, aq.AQ_F32), (700, 300, aq.AQ_F32),
+                                             (700, 296, aq.AQ_BF16)])
+def test_gemm_4bit_codes(tok, out, y_dtype):
+    """4-bit codes (16-entry codebooks): W_m decoded into the workspace, then the pair MMAs
+    (with a bf16 y of 296 rows: the bulk-store epilogue)."""
+    layer = workloads.make_layer(out, 520, G=8, M=4, B=4, book_dtype="bf16", book_std=0.05,
                                  scale_dtype="bf16", seed=tok)
     lin = AQLinear.from_layer(layer)
     xb = workloads.make_x(tok, 520, "bf16", seed=9)
     x = x_to_device(xb, "bf16")
     for m in range(1, 5):
-        y = lin.gemm(x, m, y_dtype=aq.AQ_F32)
+        y = lin.gemm(x, m, y_dtype=y_dtype)
         U.assert_product_close(U.to_f64(y), oracle.product_exact(layer, xb, "bf16", m), "m=%d" % m)
 
 
