@@ -31,7 +31,8 @@
 //               sums the m codewords in fp32 (book order), rounds once to fp16 and writes the
 //               16-byte group into the B tile in the UMMA K-major 128-byte-swizzle layout.
 //               Afterwards the same warps are the epilogue: tcgen05.ld from tensor memory,
-//               times the row scale (R1), round, store.
+//               times the row scale (R1), round; a 16-bit y is staged in the freed operand
+//               rings and written by bulk tensor stores (per-thread stores otherwise).
 // Operands are fp16 (kind::f16, fp32 accumulation): the summed weights are rounded once to
 // fp16 (about 2^-11 relative), which keeps the product inside the stated per-element bound;
 // bf16 activations are first converted to fp16 into the workspace (exact for normal-range
